@@ -1,0 +1,164 @@
+"""fp64 CPU oracle for Flexformer random-Fourier-feature linear attention.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU
+baseline leg of ``bench.py`` may import this package.  The product path (the CUDA library
+and its Python binding) never imports, links or executes anything here, and this package
+imports nothing from the product path.
+
+Contents
+  * ``flex_oracle.c`` -- the linear form (Sec. 2.2, Eq. linear att) with the stationary
+    (Eq. phi_n, Flexformer_s) and nonstationary (Eq. phi_non, Flexformer_n) feature maps,
+    forward and analytic backward, in plain fp64 C loops.  Loaded here through ctypes.
+  * ``brute.py`` -- the explicit N x N kernel-matrix form of Eq. (attention) with
+    sim(q, k) = phi(q) . phi(k) (Eq. kernel), written independently in numpy.
+
+Every function takes and returns float64 numpy arrays in the layouts
+q, k, v, out: [B, H, N, d];  W1, W2: [H, M, d];  den: [B, H, N];  phi: [B, H, N, 2M].
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+SOURCE = os.path.join(_HERE, "flex_oracle.c")
+BUILD_DIR = os.path.join(_HERE, "_build")
+LIBRARY = os.path.join(BUILD_DIR, "libflex_oracle.so")
+
+_lock = threading.Lock()
+_lib = None
+
+
+def compile_library(source_text: str | None = None, out_path: str = LIBRARY) -> str:
+    """Compile the C oracle (or a modified copy of its source text) into a shared library.
+
+    Plain gcc, -O2, no fast-math: the oracle keeps IEEE fp64 semantics.
+    """
+    os.makedirs(os.path.dirname(out_path), exist_ok=True)
+    src = SOURCE
+    if source_text is not None:
+        src = out_path[:-3] + ".c"
+        with open(src, "w") as f:
+            f.write(source_text)
+    tmp = out_path + f".tmp{os.getpid()}"
+    subprocess.run(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-pthread", src, "-o", tmp,
+                    "-lm"], check=True)
+    os.replace(tmp, out_path)
+    return out_path
+
+
+def _stale() -> bool:
+    return (not os.path.exists(LIBRARY)
+            or os.path.getmtime(LIBRARY) < os.path.getmtime(SOURCE))
+
+
+class Oracle:
+    """ctypes view of one compiled copy of ``flex_oracle.c``."""
+
+    def __init__(self, path: str):
+        lib = ctypes.CDLL(path)
+        dp = ctypes.POINTER(ctypes.c_double)
+        i = ctypes.c_int
+        lib.oracle_featmap.argtypes = [i, i, i, i, i, dp, dp, dp, dp]
+        lib.oracle_featmap_sumform.argtypes = [i, i, i, i, i, dp, dp, dp, dp]
+        lib.oracle_linattn_fwd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, i, dp, dp, i]
+        lib.oracle_linattn_bwd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, i, dp, dp, dp,
+                                           dp, dp, dp, i]
+        for fn in (lib.oracle_featmap, lib.oracle_featmap_sumform, lib.oracle_linattn_fwd,
+                   lib.oracle_linattn_bwd):
+            fn.restype = ctypes.c_int
+        self._lib = lib
+        self.path = path
+
+    @staticmethod
+    def _p(a):
+        if a is None:
+            return None
+        return a.ctypes.data_as(ctypes.POINTER(ctypes.c_double))
+
+    @staticmethod
+    def _f64(a):
+        return None if a is None else np.ascontiguousarray(a, dtype=np.float64)
+
+    def featmap(self, x, W1, W2=None):
+        """phi(x) for x [B, H, N, d] with per-head frequencies [H, M, d] -> [B, H, N, 2M]."""
+        x, W1, W2 = self._f64(x), self._f64(W1), self._f64(W2)
+        B, H, N, d = x.shape
+        M = W1.shape[1]
+        phi = np.empty((B, H, N, 2 * M))
+        rc = self._lib.oracle_featmap(B, H, N, d, M, self._p(x), self._p(W1), self._p(W2),
+                                      self._p(phi))
+        if rc != 0:
+            raise ValueError("oracle_featmap: bad shape")
+        return phi
+
+    def featmap_sumform(self, x, W1, W2):
+        """Nonstationary phi(x) in the unsimplified Monte Carlo form of Eq. (phi_non)."""
+        x, W1, W2 = self._f64(x), self._f64(W1), self._f64(W2)
+        B, H, N, d = x.shape
+        M = W1.shape[1]
+        phi = np.empty((B, H, N, 2 * M))
+        rc = self._lib.oracle_featmap_sumform(B, H, N, d, M, self._p(x), self._p(W1),
+                                              self._p(W2), self._p(phi))
+        if rc != 0:
+            raise ValueError("oracle_featmap_sumform: bad shape")
+        return phi
+
+    def fwd(self, q, k, v, W1, W2=None, causal=True, nthreads=None):
+        """(out [B, H, N, d], den [B, H, N]) of Eq. (linear att)."""
+        q, k, v, W1, W2 = (self._f64(a) for a in (q, k, v, W1, W2))
+        B, H, N, d = q.shape
+        M = W1.shape[1]
+        out = np.empty_like(q)
+        den = np.empty((B, H, N))
+        nt = nthreads or os.cpu_count() or 1
+        rc = self._lib.oracle_linattn_fwd(B, H, N, d, M, self._p(q), self._p(k), self._p(v),
+                                          self._p(W1), self._p(W2), int(bool(causal)),
+                                          self._p(out), self._p(den), nt)
+        if rc != 0:
+            raise ValueError("oracle_linattn_fwd: bad shape")
+        return out, den
+
+    def bwd(self, q, k, v, W1, W2, causal, dout, nthreads=None):
+        """Gradients (dq, dk, dv, dW1, dW2) of L = sum(dout * out); dW2 is None if W2 is."""
+        q, k, v, W1, W2, dout = (self._f64(a) for a in (q, k, v, W1, W2, dout))
+        B, H, N, d = q.shape
+        M = W1.shape[1]
+        dq, dk, dv = np.empty_like(q), np.empty_like(q), np.empty_like(q)
+        dW1 = np.empty_like(W1)
+        dW2 = None if W2 is None else np.empty_like(W2)
+        nt = nthreads or os.cpu_count() or 1
+        rc = self._lib.oracle_linattn_bwd(B, H, N, d, M, self._p(q), self._p(k), self._p(v),
+                                          self._p(W1), self._p(W2), int(bool(causal)),
+                                          self._p(dout), self._p(dq), self._p(dk),
+                                          self._p(dv), self._p(dW1), self._p(dW2), nt)
+        if rc != 0:
+            raise ValueError("oracle_linattn_bwd: bad shape")
+        return dq, dk, dv, dW1, dW2
+
+
+def load() -> Oracle:
+    """The oracle built from ``flex_oracle.c`` (compiled on first use if needed)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if _stale():
+                compile_library()
+            _lib = Oracle(LIBRARY)
+        return _lib
+
+
+def featmap(x, W1, W2=None):
+    return load().featmap(x, W1, W2)
+
+
+def fwd(q, k, v, W1, W2=None, causal=True, nthreads=None):
+    return load().fwd(q, k, v, W1, W2, causal, nthreads)
+
+
+def bwd(q, k, v, W1, W2, causal, dout, nthreads=None):
+    return load().bwd(q, k, v, W1, W2, causal, dout, nthreads)

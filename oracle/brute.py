@@ -1,0 +1,49 @@
+"""Explicit N x N form of kernel attention, in numpy fp64.
+
+TEST INFRASTRUCTURE ONLY (see the package docstring).  This module is written separately
+from ``flex_oracle.c`` and with a different structure, so that the two can be checked
+against each other:
+
+  * the features of Flexformer_n are taken in the Monte Carlo sum form of Eq. (phi_non),
+    (cos w_1i.x + cos w_2i.x, sin w_1i.x + sin w_2i.x) / (2 sqrt M), not in the
+    product form that the C oracle uses;
+  * attention is Eq. (attention) with sim(q_i, k_j) = phi(q_i) . phi(k_j) (Eq. kernel):
+    the full N x N weight matrix is built, masked to j <= i when causal, and each row is
+    divided by its sum -- no reassociation.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def features(x, W1, W2=None):
+    """phi(x) for x [..., H, N, d] and frequencies [H, M, d] -> [..., H, N, 2M].
+
+    Stationary: M^{-1/2} [cos(x W1^T), sin(x W1^T)]  (Eq. phi_n with sigma = 1).
+    Nonstationary: (2 sqrt M)^{-1} [cos a + cos b, sin a + sin b], a = x W1^T, b = x W2^T.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    W1 = np.asarray(W1, dtype=np.float64)
+    M = W1.shape[1]
+    a = np.einsum("...hnd,hmd->...hnm", x, W1)
+    if W2 is None:
+        return np.concatenate([np.cos(a), np.sin(a)], axis=-1) / np.sqrt(M)
+    b = np.einsum("...hnd,hmd->...hnm", x, np.asarray(W2, dtype=np.float64))
+    return np.concatenate([np.cos(a) + np.cos(b), np.sin(a) + np.sin(b)], axis=-1) / (
+        2.0 * np.sqrt(M))
+
+
+def kernel_matrix(q, k, W1, W2=None):
+    """K[..., i, j] = phi(q_i) . phi(k_j)."""
+    return np.einsum("...if,...jf->...ij", features(q, W1, W2), features(k, W1, W2))
+
+
+def attention(q, k, v, W1, W2=None, causal=True):
+    """(out, den): out_i = sum_j K_ij v_j / sum_j K_ij over j <= i (causal) or all j."""
+    K = kernel_matrix(q, k, W1, W2)
+    if causal:
+        N = K.shape[-1]
+        K = K * np.tril(np.ones((N, N)))
+    den = K.sum(axis=-1)
+    out = np.einsum("...ij,...je->...ie", K, np.asarray(v, dtype=np.float64)) / den[..., None]
+    return out, den

@@ -1,0 +1,409 @@
+/*
+ * flex_oracle.c -- plain, slow, fp64 CPU oracle for Flexformer's random-Fourier-feature
+ * linear attention (stationary and nonstationary variants), forward and backward.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the test suite, the smoke check and the bench's CPU
+ * baseline may load this library.  It shares no code, header or constant with the CUDA
+ * path; it is written directly from the paper's equations:
+ *
+ *   Sec. 2.2, Eq. (kernel) / Eq. (linear att):
+ *       O_i = phi(Q_i)^T sum_j phi(K_j) V_j^T  /  phi(Q_i)^T sum_j phi(K_j)
+ *   Sec. 3.1, Eq. (phi_n):    stationary random Fourier features
+ *       phi(x) = sigma/sqrt(n) [cos w_1.x .. cos w_n.x, sin w_1.x .. sin w_n.x]
+ *   Sec. 3.2, Flexformer_s:   the frequencies w_i are the learnable matrix W1 (n = M rows)
+ *   Sec. 3.2, Eq. (phi_non):  nonstationary (Yaglom) features with frequency pairs (W1, W2)
+ *       w'_1i = (w_1i + w_2i)/2,  w'_2i = (w_1i - w_2i)/2
+ *       phi(x) = c [cos w'_1i.x cos w'_2i.x ..., sin w'_1i.x cos w'_2i.x ...]
+ *
+ * Readings taken where the paper is silent or garbled (each is listed in the design notes):
+ *   - scale: sigma = 1 and c = M^{-1/2} for both variants.  The printed nonstationary
+ *     constant sigma/(2 sqrt n) drops the factor 4 that the sum-to-product step produces;
+ *     M^{-1/2} is the value that makes the last two lines of Eq. (phi_non) agree.
+ *     Any global scale cancels in O and in every gradient.
+ *   - causal attention sums over j <= i (the diagonal is included).
+ *   - the denominator is used as it is: no epsilon, no clamp.
+ *   - the learned parameters of Flexformer_n are (W1, W2); dW1 and dW2 are returned.
+ *   - the norm prefactor exp(|x|^2 / exp(tau)) is not part of this path.
+ *
+ * The backward pass is the analytic gradient of L = sum_i dO_i . O_i, derived by hand
+ * from Eq. (linear att) (the paper gives none; it only states that the frequencies are
+ * trained end to end):
+ *   g_i = dO_i / den_i,  c_i = -(dO_i . O_i) / den_i
+ *   dphi(q_i) = S_i g_i + c_i z_i           (S_i, z_i: running sums over j <= i)
+ *   dphi(k_j) = R_j v_j + r_j               (R_j = sum_{i>=j} phi(q_i) g_i^T, r_j = sum c_i phi(q_i))
+ *   dv_j      = R_j^T phi(k_j)
+ * and through the feature map by the chain rule.  For non-causal attention every
+ * running sum is replaced by the total.
+ *
+ * Layouts: q, k, v, out, dout, dq, dk, dv are [B][H][N][d]; W1, W2, dW1, dW2 are [H][M][d];
+ * den is [B][H][N]; phi is [B][H][N][2M].  All doubles, row-major, contiguous.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* ------------------------------------------------------------------------------------ */
+/* Feature map (Eq. phi_n, Eq. phi_non), one vector.                                       */
+/* ------------------------------------------------------------------------------------ */
+
+static double dot(int d, const double* a, const double* b)
+{
+    double s = 0.0;
+    for (int t = 0; t < d; ++t) s += a[t] * b[t];
+    return s;
+}
+
+/* phi (length 2M) of x (length d).  W2 == NULL selects the stationary map. */
+static void feature(int d, int M, const double* x, const double* W1, const double* W2,
+                    double* phi)
+{
+    const double c = 1.0 / sqrt((double)M);
+    for (int i = 0; i < M; ++i) {
+        const double* w1 = W1 + (size_t)i * d;
+        if (W2 == NULL) {
+            double a = dot(d, w1, x);
+            phi[i] = c * cos(a);
+            phi[M + i] = c * sin(a);
+        } else {
+            const double* w2 = W2 + (size_t)i * d;
+            double u = 0.0, w = 0.0;           /* u = w'_1i . x,  w = w'_2i . x */
+            for (int t = 0; t < d; ++t) {
+                u += 0.5 * (w1[t] + w2[t]) * x[t];
+                w += 0.5 * (w1[t] - w2[t]) * x[t];
+            }
+            phi[i] = c * cos(u) * cos(w);
+            phi[M + i] = c * sin(u) * cos(w);
+        }
+    }
+}
+
+/* The same nonstationary map written as the Monte Carlo sum of Eq. (phi_non) before the
+ * sum-to-product step: (cos w_1i.x + cos w_2i.x, sin w_1i.x + sin w_2i.x) / (2 sqrt M).
+ * Used only to check the product form above against the paper's own derivation. */
+static void feature_sumform(int d, int M, const double* x, const double* W1, const double* W2,
+                            double* phi)
+{
+    const double c = 0.5 / sqrt((double)M);
+    for (int i = 0; i < M; ++i) {
+        double a = dot(d, W1 + (size_t)i * d, x);
+        double b = dot(d, W2 + (size_t)i * d, x);
+        phi[i] = c * (cos(a) + cos(b));
+        phi[M + i] = c * (sin(a) + sin(b));
+    }
+}
+
+/* Gradient of the feature map.  Given x and dphi (length 2M), adds the contribution to
+ * dx (length d) and to dA, dB ([M][d] each).  Stationary: dA = dW1, dB unused.
+ * Nonstationary: dA = dU, dB = dV for U = (W1+W2)/2 and V = (W1-W2)/2; the caller turns
+ * them into dW1 = (dU+dV)/2, dW2 = (dU-dV)/2. */
+static void feature_backward(int d, int M, const double* x, const double* W1,
+                             const double* W2, const double* dphi, double* dx, double* dA,
+                             double* dB)
+{
+    const double c = 1.0 / sqrt((double)M);
+    for (int i = 0; i < M; ++i) {
+        const double* w1 = W1 + (size_t)i * d;
+        const double dc = dphi[i], ds = dphi[M + i];
+        if (W2 == NULL) {
+            double a = dot(d, w1, x);
+            double da = c * (-sin(a) * dc + cos(a) * ds);
+            for (int t = 0; t < d; ++t) {
+                dx[t] += da * w1[t];
+                dA[(size_t)i * d + t] += da * x[t];
+            }
+        } else {
+            const double* w2 = W2 + (size_t)i * d;
+            double u = 0.0, w = 0.0;
+            for (int t = 0; t < d; ++t) {
+                u += 0.5 * (w1[t] + w2[t]) * x[t];
+                w += 0.5 * (w1[t] - w2[t]) * x[t];
+            }
+            /* phi_c = c cos u cos w, phi_s = c sin u cos w */
+            double du = c * cos(w) * (-sin(u) * dc + cos(u) * ds);
+            double dw = -c * sin(w) * (cos(u) * dc + sin(u) * ds);
+            for (int t = 0; t < d; ++t) {
+                dx[t] += du * 0.5 * (w1[t] + w2[t]) + dw * 0.5 * (w1[t] - w2[t]);
+                dA[(size_t)i * d + t] += du * x[t];
+                dB[(size_t)i * d + t] += dw * x[t];
+            }
+        }
+    }
+}
+
+/* ------------------------------------------------------------------------------------ */
+/* Linear attention of one (b, h) sequence (Eq. linear att).                               */
+/* ------------------------------------------------------------------------------------ */
+
+typedef struct {
+    int N, d, M, causal;
+    const double *q, *k, *v, *W1, *W2, *dout;
+    double *out, *den, *dq, *dk, *dv, *dA, *dB;
+} seq_job;
+
+/* out[i] = phi(q_i)^T S / phi(q_i)^T z with S = sum phi(k_j) v_j^T, z = sum phi(k_j);
+ * j runs over j <= i when causal, over all j otherwise. */
+static void forward_seq(const seq_job* J)
+{
+    const int N = J->N, d = J->d, M = J->M, D = 2 * M;
+    double* S = calloc((size_t)D * d, sizeof(double));
+    double* z = calloc((size_t)D, sizeof(double));
+    double* pk = malloc(sizeof(double) * D);
+    double* pq = malloc(sizeof(double) * D);
+    double* num = malloc(sizeof(double) * d);
+
+    if (!J->causal) {
+        for (int j = 0; j < N; ++j) {
+            feature(d, M, J->k + (size_t)j * d, J->W1, J->W2, pk);
+            for (int f = 0; f < D; ++f) {
+                z[f] += pk[f];
+                for (int e = 0; e < d; ++e) S[(size_t)f * d + e] += pk[f] * J->v[(size_t)j * d + e];
+            }
+        }
+    }
+    for (int i = 0; i < N; ++i) {
+        if (J->causal) {
+            feature(d, M, J->k + (size_t)i * d, J->W1, J->W2, pk);
+            for (int f = 0; f < D; ++f) {
+                z[f] += pk[f];
+                for (int e = 0; e < d; ++e) S[(size_t)f * d + e] += pk[f] * J->v[(size_t)i * d + e];
+            }
+        }
+        feature(d, M, J->q + (size_t)i * d, J->W1, J->W2, pq);
+        double dn = 0.0;
+        for (int e = 0; e < d; ++e) num[e] = 0.0;
+        for (int f = 0; f < D; ++f) {
+            dn += pq[f] * z[f];
+            for (int e = 0; e < d; ++e) num[e] += pq[f] * S[(size_t)f * d + e];
+        }
+        for (int e = 0; e < d; ++e) J->out[(size_t)i * d + e] = num[e] / dn;
+        if (J->den) J->den[i] = dn;
+    }
+    free(S); free(z); free(pk); free(pq); free(num);
+}
+
+/* Gradient of L = sum_i dout_i . out_i with respect to q, k, v and the frequencies. */
+static void backward_seq(const seq_job* J)
+{
+    const int N = J->N, d = J->d, M = J->M, D = 2 * M;
+    double* out = malloc(sizeof(double) * (size_t)N * d);
+    double* den = malloc(sizeof(double) * (size_t)N);
+    seq_job F = *J;
+    F.out = out;
+    F.den = den;
+    forward_seq(&F);
+
+    double* PQ = malloc(sizeof(double) * (size_t)N * D);   /* phi(q_i) */
+    double* PK = malloc(sizeof(double) * (size_t)N * D);   /* phi(k_j) */
+    double* g = malloc(sizeof(double) * (size_t)N * d);    /* dout_i / den_i */
+    double* cc = malloc(sizeof(double) * (size_t)N);       /* -(dout_i . out_i) / den_i */
+    for (int i = 0; i < N; ++i) {
+        feature(d, M, J->q + (size_t)i * d, J->W1, J->W2, PQ + (size_t)i * D);
+        feature(d, M, J->k + (size_t)i * d, J->W1, J->W2, PK + (size_t)i * D);
+        const double* dO = J->dout + (size_t)i * d;
+        double s = 0.0;
+        for (int e = 0; e < d; ++e) {
+            g[(size_t)i * d + e] = dO[e] / den[i];
+            s += dO[e] * out[(size_t)i * d + e];
+        }
+        cc[i] = -s / den[i];
+    }
+
+    double* S = calloc((size_t)D * d, sizeof(double));
+    double* z = calloc((size_t)D, sizeof(double));
+    double* dphi = malloc(sizeof(double) * D);
+
+    /* dq: forward-direction running sums S_i, z_i (totals when non-causal). */
+    if (!J->causal) {
+        for (int j = 0; j < N; ++j)
+            for (int f = 0; f < D; ++f) {
+                z[f] += PK[(size_t)j * D + f];
+                for (int e = 0; e < d; ++e)
+                    S[(size_t)f * d + e] += PK[(size_t)j * D + f] * J->v[(size_t)j * d + e];
+            }
+    }
+    for (int i = 0; i < N; ++i) {
+        if (J->causal)
+            for (int f = 0; f < D; ++f) {
+                z[f] += PK[(size_t)i * D + f];
+                for (int e = 0; e < d; ++e)
+                    S[(size_t)f * d + e] += PK[(size_t)i * D + f] * J->v[(size_t)i * d + e];
+            }
+        for (int f = 0; f < D; ++f) {
+            double s = cc[i] * z[f];
+            for (int e = 0; e < d; ++e) s += S[(size_t)f * d + e] * g[(size_t)i * d + e];
+            dphi[f] = s;
+        }
+        feature_backward(d, M, J->q + (size_t)i * d, J->W1, J->W2, dphi, J->dq + (size_t)i * d,
+                         J->dA, J->dB);
+    }
+
+    /* dk, dv: reverse-direction running sums R_j, r_j (totals when non-causal). */
+    double* R = S;  /* reuse: R[f][e] */
+    double* r = z;
+    memset(R, 0, sizeof(double) * (size_t)D * d);
+    memset(r, 0, sizeof(double) * D);
+    if (!J->causal) {
+        for (int i = 0; i < N; ++i)
+            for (int f = 0; f < D; ++f) {
+                r[f] += cc[i] * PQ[(size_t)i * D + f];
+                for (int e = 0; e < d; ++e)
+                    R[(size_t)f * d + e] += PQ[(size_t)i * D + f] * g[(size_t)i * d + e];
+            }
+    }
+    for (int j = N - 1; j >= 0; --j) {
+        if (J->causal)
+            for (int f = 0; f < D; ++f) {
+                r[f] += cc[j] * PQ[(size_t)j * D + f];
+                for (int e = 0; e < d; ++e)
+                    R[(size_t)f * d + e] += PQ[(size_t)j * D + f] * g[(size_t)j * d + e];
+            }
+        const double* vj = J->v + (size_t)j * d;
+        const double* pk = PK + (size_t)j * D;
+        for (int f = 0; f < D; ++f) dphi[f] = r[f] + dot(d, R + (size_t)f * d, vj);
+        for (int e = 0; e < d; ++e) {
+            double s = 0.0;
+            for (int f = 0; f < D; ++f) s += R[(size_t)f * d + e] * pk[f];
+            J->dv[(size_t)j * d + e] = s;
+        }
+        feature_backward(d, M, J->k + (size_t)j * d, J->W1, J->W2, dphi, J->dk + (size_t)j * d,
+                         J->dA, J->dB);
+    }
+    free(out); free(den); free(PQ); free(PK); free(g); free(cc);
+    free(S); free(z); free(dphi);
+}
+
+/* ------------------------------------------------------------------------------------ */
+/* Threading over independent (b, h) sequences.                                            */
+/* ------------------------------------------------------------------------------------ */
+
+typedef struct {
+    seq_job* jobs;
+    int njobs, stride, first, backward;
+} worker_arg;
+
+static void* worker(void* p)
+{
+    worker_arg* a = (worker_arg*)p;
+    for (int u = a->first; u < a->njobs; u += a->stride) {
+        if (a->backward) backward_seq(&a->jobs[u]);
+        else forward_seq(&a->jobs[u]);
+    }
+    return NULL;
+}
+
+static void run_jobs(seq_job* jobs, int njobs, int nthreads, int backward)
+{
+    if (nthreads < 1) nthreads = 1;
+    if (nthreads > njobs) nthreads = njobs;
+    pthread_t* th = malloc(sizeof(pthread_t) * nthreads);
+    worker_arg* args = malloc(sizeof(worker_arg) * nthreads);
+    for (int t = 0; t < nthreads; ++t) {
+        args[t] = (worker_arg){jobs, njobs, nthreads, t, backward};
+        if (t > 0) pthread_create(&th[t], NULL, worker, &args[t]);
+    }
+    worker(&args[0]);
+    for (int t = 1; t < nthreads; ++t) pthread_join(th[t], NULL);
+    free(th); free(args);
+}
+
+static int bad_shape(int B, int H, int N, int d, int M)
+{
+    return B < 1 || H < 1 || N < 1 || d < 1 || M < 1;
+}
+
+/* ------------------------------------------------------------------------------------ */
+/* Exported entry points.  Return 0 on success, -1 on a bad shape.                         */
+/* ------------------------------------------------------------------------------------ */
+
+int oracle_featmap(int B, int H, int N, int d, int M, const double* x, const double* W1,
+                   const double* W2, double* phi)
+{
+    if (bad_shape(B, H, N, d, M)) return -1;
+    for (int b = 0; b < B; ++b)
+        for (int h = 0; h < H; ++h) {
+            const double* w1 = W1 + (size_t)h * M * d;
+            const double* w2 = W2 ? W2 + (size_t)h * M * d : NULL;
+            for (int n = 0; n < N; ++n) {
+                size_t row = ((size_t)b * H + h) * N + n;
+                feature(d, M, x + row * d, w1, w2, phi + row * 2 * M);
+            }
+        }
+    return 0;
+}
+
+int oracle_featmap_sumform(int B, int H, int N, int d, int M, const double* x,
+                           const double* W1, const double* W2, double* phi)
+{
+    if (bad_shape(B, H, N, d, M) || W2 == NULL) return -1;
+    for (int b = 0; b < B; ++b)
+        for (int h = 0; h < H; ++h)
+            for (int n = 0; n < N; ++n) {
+                size_t row = ((size_t)b * H + h) * N + n;
+                feature_sumform(d, M, x + row * d, W1 + (size_t)h * M * d,
+                                W2 + (size_t)h * M * d, phi + row * 2 * M);
+            }
+    return 0;
+}
+
+int oracle_linattn_fwd(int B, int H, int N, int d, int M, const double* q, const double* k,
+                       const double* v, const double* W1, const double* W2, int causal,
+                       double* out, double* den, int nthreads)
+{
+    if (bad_shape(B, H, N, d, M)) return -1;
+    seq_job* jobs = calloc((size_t)B * H, sizeof(seq_job));
+    for (int b = 0; b < B; ++b)
+        for (int h = 0; h < H; ++h) {
+            size_t u = (size_t)b * H + h, off = u * N * d;
+            jobs[u] = (seq_job){N, d, M, causal, q + off, k + off, v + off,
+                                W1 + (size_t)h * M * d, W2 ? W2 + (size_t)h * M * d : NULL,
+                                NULL, out + off, den ? den + u * N : NULL,
+                                NULL, NULL, NULL, NULL, NULL};
+        }
+    run_jobs(jobs, B * H, nthreads, 0);
+    free(jobs);
+    return 0;
+}
+
+/* dW1 (and dW2) are sums over the batch and the sequence; they are overwritten. */
+int oracle_linattn_bwd(int B, int H, int N, int d, int M, const double* q, const double* k,
+                       const double* v, const double* W1, const double* W2, int causal,
+                       const double* dout, double* dq, double* dk, double* dv, double* dW1,
+                       double* dW2, int nthreads)
+{
+    if (bad_shape(B, H, N, d, M)) return -1;
+    if ((W2 == NULL) != (dW2 == NULL)) return -1;
+    const size_t per = (size_t)M * d;
+    double* dA = calloc((size_t)B * H * per, sizeof(double));
+    double* dB = calloc((size_t)B * H * per, sizeof(double));
+    seq_job* jobs = calloc((size_t)B * H, sizeof(seq_job));
+    for (int b = 0; b < B; ++b)
+        for (int h = 0; h < H; ++h) {
+            size_t u = (size_t)b * H + h, off = u * N * d;
+            memset(dq + off, 0, sizeof(double) * (size_t)N * d);
+            memset(dk + off, 0, sizeof(double) * (size_t)N * d);
+            jobs[u] = (seq_job){N, d, M, causal, q + off, k + off, v + off,
+                                W1 + (size_t)h * per, W2 ? W2 + (size_t)h * per : NULL,
+                                dout + off, NULL, NULL, dq + off, dk + off, dv + off,
+                                dA + u * per, dB + u * per};
+        }
+    run_jobs(jobs, B * H, nthreads, 1);
+    /* Sum the per-sequence parameter gradients over the batch in a fixed order. */
+    for (int h = 0; h < H; ++h)
+        for (size_t t = 0; t < per; ++t) {
+            double a = 0.0, bb = 0.0;
+            for (int b = 0; b < B; ++b) {
+                size_t u = (size_t)b * H + h;
+                a += dA[u * per + t];
+                bb += dB[u * per + t];
+            }
+            if (W2 == NULL) {
+                dW1[h * per + t] = a;
+            } else {
+                dW1[h * per + t] = 0.5 * (a + bb);
+                dW2[h * per + t] = 0.5 * (a - bb);
+            }
+        }
+    free(dA); free(dB); free(jobs);
+    return 0;
+}

@@ -1,0 +1,203 @@
+"""Checks that pin the fp64 oracle to facts fixed by the paper and by mathematics.
+
+Each ``pin_*`` function takes one compiled copy of the C oracle (``oracle.Oracle``) and
+raises AssertionError when the copy disagrees with the fact it checks.  The same
+functions run against the real oracle (all must pass) and against copies with planted
+mistakes (at least one must fail), so every pin is itself checked.
+
+Facts used (none is the oracle's own formula retyped):
+  * x = 0 gives phi = M^{-1/2} [1..1, 0..0]: fixes feature order (cos block first,
+    Eq. phi_n) and the scale.
+  * |phi_s(x)| = 1 (cos^2 + sin^2 = 1): fixes the stationary scale.
+  * Eq. (phi_non): the product form equals the Monte Carlo sum form (sum-to-product).
+  * W2 = W1 reduces Flexformer_n to Flexformer_s.
+  * Bochner (Thm. bochner): with w ~ N(0, s^-2 I), phi(x).phi(y) -> exp(-|x-y|^2 / 2 s^2).
+  * Yaglom (Thm. yaglom) with independent Gaussian W1, W2:
+      E = 1/2 exp(-|x-y|^2 / 2 s^2) + 1/2 exp(-(|x|^2 + |y|^2) / 2 s^2).
+  * Eq. (linear att) is an exact reassociation of Eq. (attention): the C linear form
+    equals the numpy N x N form (different module, different feature form).
+  * d = 1, M = 1: phi_s(q).phi_s(k) = cos(w (q - k)) in closed form.
+  * causal output at the last position equals the non-causal output.
+  * causal O_0 = v_0; constant v = c gives O = c (rows of weights sum to one).
+  * gradients: central finite differences of the numpy N x N form; the exact invariants
+    sum_j dv_j = sum_i dO_i, translation invariance of the stationary kernel
+    (sum dq + sum dk = 0) and Euler's identity for a = W x
+    (<dW1, W1> + <dW2, W2> = sum <dq, q> + sum <dk, k>).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from oracle import brute
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+def _case(seed, B, H, N, d, M, variant, qk_scale=0.5):
+    g = _rng(seed)
+    q = g.standard_normal((B, H, N, d)) * qk_scale
+    k = g.standard_normal((B, H, N, d)) * qk_scale
+    v = g.standard_normal((B, H, N, d))
+    W1 = g.standard_normal((H, M, d)) / np.sqrt(d)
+    W2 = g.standard_normal((H, M, d)) / np.sqrt(d) if variant == "n" else None
+    return q, k, v, W1, W2
+
+
+def _rel(a, b):
+    return float(np.max(np.abs(a - b)) / max(np.max(np.abs(b)), 1e-300))
+
+
+def pin_origin_features(orc):
+    for W2 in (None, np.full((2, 5, 3), 0.3)):
+        W1 = _rng(1).standard_normal((2, 5, 3))
+        phi = orc.featmap(np.zeros((1, 2, 4, 3)), W1, W2)
+        expect = np.concatenate([np.ones(5), np.zeros(5)]) / np.sqrt(5)
+        assert np.allclose(phi, expect, rtol=0, atol=1e-15), "phi(0) order or scale"
+
+
+def pin_stationary_unit_norm(orc):
+    q, _, _, W1, _ = _case(2, 2, 3, 7, 5, 11, "s", qk_scale=3.0)
+    phi = orc.featmap(q, W1)
+    assert np.allclose(np.sum(phi * phi, axis=-1), 1.0, rtol=0, atol=1e-13), "|phi_s| != 1"
+
+
+def pin_sum_to_product(orc):
+    q, _, _, W1, W2 = _case(3, 2, 2, 9, 6, 13, "n", qk_scale=2.0)
+    prod = orc.featmap(q, W1, W2)
+    assert _rel(prod, brute.features(q, W1, W2)) < 1e-13, "product form != sum form (numpy)"
+    assert _rel(prod, orc.featmap_sumform(q, W1, W2)) < 1e-13, "product form != sum form (C)"
+
+
+def pin_w2_equals_w1(orc):
+    q, _, _, W1, _ = _case(4, 1, 2, 6, 4, 8, "s", qk_scale=2.0)
+    assert _rel(orc.featmap(q, W1, W1.copy()), orc.featmap(q, W1)) < 1e-15, "W2=W1 != phi_s"
+
+
+def _kernel_estimate(orc, x, y, W1, W2):
+    """phi(x).phi(y) and the per-frequency terms whose mean it is."""
+    px = orc.featmap(x[None, None, None], W1[None], None if W2 is None else W2[None])[0, 0, 0]
+    py = orc.featmap(y[None, None, None], W1[None], None if W2 is None else W2[None])[0, 0, 0]
+    M = W1.shape[0]
+    terms = M * (px[:M] * py[:M] + px[M:] * py[M:])
+    return float(px @ py), terms
+
+
+def pin_bochner(orc):
+    g = _rng(5)
+    d, M, sigma = 6, 1 << 16, 1.3
+    W = g.standard_normal((M, d)) / sigma
+    for _ in range(3):
+        x, y = g.standard_normal(d) * 0.8, g.standard_normal(d) * 0.8
+        est, terms = _kernel_estimate(orc, x, y, W, None)
+        exact = np.exp(-np.sum((x - y) ** 2) / (2 * sigma ** 2))
+        assert abs(est - exact) <= 5 * terms.std() / np.sqrt(M), "Bochner estimate off"
+
+
+def pin_yaglom(orc):
+    g = _rng(6)
+    d, M, sigma = 6, 1 << 16, 1.3
+    W1 = g.standard_normal((M, d)) / sigma
+    W2 = g.standard_normal((M, d)) / sigma
+    for _ in range(3):
+        x, y = g.standard_normal(d) * 0.8, g.standard_normal(d) * 0.8
+        est, terms = _kernel_estimate(orc, x, y, W1, W2)
+        exact = 0.5 * np.exp(-np.sum((x - y) ** 2) / (2 * sigma ** 2)) + 0.5 * np.exp(
+            -(np.sum(x * x) + np.sum(y * y)) / (2 * sigma ** 2))
+        assert abs(est - exact) <= 5 * terms.std() / np.sqrt(M), "Yaglom estimate off"
+
+
+def pin_linear_equals_brute(orc):
+    for variant in ("s", "n"):
+        for causal in (True, False):
+            for N in (1, 2, 3, 17, 64, 256):
+                q, k, v, W1, W2 = _case(10 + N, 2, 2, N, 5, 7, variant)
+                out, den = orc.fwd(q, k, v, W1, W2, causal)
+                bo, bd = brute.attention(q, k, v, W1, W2, causal)
+                assert _rel(den, bd) < 1e-12, f"den {variant} causal={causal} N={N}"
+                assert _rel(out, bo) < 1e-11, f"out {variant} causal={causal} N={N}"
+
+
+def pin_closed_form_d1(orc):
+    q = np.array([0.3, -1.1, 0.7]).reshape(1, 1, 3, 1)
+    k = np.array([0.1, 0.5, -0.4]).reshape(1, 1, 3, 1)
+    v = np.array([1.0, 2.0, -3.0]).reshape(1, 1, 3, 1)
+    w = 0.9
+    out, den = orc.fwd(q, k, v, np.array([[[w]]]), None, causal=True)
+    A = np.cos(w * (q.reshape(3, 1) - k.reshape(1, 3))) * np.tril(np.ones((3, 3)))
+    assert np.allclose(den[0, 0], A.sum(1), rtol=1e-14, atol=0), "closed form den"
+    assert np.allclose(out[0, 0, :, 0], A @ v.reshape(3) / A.sum(1), rtol=1e-13), "closed form"
+
+
+def pin_causal_last_equals_noncausal(orc):
+    for variant in ("s", "n"):
+        q, k, v, W1, W2 = _case(20, 2, 2, 33, 4, 6, variant)
+        oc, dc = orc.fwd(q, k, v, W1, W2, True)
+        on, dn = orc.fwd(q, k, v, W1, W2, False)
+        assert _rel(oc[:, :, -1], on[:, :, -1]) < 1e-12, "causal last != non-causal"
+        assert _rel(dc[:, :, -1], dn[:, :, -1]) < 1e-12, "causal last den != non-causal"
+
+
+def pin_first_and_constant(orc):
+    for variant in ("s", "n"):
+        q, k, v, W1, W2 = _case(21, 2, 2, 19, 4, 6, variant)
+        out, _ = orc.fwd(q, k, v, W1, W2, True)
+        assert _rel(out[:, :, 0], v[:, :, 0]) < 1e-13, "causal O_0 != v_0"
+        for causal in (True, False):
+            c = np.full_like(v, 1.75)
+            out, _ = orc.fwd(q, k, c, W1, W2, causal)
+            assert np.allclose(out, 1.75, rtol=1e-12, atol=0), "constant v not preserved"
+
+
+def _loss(q, k, v, W1, W2, causal, dO):
+    return float(np.sum(brute.attention(q, k, v, W1, W2, causal)[0] * dO))
+
+
+def pin_finite_differences(orc):
+    h = 1e-6
+    for variant in ("s", "n"):
+        for causal in (True, False):
+            q, k, v, W1, W2 = _case(30, 2, 2, 5, 3, 4, variant)
+            dO = _rng(31).standard_normal(q.shape)
+            grads = orc.bwd(q, k, v, W1, W2, causal, dO)
+            params = [q, k, v, W1] + ([W2] if W2 is not None else [])
+            for idx, (p, gp) in enumerate(zip(params, grads)):
+                fd = np.zeros_like(p)
+                it = np.nditer(p, flags=["multi_index"])
+                for _ in it:
+                    mi = it.multi_index
+                    old = p[mi]
+                    p[mi] = old + h
+                    lp = _loss(q, k, v, W1, W2, causal, dO)
+                    p[mi] = old - h
+                    lm = _loss(q, k, v, W1, W2, causal, dO)
+                    p[mi] = old
+                    fd[mi] = (lp - lm) / (2 * h)
+                err = np.linalg.norm(gp - fd) / np.linalg.norm(fd)
+                assert err < 1e-6, f"FD {variant} causal={causal} grad #{idx}: {err:.2e}"
+
+
+def pin_gradient_invariants(orc):
+    for variant in ("s", "n"):
+        for causal in (True, False):
+            q, k, v, W1, W2 = _case(40, 2, 3, 23, 5, 7, variant)
+            dO = _rng(41).standard_normal(q.shape)
+            dq, dk, dv, dW1, dW2 = orc.bwd(q, k, v, W1, W2, causal, dO)
+            s_dv, s_do = dv.sum(axis=2), dO.sum(axis=2)
+            assert _rel(s_dv, s_do) < 1e-11, "sum dv != sum dO"
+            lhs = np.sum(dW1 * W1) + (np.sum(dW2 * W2) if W2 is not None else 0.0)
+            rhs = np.sum(dq * q) + np.sum(dk * k)
+            assert abs(lhs - rhs) < 1e-10 * max(abs(rhs), 1.0), "Euler identity"
+            if variant == "s":
+                t = dq.sum(axis=2) + dk.sum(axis=2)
+                scale = np.abs(dq).sum(axis=2) + np.abs(dk).sum(axis=2)
+                assert np.all(np.abs(t) < 1e-11 * scale), "translation invariance"
+
+
+ALL_PINS = [
+    pin_origin_features, pin_stationary_unit_norm, pin_sum_to_product, pin_w2_equals_w1,
+    pin_bochner, pin_yaglom, pin_linear_equals_brute, pin_closed_form_d1,
+    pin_causal_last_equals_noncausal, pin_first_and_constant, pin_finite_differences,
+    pin_gradient_invariants,
+]

@@ -1,0 +1,67 @@
+"""Each planted mistake in a copy of the C oracle must make at least one pin fail.
+
+The mistakes are planted in a copy of the oracle's source text, compiled on the CPU into
+a separate library; the oracle itself is never modified.
+"""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+import oracle_pins
+
+# (name, exact text in flex_oracle.c, replacement, occurrence to replace (0 = first))
+MUTATIONS = [
+    ("swap_sin_cos_stationary",
+     "phi[i] = c * cos(a);\n            phi[M + i] = c * sin(a);",
+     "phi[i] = c * sin(a);\n            phi[M + i] = c * cos(a);", 0),
+    ("omega_prime_without_half",
+     "u += 0.5 * (w1[t] + w2[t]) * x[t];\n                w += 0.5 * (w1[t] - w2[t]) * x[t];\n            }\n            phi[i]",
+     "u += (w1[t] + w2[t]) * x[t];\n                w += (w1[t] - w2[t]) * x[t];\n            }\n            phi[i]", 0),
+    ("sum_instead_of_average_scale",
+     "phi[i] = c * cos(u) * cos(w);", "phi[i] = 2.0 * c * cos(u) * cos(w);", 0),
+    ("sin_block_uses_sin_w",
+     "phi[M + i] = c * sin(u) * cos(w);", "phi[M + i] = c * sin(u) * sin(w);", 0),
+    ("forget_normaliser_z", "dn += pq[f] * z[f];", "dn += pq[f];", 0),
+    ("causal_mask_exclusive",
+     "for (int i = 0; i < N; ++i) {\n        if (J->causal) {\n            feature(d, M, J->k + (size_t)i * d",
+     "for (int i = 0; i < N; ++i) {\n        if (J->causal && i > 0) {\n            feature(d, M, J->k + (size_t)(i - 1) * d", 0),
+    ("drop_half_in_dW1", "dW1[h * per + t] = 0.5 * (a + bb);", "dW1[h * per + t] = (a + bb);", 0),
+    ("wrong_sign_du", "double du = c * cos(w) * (-sin(u) * dc + cos(u) * ds);",
+     "double du = c * cos(w) * (sin(u) * dc + cos(u) * ds);", 0),
+    ("wrong_sign_da_stationary", "double da = c * (-sin(a) * dc + cos(a) * ds);",
+     "double da = c * (sin(a) * dc + cos(a) * ds);", 0),
+    ("drop_normaliser_grad_in_dq", "double s = cc[i] * z[f];", "double s = 0.0;", 0),
+    ("drop_normaliser_grad_in_dk", "dphi[f] = r[f] + dot(d, R + (size_t)f * d, vj);",
+     "dphi[f] = dot(d, R + (size_t)f * d, vj);", 0),
+    ("denominator_sign_in_c", "cc[i] = -s / den[i];", "cc[i] = s / den[i];", 0),
+    ("reverse_scan_exclusive",
+     "for (int j = N - 1; j >= 0; --j) {\n        if (J->causal)",
+     "for (int j = N - 1; j >= 0; --j) {\n        if (J->causal && 0)", 0),
+]
+
+
+def _apply(src, old, new, occurrence):
+    assert src.count(old) >= 1, "mutation target not found in the oracle source"
+    pos = -1
+    for _ in range(occurrence + 1):
+        pos = src.index(old, pos + 1)
+    return src[:pos] + new + src[pos + len(old):]
+
+
+@pytest.mark.parametrize("name,old,new,occ", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_planted_mistake_is_caught(tmp_path, name, old, new, occ):
+    with open(oracle.SOURCE) as f:
+        src = f.read()
+    path = oracle.compile_library(_apply(src, old, new, occ),
+                                  os.path.join(str(tmp_path), f"mut_{name}.so"))
+    mutant = oracle.Oracle(path)
+    failed = []
+    with np.errstate(all="ignore"):
+        for pin in oracle_pins.ALL_PINS:
+            try:
+                pin(mutant)
+            except (AssertionError, FloatingPointError, ValueError):
+                failed.append(pin.__name__)
+    assert failed, f"no pin caught the planted mistake {name}"
