@@ -1,0 +1,375 @@
+#!/usr/bin/env python
+"""Forward throughput of random-Fourier-feature linear attention on GB300.
+
+Default workload: nonstationary (Flexformer_n) causal forward, bf16 storage,
+B=4, H=16, N=16384, d=64, M=128 (d'=256), seeded synthetic inputs.  A step is one call
+of flex_linattn_fwd over the whole batch.  Prints one JSON line (rank 0).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload NAME]
+
+`--impl reference` times the fp64 CPU oracle on the host cores instead (each step a
+bounded sample of whole sequences of the same workload).  Under torchrun each rank runs
+its own full replica of the workload (the (b, h) sequences are independent; no
+collective on the data path), so the value is weak-scaled.
+"""
+from __future__ import annotations
+
+import argparse
+import glob
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2606_27748_gb300 import workloads  # noqa: E402
+
+METRIC = "RFF linear-attn fwd tokens/s (N=16K causal) & % of bf16 tensor/HBM roofline"
+L2_BYTES = 129 * 1024 * 1024
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=workloads.HEADLINE.name,
+                    choices=list(workloads.WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------------------
+# Work accounting (algorithmic, per token-head): q, k, v read + out written; flops of the
+# two projections and of the state read and update (Eq. linear att, Eq. phi_n/phi_non).
+# ---------------------------------------------------------------------------------------
+def elem_bytes(w):
+    return 2 if w.dtype == "bf16" else 4
+
+
+def algorithmic_bytes(w):
+    return w.token_heads * 4 * w.d * elem_bytes(w)
+
+
+def algorithmic_flops(w):
+    mc = 2 * w.M if w.variant == "n" else w.M
+    per = 2 * (2 * w.d * mc) + 2 * (2 * (2 * w.M) * w.d)
+    return w.token_heads * per
+
+
+def source_digest():
+    h = hashlib.sha256()
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2606_27748_gb300", "csrc", "*"))):
+        h.update(open(f, "rb").read())
+    return h.hexdigest()
+
+
+def load_peaks():
+    if os.path.exists(PEAKS_FILE):
+        return json.load(open(PEAKS_FILE)), "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+def recorded_traffic(w, kernel_digest):
+    """DRAM bytes per launch from the committed ncu summary, if it is for this source."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    try:
+        t = json.load(open(TRAFFIC_FILE)).get(w.name)
+    except ValueError:
+        return None
+    if not t or t.get("source_sha256") != kernel_digest:
+        return None
+    return t.get("dram_bytes_per_launch")
+
+
+# ---------------------------------------------------------------------------------------
+# Clock sampling during the timed region.
+# ---------------------------------------------------------------------------------------
+class Clocks:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.2)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), float(parts[3]), parts[5:9]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        smax = max(r[1] for r in rows)
+        loaded = [r for r in rows if r[2] > 200.0] or rows
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[3]) if v == "Active"})
+        return {"sm_mhz": statistics.median(r[0] for r in loaded), "sm_max_mhz": smax,
+                "reasons": reasons, "samples": len(rows), "samples_under_load": len(loaded)}
+
+
+# ---------------------------------------------------------------------------------------
+# CPU oracle timing (the reported baseline and the reference arm).
+# ---------------------------------------------------------------------------------------
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def oracle_sample(w, nseq, cores):
+    """Time the oracle forward over the first `nseq` whole sequences of `w`."""
+    import oracle
+    nb = -(-nseq // w.H)
+    ins = workloads.make_inputs(w, bs=range(nb))
+    # the first nseq (b, h) sequences in order, laid out as one batch row of nseq "heads",
+    # each with its own head's frequencies
+    q, k, v = (ins[n].reshape(nb * w.H, w.N, w.d)[None, :nseq] for n in "qkv")
+    heads = [s % w.H for s in range(nseq)]
+    W1 = ins["W1"][heads]
+    W2 = None if ins["W2"] is None else ins["W2"][heads]
+    t0 = time.perf_counter()
+    oracle.fwd(q, k, v, W1, W2, w.causal, nthreads=cores)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(w, cores, target_s=12.0):
+    bh = w.B * w.H
+    n1 = min(bh, cores)
+    t1 = oracle_sample(w, n1, cores)
+    nseq, t = n1, t1
+    if t1 < target_s / 2 and n1 < bh:
+        nseq = min(bh, n1 * max(1, int(target_s / max(t1, 1e-3))))
+        if nseq > n1:
+            t = oracle_sample(w, nseq, cores)
+    tokens = nseq * w.N / w.H
+    return {"value": tokens / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{nseq} of {bh} whole (b,h) sequences of N={w.N} (fp64 C oracle, "
+                      f"{cores} threads), {t:.2f} s; tokens = sequences*N/H"}
+
+
+def run_reference(args, w):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    cores = cpu_cores()
+    nseq = min(w.B * w.H, cores)
+    for _ in range(args.warmup):
+        oracle_sample(w, nseq, cores)
+    times = [oracle_sample(w, nseq, cores) for _ in range(args.steps)]
+    step = sum(times) / len(times)
+    value = nseq * w.N / w.H / step
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "impl": "reference",
+        "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d, "M": w.M,
+                   "variant": w.variant, "causal": w.causal},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{nseq} whole (b,h) sequences of N={w.N} per step"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------------------
+# Our arm.
+# ---------------------------------------------------------------------------------------
+def run_ours(args, w):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2606_27748_gb300 import build, flexattn
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if rank == 0 or not os.path.exists(flexattn.LIBRARY):
+        build.build()
+    if world > 1:
+        dist.barrier()
+    flexattn.load()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    ins = workloads.make_inputs(w)
+    tdt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    host = {n: torch.from_numpy(ins[n]).to(tdt).pin_memory() for n in "qkv"}
+    W1 = torch.from_numpy(ins["W1"]).to(dev)
+    W2 = None if ins["W2"] is None else torch.from_numpy(ins["W2"]).to(dev)
+    del ins
+    q, k, v = (host[n].to(dev) for n in "qkv")
+    out = torch.empty_like(q)
+    den = torch.empty(q.shape[:3], dtype=torch.float32, device=dev)
+    shape = flexattn.shape_of(q, W1)
+    ws = flexattn.workspace(shape, w.causal, False, dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        flexattn.linattn_fwd(q, k, v, W1, W2, w.causal, out=out, den=den, ws=ws)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    flexattn.check_status(ws)
+
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
+    clocks = Clocks(torch.cuda.current_device()) if rank == 0 else None
+    if clocks:
+        clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    launches0 = flexattn.kernel_launches()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(K):
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = flexattn.kernel_launches() - launches0
+    clk = clocks.stop() if clocks else None
+    flexattn.check_status(ws)
+    total_ms = t_start.elapsed_time(t_end)
+    kernel_ms = sum(a.elapsed_time(b) for a, b in ev) / K
+    if world > 1:
+        t = torch.tensor([total_ms, kernel_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms, kernel_ms = t.tolist()
+    ms_per_step = total_ms / K
+    value = world * w.tokens / (ms_per_step * 1e-3)
+
+    # End to end through the same C-ABI call with host buffers: H2D of q, k, v from pinned
+    # memory, the forward, D2H of out, every step.
+    e2e = None
+    if not args.no_e2e:
+        host_out = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+
+        def e2e_step():
+            for n, t in (("q", q), ("k", k), ("v", v)):
+                t.copy_(host[n], non_blocking=True)
+            step()
+            host_out.copy_(out, non_blocking=True)
+
+        for _ in range(max(3, args.warmup)):
+            e2e_step()
+        barrier()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(K):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e2e_ms = a.elapsed_time(b) / K
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = t.item()
+        h2d = sum(host[n].numel() * host[n].element_size() for n in "qkv")
+        e2e = {"value": world * w.tokens / (e2e_ms * 1e-3), "unit": "tokens/s",
+               "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": host_out.numel() * host_out.element_size()}
+
+    peaks, peaks_src = load_peaks()
+    nbytes = algorithmic_bytes(w)
+    achieved = nbytes / (kernel_ms * 1e-3) / 1e9
+    roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": achieved / peaks["hbm_gbs"], "traffic": recorded_traffic(w, source_digest()),
+            "peak_source": peaks_src,
+            "algorithmic_bytes_per_launch": nbytes,
+            "algorithmic_tflops": algorithmic_flops(w) / (kernel_ms * 1e-3) / 1e12,
+            "tensor_frac_of_burst_peak": algorithmic_flops(w) / (kernel_ms * 1e-3) / 1e12
+            / peaks["bf16_tflops"],
+            "kernel_ms": kernel_ms}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, cpu_cores())
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": K, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": w.dtype, "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d, "M": w.M,
+                       "variant": w.variant, "causal": w.causal,
+                       "l2": f"inputs {3 * w.token_heads * w.d * elem_bytes(w) / 1e6:.0f} MB "
+                             f"> L2 {L2_BYTES / 1e6:.0f} MB, no flush",
+                       "parallelism": f"replicas x{world}"},
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+            "gpu_launches": launches,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    w = workloads.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_ours(args, w)
+
+
+if __name__ == "__main__":
+    main()

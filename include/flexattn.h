@@ -1,0 +1,117 @@
+/*
+ * flexattn.h -- C ABI of the GB300 (sm_103a) random-Fourier-feature linear attention
+ * library (Flexformer: learnable spectral frequencies, stationary and nonstationary).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * Tensors (device pointers, contiguous, row-major):
+ *   q, k, v, out, dout, dq, dk, dv : [B][H][N][d]   in `dtype` (fp32 or bf16)
+ *   phi                            : [B][H][N][2M]  in `dtype`
+ *   W1, W2, dW1, dW2               : [H][M][d]      fp32, one frequency set per head
+ *   den                            : [B][H][N]      fp32
+ * W2 == NULL selects the stationary variant (Flexformer_s, Sec. 3.2); a non-NULL W2 selects
+ * the nonstationary variant (Flexformer_n, Eq. phi_non) with frequency pairs (W1, W2).
+ * The feature dimension is d' = 2M (Appendix "Complexity Analysis").
+ *
+ * Feature map (scale sigma = 1, i.e. M^{-1/2} for both variants):
+ *   stationary    phi(x) = M^{-1/2} [cos(W1 x), sin(W1 x)]                     (Eq. phi_n)
+ *   nonstationary u = (W1+W2)/2 x,  w = (W1-W2)/2 x,
+ *                 phi(x) = M^{-1/2} [cos u * cos w, sin u * cos w]              (Eq. phi_non)
+ * all cosine features first, then all sine features.
+ *
+ * Attention (Eq. linear att):
+ *   out_i = phi(q_i)^T S_i / den_i,  den_i = phi(q_i)^T z_i,
+ *   S_i = sum_j phi(k_j) v_j^T,  z_i = sum_j phi(k_j),
+ * with j <= i when causal (the diagonal is included) and all j otherwise.  The
+ * denominator is used as computed: no epsilon, no clamp.
+ *
+ * Ownership and ordering: the caller owns every buffer.  The library never allocates,
+ * frees or synchronises (except flex_check_status); all work is enqueued on `stream`
+ * (a cudaStream_t; NULL means the legacy default stream) of the current device.
+ * Scratch memory is the caller's workspace `ws` of at least flex_workspace_bytes()
+ * bytes, 256-byte aligned and zero-filled before its first use (kernels leave its
+ * control words as they found them); one workspace must not be used by two calls that
+ * may run concurrently.
+ *
+ * Errors: every entry point returns FLEX_OK or a negative flex_status and enqueues
+ * nothing on error.  Kernels that give up on the device (a bounded wait that ran out)
+ * record FLEX_ETIMEOUT in the workspace; flex_check_status() reports it.
+ */
+#ifndef FLEXATTN_H
+#define FLEXATTN_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum { FLEX_F32 = 0, FLEX_BF16 = 1 } flex_dtype;
+
+typedef struct {
+    int B;      /* batch */
+    int H;      /* heads */
+    int N;      /* sequence length, >= 1 */
+    int d;      /* head size */
+    int M;      /* frequencies per set; features d' = 2M */
+    int dtype;  /* flex_dtype of q, k, v, out, phi, dout, dq, dk, dv */
+} flex_shape;
+
+enum flex_status {
+    FLEX_OK = 0,
+    FLEX_EINVAL = -1,       /* NULL or misaligned pointer, N < 1, W2/dW2 mismatch, ... */
+    FLEX_EUNSUPPORTED = -2, /* valid but unsupported shape/dtype combination */
+    FLEX_EWORKSPACE = -3,   /* ws_bytes smaller than flex_workspace_bytes() */
+    FLEX_ECUDA = -4,        /* a CUDA launch or runtime call failed */
+    FLEX_ETIMEOUT = -5      /* a device-side bounded wait gave up (see flex_check_status) */
+};
+
+/* Human-readable text for a flex_status value. */
+const char* flex_strerror(int status);
+
+/* Workspace bytes needed by flex_linattn_fwd (backward = 0) or flex_linattn_bwd
+ * (backward = 1) for this shape; 0 if the shape is invalid or unsupported. */
+size_t flex_workspace_bytes(const flex_shape* shape, int causal, int backward);
+
+/* Feature map phi of Eq. phi_n (W2 == NULL) or Eq. phi_non (W2 != NULL), written out.
+ * x: [B][H][N][d], phi: [B][H][N][2M], both in shape->dtype.  This is the only entry
+ * point that writes phi to memory; the attention entry points keep it on chip. */
+int flex_featmap(const flex_shape* shape, const void* x, const float* W1, const float* W2,
+                 void* phi, void* stream);
+
+/* Forward linear attention, Eq. (linear att) with the feature map above.
+ * out: [B][H][N][d] in shape->dtype.  den: NULL, or [B][H][N] fp32 receiving den_i
+ * (needed by flex_linattn_bwd).  ws: workspace of ws_bytes bytes. */
+int flex_linattn_fwd(const flex_shape* shape, const void* q, const void* k, const void* v,
+                     const float* W1, const float* W2, int causal, void* out, float* den,
+                     void* ws, size_t ws_bytes, void* stream);
+
+/* Backward of flex_linattn_fwd: gradients of L = sum(dout * out) with respect to q, k,
+ * v and the frequencies.  out and den are the forward's outputs for the same inputs.
+ * dq, dk, dv: [B][H][N][d] in shape->dtype.  dW1 (and dW2, which must be NULL exactly
+ * when W2 is) are fp32 [H][M][d], summed over the batch and the sequence, overwritten.
+ * The paper gives no backward formulas; this is the analytic gradient of Eq. (linear
+ * att): with g_i = dout_i / den_i and c_i = -(dout_i . out_i) / den_i,
+ *   dphi(q_i) = S_i g_i + c_i z_i,  dphi(k_j) = R_j v_j + r_j,  dv_j = R_j^T phi(k_j),
+ *   R_j = sum_{i >= j} phi(q_i) g_i^T,  r_j = sum_{i >= j} c_i phi(q_i)
+ * (totals when non-causal), then through the feature map by the chain rule; for the
+ * nonstationary variant dW1 = (dU + dV)/2 and dW2 = (dU - dV)/2. */
+int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, const void* v,
+                     const float* W1, const float* W2, int causal, const void* out,
+                     const float* den, const void* dout, void* dq, void* dk, void* dv,
+                     float* dW1, float* dW2, void* ws, size_t ws_bytes, void* stream);
+
+/* Cumulative number of kernels this library has enqueued in this process (all entry
+ * points, all devices).  Lets a caller count the launches inside a timed region. */
+unsigned long long flex_kernel_launches(void);
+
+/* Synchronises `stream`, then returns FLEX_ETIMEOUT if a kernel that used `ws` gave up
+ * on a bounded wait since the workspace was last checked, FLEX_ECUDA on a pending CUDA
+ * error, else FLEX_OK.  Clears the recorded status. */
+int flex_check_status(void* ws, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FLEXATTN_H */

@@ -1,0 +1,160 @@
+// Host side of the C ABI declared in include/flexattn.h: argument validation, workspace
+// layout and kernel dispatch.  Nothing here allocates device memory or synchronises,
+// except flex_check_status.
+#include "flex_internal.h"
+
+#include <stdint.h>
+
+#include <atomic>
+
+using flex::Problem;
+
+namespace {
+
+bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+// Fills `p` from `s`; FLEX_OK or the error to return.
+int make_problem(const flex_shape* s, const float* W2, int causal, Problem* p)
+{
+    if (!s) return FLEX_EINVAL;
+    if (s->B < 1 || s->H < 1 || s->N < 1 || s->d < 1 || s->M < 1) return FLEX_EINVAL;
+    if (s->dtype != FLEX_F32 && s->dtype != FLEX_BF16) return FLEX_EINVAL;
+    if ((long long)s->B * s->H > (1LL << 30)) return FLEX_EUNSUPPORTED;
+    if ((long long)s->N > (1LL << 30)) return FLEX_EUNSUPPORTED;
+    if (s->d > 128 || s->M > 256 || s->d % 4 != 0) return FLEX_EUNSUPPORTED;
+    p->B = s->B; p->H = s->H; p->N = s->N; p->d = s->d; p->M = s->M;
+    p->bf16 = s->dtype == FLEX_BF16;
+    p->nonstat = W2 != nullptr;
+    p->causal = causal ? 1 : 0;
+    return FLEX_OK;
+}
+
+size_t header_bytes() { return sizeof(flex::WsHeader); }
+
+int check_ws(void* ws, size_t ws_bytes, size_t need)
+{
+    if (!ws) return FLEX_EINVAL;
+    if (!aligned(ws, 256)) return FLEX_EINVAL;
+    if (ws_bytes < need) return FLEX_EWORKSPACE;
+    return FLEX_OK;
+}
+
+size_t fwd_ws_bytes(const Problem& p)
+{
+    (void)p;
+    return header_bytes();
+}
+
+size_t bwd_ws_bytes(const Problem& p)
+{
+    return header_bytes() + flex::align_up(flex::simt_bwd_ws_bytes(p), 256);
+}
+
+std::atomic<unsigned long long> g_launches{0};
+
+// Records `n` enqueued kernels when the launch sequence succeeded.
+int count(int n, cudaError_t e)
+{
+    if (e != cudaSuccess) return FLEX_ECUDA;
+    g_launches += (unsigned long long)n;
+    return FLEX_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* flex_strerror(int status)
+{
+    switch (status) {
+    case FLEX_OK: return "ok";
+    case FLEX_EINVAL: return "invalid argument (null/misaligned pointer, bad shape or W2/dW2 mismatch)";
+    case FLEX_EUNSUPPORTED: return "unsupported shape or dtype";
+    case FLEX_EWORKSPACE: return "workspace too small";
+    case FLEX_ECUDA: return "CUDA error";
+    case FLEX_ETIMEOUT: return "a device-side bounded wait gave up";
+    default: return "unknown status";
+    }
+}
+
+size_t flex_workspace_bytes(const flex_shape* shape, int causal, int backward)
+{
+    Problem p;
+    if (make_problem(shape, nullptr, causal, &p) != FLEX_OK) return 0;
+    // The nonstationary variant needs the larger scratch; size for it.
+    p.nonstat = 1;
+    return backward ? bwd_ws_bytes(p) : fwd_ws_bytes(p);
+}
+
+int flex_featmap(const flex_shape* shape, const void* x, const float* W1, const float* W2,
+                 void* phi, void* stream)
+{
+    Problem p;
+    int rc = make_problem(shape, W2, 0, &p);
+    if (rc) return rc;
+    if (!x || !W1 || !phi) return FLEX_EINVAL;
+    if (!aligned(x, 16) || !aligned(W1, 16) || !aligned(phi, 16) || (W2 && !aligned(W2, 16)))
+        return FLEX_EINVAL;
+    return count(1, flex::launch_featmap(p, x, W1, W2, phi, (cudaStream_t)stream));
+}
+
+int flex_linattn_fwd(const flex_shape* shape, const void* q, const void* k, const void* v,
+                     const float* W1, const float* W2, int causal, void* out, float* den,
+                     void* ws, size_t ws_bytes, void* stream)
+{
+    Problem p;
+    int rc = make_problem(shape, W2, causal, &p);
+    if (rc) return rc;
+    if (!q || !k || !v || !W1 || !out) return FLEX_EINVAL;
+    for (const void* t : {q, k, v, (const void*)W1, (const void*)out})
+        if (!aligned(t, 16)) return FLEX_EINVAL;
+    if ((W2 && !aligned(W2, 16)) || (den && !aligned(den, 16))) return FLEX_EINVAL;
+    if ((rc = check_ws(ws, ws_bytes, fwd_ws_bytes(p)))) return rc;
+    if (flex::simt_pick_chunk_fwd(p) == 0) return FLEX_EUNSUPPORTED;
+    cudaStream_t s = (cudaStream_t)stream;
+    return count(1, flex::launch_simt_fwd(p, q, k, v, W1, W2, out, den, s));
+}
+
+int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, const void* v,
+                     const float* W1, const float* W2, int causal, const void* out,
+                     const float* den, const void* dout, void* dq, void* dk, void* dv,
+                     float* dW1, float* dW2, void* ws, size_t ws_bytes, void* stream)
+{
+    Problem p;
+    int rc = make_problem(shape, W2, causal, &p);
+    if (rc) return rc;
+    if (!q || !k || !v || !W1 || !out || !den || !dout || !dq || !dk || !dv || !dW1)
+        return FLEX_EINVAL;
+    if ((W2 == nullptr) != (dW2 == nullptr)) return FLEX_EINVAL;
+    for (const void* t : {q, k, v, (const void*)W1, out, (const void*)den, dout, (const void*)dq,
+                          (const void*)dk, (const void*)dv, (const void*)dW1})
+        if (!aligned(t, 16)) return FLEX_EINVAL;
+    if ((W2 && !aligned(W2, 16)) || (dW2 && !aligned(dW2, 16))) return FLEX_EINVAL;
+    if ((rc = check_ws(ws, ws_bytes, bwd_ws_bytes(p)))) return rc;
+    if (flex::simt_pick_chunk_bwd(p) == 0) return FLEX_EUNSUPPORTED;
+    cudaStream_t s = (cudaStream_t)stream;
+    void* scratch = (char*)ws + header_bytes();
+    return count(2, flex::launch_simt_bwd(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1,
+                                          dW2, scratch, s));
+}
+
+unsigned long long flex_kernel_launches(void) { return g_launches.load(); }
+
+int flex_check_status(void* ws, void* stream)
+{
+    if (!ws || !aligned(ws, 256)) return FLEX_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return FLEX_ECUDA;
+    flex::WsHeader h;
+    if (cudaMemcpyAsync(&h, ws, sizeof(h), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return FLEX_ECUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return FLEX_ECUDA;
+    if (h.status != FLEX_OK) {
+        if (cudaMemsetAsync(ws, 0, sizeof(int), s) != cudaSuccess) return FLEX_ECUDA;
+        if (cudaStreamSynchronize(s) != cudaSuccess) return FLEX_ECUDA;
+        return h.status;
+    }
+    return cudaGetLastError() == cudaSuccess ? FLEX_OK : FLEX_ECUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,49 @@
+// Internal declarations shared by the host API and the kernel translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "flexattn.h"
+
+namespace flex {
+
+// Workspace layout.  The first 256 bytes hold control words; the rest is scratch whose
+// meaning depends on the entry point.
+struct WsHeader {
+    int status;          // FLEX_OK or FLEX_ETIMEOUT, set by kernels, cleared by check
+    int timeout_where;   // diagnostic: which wait gave up
+    unsigned int ticket; // dynamic work counter of persistent kernels
+    unsigned int pad[61];
+};
+static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
+
+struct Problem {
+    int B, H, N, d, M;
+    int bf16;       // storage type of activations: 1 = bf16, 0 = fp32
+    int nonstat;    // 1 = nonstationary (W2 given)
+    int causal;
+};
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// ---- SIMT path (fp32 arithmetic; any supported dtype) --------------------------------
+size_t simt_fwd_smem_bytes(const Problem& p, int chunk);
+size_t simt_bwd_smem_bytes(const Problem& p, int chunk);
+int simt_pick_chunk_fwd(const Problem& p);   // 0 if nothing fits
+int simt_pick_chunk_bwd(const Problem& p);
+size_t simt_bwd_ws_bytes(const Problem& p);
+
+cudaError_t launch_featmap(const Problem& p, const void* x, const float* W1, const float* W2,
+                           void* phi, cudaStream_t s);
+cudaError_t launch_simt_fwd(const Problem& p, const void* q, const void* k, const void* v,
+                            const float* W1, const float* W2, void* out, float* den,
+                            cudaStream_t s);
+cudaError_t launch_simt_bwd(const Problem& p, const void* q, const void* k, const void* v,
+                            const float* W1, const float* W2, const void* out,
+                            const float* den, const void* dout, void* dq, void* dk, void* dv,
+                            float* dW1, float* dW2, void* scratch, cudaStream_t s);
+
+}  // namespace flex

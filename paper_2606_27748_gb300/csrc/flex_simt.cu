@@ -1,0 +1,615 @@
+// SIMT kernels: fp32 arithmetic on the CUDA cores, one CTA per (b, h) sequence.
+//
+// These kernels serve the fp32 storage type, whose tolerance (relative L2 <= 1e-4)
+// excludes bf16/tf32 tensor-core operands, and the feature-map entry point.  They run the
+// chunked form of Eq. (linear att): inside a chunk of C tokens the masked C x C kernel
+// matrix phi(Q) phi(K)^T is applied directly, across chunks the running state
+// S = sum phi(k) v^T and z = sum phi(k) carries the prefix.  z rides in S as column d
+// (v is extended with a constant 1), so numerator and denominator share every product.
+//
+// Inside the attention kernels the features are unscaled, phi' = [cos, sin] (times cos w
+// for the nonstationary map): the global factor M^{-1/2} of Eq. phi_n / phi_non cancels in
+// out and in every gradient, and only the stored denominator is rescaled, den = den'/M.
+#include "flex_internal.h"
+
+#include <math.h>
+
+#include <algorithm>
+
+namespace flex {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kMaxDwPerThread = 64;  // Mc * d <= kThreads * 64
+
+__device__ __forceinline__ float load_act(const float* p, size_t i) { return p[i]; }
+__device__ __forceinline__ float load_act(const __nv_bfloat16* p, size_t i)
+{
+    return __bfloat162float(p[i]);
+}
+__device__ __forceinline__ void store_act(float* p, size_t i, float x) { p[i] = x; }
+__device__ __forceinline__ void store_act(__nv_bfloat16* p, size_t i, float x)
+{
+    p[i] = __float2bfloat16_rn(x);
+}
+
+// Projection rows of one head into shared memory, row stride d + 1:
+// stationary: W1 (M rows); nonstationary: U = (W1+W2)/2 then V = (W1-W2)/2 (2M rows).
+__device__ void load_projection(const Problem& p, const float* W1, const float* W2, int h,
+                                float* W)
+{
+    const int d = p.d, M = p.M;
+    const float* w1 = W1 + (size_t)h * M * d;
+    const float* w2 = p.nonstat ? W2 + (size_t)h * M * d : nullptr;
+    for (int idx = threadIdx.x; idx < M * d; idx += blockDim.x) {
+        int m = idx / d, i = idx % d;
+        if (!p.nonstat) {
+            W[m * (d + 1) + i] = w1[idx];
+        } else {
+            W[m * (d + 1) + i] = 0.5f * (w1[idx] + w2[idx]);
+            W[(M + m) * (d + 1) + i] = 0.5f * (w1[idx] - w2[idx]);
+        }
+    }
+}
+
+template <typename T>
+__device__ void load_rows(const T* src, size_t base, int rows, int d, float* dst, int stride)
+{
+    for (int idx = threadIdx.x; idx < rows * d; idx += blockDim.x) {
+        int t = idx / d, i = idx % d;
+        dst[t * stride + i] = load_act(src, base + (size_t)t * d + i);
+    }
+}
+
+// Unscaled features of `rows` vectors X[t][0..d) into P[t][0..2M), row stride pstride.
+__device__ void features(const Problem& p, const float* X, int rows, const float* W, float* P,
+                         int pstride)
+{
+    const int d = p.d, M = p.M;
+    for (int idx = threadIdx.x; idx < rows * M; idx += blockDim.x) {
+        int t = idx / M, m = idx % M;
+        const float* x = X + t * d;
+        const float* wa = W + m * (d + 1);
+        float a = 0.f;
+        for (int i = 0; i < d; ++i) a = fmaf(x[i], wa[i], a);
+        float sa, ca;
+        sincosf(a, &sa, &ca);
+        if (!p.nonstat) {
+            P[t * pstride + m] = ca;
+            P[t * pstride + M + m] = sa;
+        } else {
+            const float* wb = W + (M + m) * (d + 1);
+            float w = 0.f;
+            for (int i = 0; i < d; ++i) w = fmaf(x[i], wb[i], w);
+            float cw = cosf(w);
+            P[t * pstride + m] = ca * cw;
+            P[t * pstride + M + m] = sa * cw;
+        }
+    }
+}
+
+// ------------------------------------------------------------------------------------
+// Feature map entry point (writes phi, scaled by M^{-1/2}).
+// ------------------------------------------------------------------------------------
+template <typename T>
+__global__ void featmap_kernel(Problem p, const T* x, const float* W1, const float* W2, T* phi,
+                               float scale)
+{
+    const int d = p.d, M = p.M;
+    const size_t rows = (size_t)p.B * p.H * p.N;
+    for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < rows * M;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        size_t row = idx / M;
+        int m = (int)(idx % M);
+        int h = (int)((row / p.N) % p.H);
+        const float* w1 = W1 + ((size_t)h * M + m) * d;
+        float a = 0.f, w = 0.f;
+        if (!p.nonstat) {
+            for (int i = 0; i < d; ++i) a = fmaf(load_act(x, row * d + i), w1[i], a);
+        } else {
+            const float* w2 = W2 + ((size_t)h * M + m) * d;
+            for (int i = 0; i < d; ++i) {
+                float xi = load_act(x, row * d + i);
+                a = fmaf(xi, 0.5f * (w1[i] + w2[i]), a);
+                w = fmaf(xi, 0.5f * (w1[i] - w2[i]), w);
+            }
+        }
+        float sa, ca;
+        sincosf(a, &sa, &ca);
+        float cw = p.nonstat ? cosf(w) : 1.f;
+        store_act(phi, row * 2 * M + m, scale * ca * cw);
+        store_act(phi, row * 2 * M + M + m, scale * sa * cw);
+    }
+}
+
+// ------------------------------------------------------------------------------------
+// Forward.
+// ------------------------------------------------------------------------------------
+struct FwdLayout {
+    size_t W, S, Xq, Xk, Vx, Pq, Pk, A, O, total;  // offsets in floats
+};
+
+__host__ __device__ inline FwdLayout fwd_layout(const Problem& p, int C)
+{
+    const int d = p.d, D = 2 * p.M, Mc = p.nonstat ? 2 * p.M : p.M;
+    FwdLayout L;
+    size_t o = 0;
+    L.W = o;  o += (size_t)Mc * (d + 1);
+    L.S = o;  o += (size_t)D * (d + 1);
+    L.Xq = o; o += (size_t)C * d;
+    L.Xk = o; o += (size_t)C * d;
+    L.Vx = o; o += (size_t)C * (d + 1);
+    L.Pq = o; o += (size_t)C * (D + 1);
+    L.Pk = o; o += (size_t)C * (D + 1);
+    L.A = o;  o += (size_t)C * C;
+    L.O = o;  o += (size_t)C * (d + 1);
+    L.total = o;
+    return L;
+}
+
+// S[f][e] += sum_{j < rows} Pk[j][f] * Vx[j][e]
+__device__ void state_update(const float* Pk, const float* Vx, int rows, int D, int d,
+                             float* S)
+{
+    for (int idx = threadIdx.x; idx < D * (d + 1); idx += blockDim.x) {
+        int f = idx / (d + 1), e = idx % (d + 1);
+        float acc = S[idx];
+        for (int j = 0; j < rows; ++j) acc = fmaf(Pk[j * (D + 1) + f], Vx[j * (d + 1) + e], acc);
+        S[idx] = acc;
+    }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) simt_fwd_kernel(Problem p, int C, const T* q,
+                                                            const T* k, const T* v,
+                                                            const float* W1, const float* W2,
+                                                            T* out, float* den)
+{
+    extern __shared__ float sm[];
+    const int d = p.d, D = 2 * p.M, N = p.N;
+    const int bh = blockIdx.x, h = bh % p.H;
+    const size_t base = (size_t)bh * N * d;
+    const FwdLayout L = fwd_layout(p, C);
+    float *W = sm + L.W, *S = sm + L.S, *Xq = sm + L.Xq, *Xk = sm + L.Xk, *Vx = sm + L.Vx;
+    float *Pq = sm + L.Pq, *Pk = sm + L.Pk, *A = sm + L.A, *O = sm + L.O;
+    const float inv_m = 1.0f / (float)p.M;
+
+    load_projection(p, W1, W2, h, W);
+    for (int idx = threadIdx.x; idx < D * (d + 1); idx += blockDim.x) S[idx] = 0.f;
+    for (int idx = threadIdx.x; idx < C; idx += blockDim.x) Vx[idx * (d + 1) + d] = 1.f;
+    __syncthreads();
+
+    if (!p.causal) {  // totals S, z over the whole sequence first
+        for (int t0 = 0; t0 < N; t0 += C) {
+            const int CL = min(C, N - t0);
+            load_rows(k, base + (size_t)t0 * d, CL, d, Xk, d);
+            load_rows(v, base + (size_t)t0 * d, CL, d, Vx, d + 1);
+            __syncthreads();
+            features(p, Xk, CL, W, Pk, D + 1);
+            __syncthreads();
+            state_update(Pk, Vx, CL, D, d, S);
+            __syncthreads();
+        }
+    }
+    for (int t0 = 0; t0 < N; t0 += C) {
+        const int CL = min(C, N - t0);
+        load_rows(q, base + (size_t)t0 * d, CL, d, Xq, d);
+        if (p.causal) {
+            load_rows(k, base + (size_t)t0 * d, CL, d, Xk, d);
+            load_rows(v, base + (size_t)t0 * d, CL, d, Vx, d + 1);
+        }
+        __syncthreads();
+        features(p, Xq, CL, W, Pq, D + 1);
+        if (p.causal) features(p, Xk, CL, W, Pk, D + 1);
+        __syncthreads();
+        if (p.causal) {
+            for (int idx = threadIdx.x; idx < CL * CL; idx += blockDim.x) {
+                int i = idx / CL, j = idx % CL;
+                float a = 0.f;
+                if (j <= i)
+                    for (int f = 0; f < D; ++f) a = fmaf(Pq[i * (D + 1) + f], Pk[j * (D + 1) + f], a);
+                A[i * C + j] = a;
+            }
+            __syncthreads();
+        }
+        // numerator (columns < d) and denominator (column d) of every row of the chunk
+        for (int idx = threadIdx.x; idx < CL * (d + 1); idx += blockDim.x) {
+            int i = idx / (d + 1), e = idx % (d + 1);
+            float acc = 0.f;
+            if (p.causal)
+                for (int j = 0; j <= i; ++j) acc = fmaf(A[i * C + j], Vx[j * (d + 1) + e], acc);
+            for (int f = 0; f < D; ++f) acc = fmaf(Pq[i * (D + 1) + f], S[f * (d + 1) + e], acc);
+            O[i * (d + 1) + e] = acc;
+        }
+        __syncthreads();
+        for (int idx = threadIdx.x; idx < CL * d; idx += blockDim.x) {
+            int i = idx / d, e = idx % d;
+            store_act(out, base + (size_t)(t0 + i) * d + e, O[i * (d + 1) + e] / O[i * (d + 1) + d]);
+        }
+        if (den)
+            for (int i = threadIdx.x; i < CL; i += blockDim.x)
+                den[(size_t)bh * N + t0 + i] = O[i * (d + 1) + d] * inv_m;
+        if (p.causal) state_update(Pk, Vx, CL, D, d, S);
+        __syncthreads();
+    }
+}
+
+// ------------------------------------------------------------------------------------
+// Backward.
+// ------------------------------------------------------------------------------------
+struct BwdLayout {
+    size_t W, S, Xq, Xk, Vx, Gx, Pq, Pk, dP, A, dA, dAct, total;
+};
+
+__host__ __device__ inline BwdLayout bwd_layout(const Problem& p, int C)
+{
+    const int d = p.d, D = 2 * p.M, Mc = p.nonstat ? 2 * p.M : p.M;
+    BwdLayout L;
+    size_t o = 0;
+    L.W = o;    o += (size_t)Mc * (d + 1);
+    L.S = o;    o += (size_t)D * (d + 1);
+    L.Xq = o;   o += (size_t)C * d;
+    L.Xk = o;   o += (size_t)C * d;
+    L.Vx = o;   o += (size_t)C * (d + 1);
+    L.Gx = o;   o += (size_t)C * (d + 1);
+    L.Pq = o;   o += (size_t)C * (D + 1);
+    L.Pk = o;   o += (size_t)C * (D + 1);
+    L.dP = o;   o += (size_t)C * (D + 1);
+    L.A = o;    o += (size_t)C * C;
+    L.dA = o;   o += (size_t)C * C;
+    L.dAct = o; o += (size_t)C * (Mc + 1);
+    L.total = o;
+    return L;
+}
+
+// Gx[t] = [dout_t / den'_t, -(dout_t . out_t) / den'_t] with den' = M * den.
+template <typename T>
+__device__ void load_upstream(const Problem& p, const T* dout, const T* out, const float* den,
+                              size_t base, size_t den_base, int rows, float* Gx)
+{
+    const int d = p.d;
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32, nwarps = blockDim.x / 32;
+    for (int t = warp; t < rows; t += nwarps) {
+        const float dn = den[den_base + t] * (float)p.M;
+        float s = 0.f;
+        for (int e = lane; e < d; e += 32) {
+            float g = load_act(dout, base + (size_t)t * d + e);
+            s = fmaf(g, load_act(out, base + (size_t)t * d + e), s);
+            Gx[t * (d + 1) + e] = g / dn;
+        }
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (lane == 0) Gx[t * (d + 1) + d] = -s / dn;
+    }
+}
+
+// Chain rule through the feature map: dAct[t][m] = d/da (stationary) or (du, dw).
+__device__ void feature_backward(const Problem& p, const float* X, const float* P,
+                                 const float* dP, int rows, const float* W, float* dAct)
+{
+    const int d = p.d, M = p.M, D = 2 * M, Mc = p.nonstat ? 2 * M : M;
+    for (int idx = threadIdx.x; idx < rows * M; idx += blockDim.x) {
+        int t = idx / M, m = idx % M;
+        const float dc = dP[t * (D + 1) + m], ds = dP[t * (D + 1) + M + m];
+        if (!p.nonstat) {
+            const float c = P[t * (D + 1) + m], s = P[t * (D + 1) + M + m];
+            dAct[t * (Mc + 1) + m] = -s * dc + c * ds;
+        } else {
+            const float* x = X + t * d;
+            const float *wa = W + m * (d + 1), *wb = W + (M + m) * (d + 1);
+            float u = 0.f, w = 0.f;
+            for (int i = 0; i < d; ++i) {
+                u = fmaf(x[i], wa[i], u);
+                w = fmaf(x[i], wb[i], w);
+            }
+            float su, cu, sw, cw;
+            sincosf(u, &su, &cu);
+            sincosf(w, &sw, &cw);
+            dAct[t * (Mc + 1) + m] = cw * (-su * dc + cu * ds);
+            dAct[t * (Mc + 1) + M + m] = -sw * (cu * dc + su * ds);
+        }
+    }
+}
+
+// dx[t][i] = sum_m dAct[t][m] W[m][i]; dW[m][i] += sum_t dAct[t][m] X[t][i].
+template <typename T>
+__device__ void project_back(const Problem& p, const float* X, const float* dAct, int rows,
+                             const float* W, T* dx, size_t base, float* dw_acc)
+{
+    const int d = p.d, Mc = p.nonstat ? 2 * p.M : p.M;
+    for (int idx = threadIdx.x; idx < rows * d; idx += blockDim.x) {
+        int t = idx / d, i = idx % d;
+        float acc = 0.f;
+        for (int m = 0; m < Mc; ++m) acc = fmaf(dAct[t * (Mc + 1) + m], W[m * (d + 1) + i], acc);
+        store_act(dx, base + (size_t)t * d + i, acc);
+    }
+#pragma unroll
+    for (int r = 0; r < kMaxDwPerThread; ++r) {
+        int e = r * kThreads + threadIdx.x;
+        if (e < Mc * d) {
+            int m = e / d, i = e % d;
+            float acc = dw_acc[r];
+            for (int t = 0; t < rows; ++t) acc = fmaf(dAct[t * (Mc + 1) + m], X[t * d + i], acc);
+            dw_acc[r] = acc;
+        }
+    }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
+    Problem p, int C, const T* q, const T* k, const T* v, const float* W1, const float* W2,
+    const T* out, const float* den, const T* dout, T* dq, T* dk, T* dv, float* dw_part)
+{
+    extern __shared__ float sm[];
+    const int d = p.d, D = 2 * p.M, N = p.N, Mc = p.nonstat ? 2 * p.M : p.M;
+    const int bh = blockIdx.x, h = bh % p.H;
+    const size_t base = (size_t)bh * N * d, den_base = (size_t)bh * N;
+    const BwdLayout L = bwd_layout(p, C);
+    float *W = sm + L.W, *S = sm + L.S, *Xq = sm + L.Xq, *Xk = sm + L.Xk, *Vx = sm + L.Vx;
+    float *Gx = sm + L.Gx, *Pq = sm + L.Pq, *Pk = sm + L.Pk, *dP = sm + L.dP;
+    float *A = sm + L.A, *dA = sm + L.dA, *dAct = sm + L.dAct;
+
+    float dw_acc[kMaxDwPerThread];
+#pragma unroll
+    for (int r = 0; r < kMaxDwPerThread; ++r) dw_acc[r] = 0.f;
+
+    load_projection(p, W1, W2, h, W);
+    for (int idx = threadIdx.x; idx < D * (d + 1); idx += blockDim.x) S[idx] = 0.f;
+    for (int idx = threadIdx.x; idx < C; idx += blockDim.x) Vx[idx * (d + 1) + d] = 1.f;
+    __syncthreads();
+
+    // ---- dq: forward direction with S_i, z_i ----
+    if (!p.causal) {
+        for (int t0 = 0; t0 < N; t0 += C) {
+            const int CL = min(C, N - t0);
+            load_rows(k, base + (size_t)t0 * d, CL, d, Xk, d);
+            load_rows(v, base + (size_t)t0 * d, CL, d, Vx, d + 1);
+            __syncthreads();
+            features(p, Xk, CL, W, Pk, D + 1);
+            __syncthreads();
+            state_update(Pk, Vx, CL, D, d, S);
+            __syncthreads();
+        }
+    }
+    for (int t0 = 0; t0 < N; t0 += C) {
+        const int CL = min(C, N - t0);
+        const size_t off = base + (size_t)t0 * d;
+        load_rows(q, off, CL, d, Xq, d);
+        load_upstream(p, dout, out, den, off, den_base + t0, CL, Gx);
+        if (p.causal) {
+            load_rows(k, off, CL, d, Xk, d);
+            load_rows(v, off, CL, d, Vx, d + 1);
+        }
+        __syncthreads();
+        features(p, Xq, CL, W, Pq, D + 1);
+        if (p.causal) features(p, Xk, CL, W, Pk, D + 1);
+        if (p.causal)
+            for (int idx = threadIdx.x; idx < CL * CL; idx += blockDim.x) {
+                int i = idx / CL, j = idx % CL;
+                float a = 0.f;
+                if (j <= i)
+                    for (int e = 0; e <= d; ++e) a = fmaf(Gx[i * (d + 1) + e], Vx[j * (d + 1) + e], a);
+                dA[i * C + j] = a;
+            }
+        __syncthreads();
+        for (int idx = threadIdx.x; idx < CL * D; idx += blockDim.x) {
+            int i = idx / D, f = idx % D;
+            float acc = 0.f;
+            if (p.causal)
+                for (int j = 0; j <= i; ++j) acc = fmaf(dA[i * C + j], Pk[j * (D + 1) + f], acc);
+            for (int e = 0; e <= d; ++e) acc = fmaf(S[f * (d + 1) + e], Gx[i * (d + 1) + e], acc);
+            dP[i * (D + 1) + f] = acc;
+        }
+        __syncthreads();
+        if (p.causal) state_update(Pk, Vx, CL, D, d, S);
+        feature_backward(p, Xq, Pq, dP, CL, W, dAct);
+        __syncthreads();
+        project_back(p, Xq, dAct, CL, W, dq, off, dw_acc);
+        __syncthreads();
+    }
+
+    // ---- dk, dv: reverse direction with R_j, r_j (S's buffer is reused for R) ----
+    for (int idx = threadIdx.x; idx < D * (d + 1); idx += blockDim.x) S[idx] = 0.f;
+    __syncthreads();
+    float* R = S;
+    if (!p.causal) {
+        for (int t0 = 0; t0 < N; t0 += C) {
+            const int CL = min(C, N - t0);
+            const size_t off = base + (size_t)t0 * d;
+            load_rows(q, off, CL, d, Xq, d);
+            load_upstream(p, dout, out, den, off, den_base + t0, CL, Gx);
+            __syncthreads();
+            features(p, Xq, CL, W, Pq, D + 1);
+            __syncthreads();
+            state_update(Pq, Gx, CL, D, d, R);
+            __syncthreads();
+        }
+    }
+    const int nchunks = (N + C - 1) / C;
+    for (int c = nchunks - 1; c >= 0; --c) {
+        const int t0 = c * C, CL = min(C, N - t0);
+        const size_t off = base + (size_t)t0 * d;
+        load_rows(k, off, CL, d, Xk, d);
+        load_rows(v, off, CL, d, Vx, d + 1);
+        if (p.causal) {
+            load_rows(q, off, CL, d, Xq, d);
+            load_upstream(p, dout, out, den, off, den_base + t0, CL, Gx);
+        }
+        __syncthreads();
+        features(p, Xk, CL, W, Pk, D + 1);
+        if (p.causal) features(p, Xq, CL, W, Pq, D + 1);
+        __syncthreads();
+        if (p.causal)
+            for (int idx = threadIdx.x; idx < CL * CL; idx += blockDim.x) {
+                int i = idx / CL, j = idx % CL;
+                float a = 0.f, da = 0.f;
+                if (j <= i) {
+                    for (int f = 0; f < D; ++f) a = fmaf(Pq[i * (D + 1) + f], Pk[j * (D + 1) + f], a);
+                    for (int e = 0; e <= d; ++e) da = fmaf(Gx[i * (d + 1) + e], Vx[j * (d + 1) + e], da);
+                }
+                A[i * C + j] = a;
+                dA[i * C + j] = da;
+            }
+        __syncthreads();
+        for (int idx = threadIdx.x; idx < CL * D; idx += blockDim.x) {
+            int j = idx / D, f = idx % D;
+            float acc = 0.f;
+            if (p.causal)
+                for (int i = j; i < CL; ++i) acc = fmaf(dA[i * C + j], Pq[i * (D + 1) + f], acc);
+            for (int e = 0; e <= d; ++e) acc = fmaf(R[f * (d + 1) + e], Vx[j * (d + 1) + e], acc);
+            dP[j * (D + 1) + f] = acc;
+        }
+        for (int idx = threadIdx.x; idx < CL * d; idx += blockDim.x) {
+            int j = idx / d, e = idx % d;
+            float acc = 0.f;
+            if (p.causal)
+                for (int i = j; i < CL; ++i) acc = fmaf(A[i * C + j], Gx[i * (d + 1) + e], acc);
+            for (int f = 0; f < D; ++f) acc = fmaf(R[f * (d + 1) + e], Pk[j * (D + 1) + f], acc);
+            store_act(dv, off + (size_t)j * d + e, acc);
+        }
+        __syncthreads();
+        if (p.causal) state_update(Pq, Gx, CL, D, d, R);
+        feature_backward(p, Xk, Pk, dP, CL, W, dAct);
+        __syncthreads();
+        project_back(p, Xk, dAct, CL, W, dk, off, dw_acc);
+        __syncthreads();
+    }
+
+    float* part = dw_part + (size_t)bh * Mc * d;
+#pragma unroll
+    for (int r = 0; r < kMaxDwPerThread; ++r) {
+        int e = r * kThreads + threadIdx.x;
+        if (e < Mc * d) part[e] = dw_acc[r];
+    }
+}
+
+// dW over the batch, in a fixed order (deterministic).  Nonstationary: the partials hold
+// dU (rows < M) and dV (rows >= M); dW1 = (dU + dV)/2, dW2 = (dU - dV)/2.
+__global__ void dw_reduce_kernel(Problem p, const float* part, float* dW1, float* dW2)
+{
+    const int d = p.d, M = p.M, Mc = p.nonstat ? 2 * M : M;
+    const size_t per = (size_t)M * d;
+    for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < (size_t)p.H * per;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        int h = (int)(idx / per);
+        size_t e = idx % per;
+        float a = 0.f, b = 0.f;
+        for (int bb = 0; bb < p.B; ++bb) {
+            const float* pp = part + ((size_t)bb * p.H + h) * Mc * d;
+            a += pp[e];
+            if (p.nonstat) b += pp[per + e];
+        }
+        if (!p.nonstat) {
+            dW1[idx] = a;
+        } else {
+            dW1[idx] = 0.5f * (a + b);
+            dW2[idx] = 0.5f * (a - b);
+        }
+    }
+}
+
+}  // namespace
+
+size_t simt_fwd_smem_bytes(const Problem& p, int chunk)
+{
+    return fwd_layout(p, chunk).total * sizeof(float);
+}
+
+size_t simt_bwd_smem_bytes(const Problem& p, int chunk)
+{
+    return bwd_layout(p, chunk).total * sizeof(float);
+}
+
+static const size_t kSmemLimit = 227 * 1024;
+
+int simt_pick_chunk_fwd(const Problem& p)
+{
+    for (int c : {32, 16, 8})
+        if (simt_fwd_smem_bytes(p, c) <= kSmemLimit) return c;
+    return 0;
+}
+
+int simt_pick_chunk_bwd(const Problem& p)
+{
+    const int Mc = p.nonstat ? 2 * p.M : p.M;
+    if ((size_t)Mc * p.d > (size_t)kThreads * kMaxDwPerThread) return 0;
+    for (int c : {32, 16, 8})
+        if (simt_bwd_smem_bytes(p, c) <= kSmemLimit) return c;
+    return 0;
+}
+
+size_t simt_bwd_ws_bytes(const Problem& p)
+{
+    const int Mc = p.nonstat ? 2 * p.M : p.M;
+    return (size_t)p.B * p.H * Mc * p.d * sizeof(float);
+}
+
+cudaError_t launch_featmap(const Problem& p, const void* x, const float* W1, const float* W2,
+                           void* phi, cudaStream_t s)
+{
+    const size_t work = (size_t)p.B * p.H * p.N * p.M;
+    const int blocks = (int)std::min<size_t>((work + kThreads - 1) / kThreads, 152 * 16);
+    const float scale = 1.0f / sqrtf((float)p.M);
+    if (p.bf16)
+        featmap_kernel<<<blocks, kThreads, 0, s>>>(p, (const __nv_bfloat16*)x, W1, W2,
+                                                   (__nv_bfloat16*)phi, scale);
+    else
+        featmap_kernel<<<blocks, kThreads, 0, s>>>(p, (const float*)x, W1, W2, (float*)phi,
+                                                   scale);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_simt_fwd(const Problem& p, const void* q, const void* k, const void* v,
+                            const float* W1, const float* W2, void* out, float* den,
+                            cudaStream_t s)
+{
+    const int C = simt_pick_chunk_fwd(p);
+    const size_t smem = simt_fwd_smem_bytes(p, C);
+    const int grid = p.B * p.H;
+    if (p.bf16) {
+        auto kern = simt_fwd_kernel<__nv_bfloat16>;
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        kern<<<grid, kThreads, smem, s>>>(p, C, (const __nv_bfloat16*)q,
+                                          (const __nv_bfloat16*)k, (const __nv_bfloat16*)v, W1,
+                                          W2, (__nv_bfloat16*)out, den);
+    } else {
+        auto kern = simt_fwd_kernel<float>;
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        kern<<<grid, kThreads, smem, s>>>(p, C, (const float*)q, (const float*)k,
+                                          (const float*)v, W1, W2, (float*)out, den);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_simt_bwd(const Problem& p, const void* q, const void* k, const void* v,
+                            const float* W1, const float* W2, const void* out,
+                            const float* den, const void* dout, void* dq, void* dk, void* dv,
+                            float* dW1, float* dW2, void* scratch, cudaStream_t s)
+{
+    const int C = simt_pick_chunk_bwd(p);
+    const size_t smem = simt_bwd_smem_bytes(p, C);
+    const int grid = p.B * p.H;
+    float* part = (float*)scratch;
+    if (p.bf16) {
+        typedef __nv_bfloat16 T;
+        auto kern = simt_bwd_kernel<T>;
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        kern<<<grid, kThreads, smem, s>>>(p, C, (const T*)q, (const T*)k, (const T*)v, W1, W2,
+                                          (const T*)out, den, (const T*)dout, (T*)dq, (T*)dk,
+                                          (T*)dv, part);
+    } else {
+        typedef float T;
+        auto kern = simt_bwd_kernel<T>;
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        kern<<<grid, kThreads, smem, s>>>(p, C, (const T*)q, (const T*)k, (const T*)v, W1, W2,
+                                          (const T*)out, den, (const T*)dout, (T*)dq, (T*)dk,
+                                          (T*)dv, part);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const size_t work = (size_t)p.H * p.M * p.d;
+    const int blocks = (int)std::min<size_t>((work + kThreads - 1) / kThreads, 152 * 8);
+    dw_reduce_kernel<<<blocks, kThreads, 0, s>>>(p, part, dW1, dW2);
+    return cudaGetLastError();
+}
+
+}  // namespace flex

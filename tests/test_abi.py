@@ -1,0 +1,73 @@
+"""The C-ABI library: it builds for sm_103a, loads, exports every declared entry point,
+and rejects bad arguments on the host (no GPU needed: no compute call is made)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADERS = [os.path.join(ROOT, "include", f) for f in os.listdir(os.path.join(ROOT, "include"))
+           if f.endswith(".h")]
+
+
+def declared_functions():
+    names = set()
+    for h in HEADERS:
+        text = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names |= set(re.findall(r"^[A-Za-z_][\w\s\*]*?\b(flex_\w+)\s*\(", text, flags=re.M))
+    return sorted(names)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2606_27748_gb300 import build, flexattn
+    build.build()
+    return flexattn.load()
+
+
+def test_header_declares_the_entry_points():
+    names = declared_functions()
+    for n in ("flex_featmap", "flex_linattn_fwd", "flex_linattn_bwd", "flex_check_status",
+              "flex_workspace_bytes", "flex_strerror"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_binding_names_match_header():
+    from paper_2606_27748_gb300 import flexattn
+    assert set(flexattn.EXPORTS) <= set(declared_functions())
+
+
+def test_host_validation_without_gpu(lib):
+    from paper_2606_27748_gb300.flexattn import FlexShape, FLEX_EINVAL, FLEX_EWORKSPACE
+    ok = FlexShape(2, 3, 100, 64, 64, 1)
+    assert lib.flex_workspace_bytes(ctypes.byref(ok), 1, 0) >= 256
+    assert lib.flex_workspace_bytes(ctypes.byref(ok), 1, 1) > lib.flex_workspace_bytes(
+        ctypes.byref(ok), 1, 0)
+    bad = FlexShape(2, 3, 0, 64, 64, 1)
+    assert lib.flex_workspace_bytes(ctypes.byref(bad), 1, 0) == 0
+    p = ctypes.c_void_p(4096)  # never dereferenced: validation fails first
+    # null shape / N < 1 / null input
+    assert lib.flex_linattn_fwd(None, p, p, p, p, None, 1, p, None, p, 1 << 20, None) == FLEX_EINVAL
+    assert lib.flex_linattn_fwd(ctypes.byref(bad), p, p, p, p, None, 1, p, None, p, 1 << 20,
+                                None) == FLEX_EINVAL
+    assert lib.flex_linattn_fwd(ctypes.byref(ok), None, p, p, p, None, 1, p, None, p, 1 << 20,
+                                None) == FLEX_EINVAL
+    # misaligned pointer
+    mis = ctypes.c_void_p(4096 + 2)
+    assert lib.flex_linattn_fwd(ctypes.byref(ok), mis, p, p, p, None, 1, p, None, p, 1 << 20,
+                                None) == FLEX_EINVAL
+    # workspace too small
+    assert lib.flex_linattn_fwd(ctypes.byref(ok), p, p, p, p, None, 1, p, None, p, 16,
+                                None) == FLEX_EWORKSPACE
+    # W2 given without dW2 (and the reverse)
+    args = [p] * 3 + [p, p, 1, p, p, p, p, p, p, p]
+    assert lib.flex_linattn_bwd(ctypes.byref(ok), *args, None, p, 1 << 24, None) == FLEX_EINVAL
+    args = [p] * 3 + [p, None, 1, p, p, p, p, p, p, p]
+    assert lib.flex_linattn_bwd(ctypes.byref(ok), *args, p, p, 1 << 24, None) == FLEX_EINVAL
+    assert lib.flex_strerror(FLEX_EINVAL)
