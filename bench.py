@@ -32,7 +32,7 @@ sys.path.insert(0, ROOT)
 from paper_2606_27748_gb300 import workloads  # noqa: E402
 
 METRIC = "RFF linear-attn fwd tokens/s (N=16K causal) & % of bf16 tensor/HBM roofline"
-L2_BYTES = 129 * 1024 * 1024
+L2_BYTES = 129e6
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
