@@ -110,8 +110,11 @@ int flex_linattn_fwd(const flex_shape* shape, const void* q, const void* k, cons
         if (!aligned(t, 16)) return FLEX_EINVAL;
     if ((W2 && !aligned(W2, 16)) || (den && !aligned(den, 16))) return FLEX_EINVAL;
     if ((rc = check_ws(ws, ws_bytes, fwd_ws_bytes(p)))) return rc;
-    if (flex::simt_pick_chunk_fwd(p) == 0) return FLEX_EUNSUPPORTED;
     cudaStream_t s = (cudaStream_t)stream;
+    int* status = &((flex::WsHeader*)ws)->status;
+    if (flex::tc_fwd_supported(p))
+        return count(1, flex::launch_tc_fwd(p, q, k, v, W1, W2, out, den, status, s));
+    if (flex::simt_pick_chunk_fwd(p) == 0) return FLEX_EUNSUPPORTED;
     return count(1, flex::launch_simt_fwd(p, q, k, v, W1, W2, out, den, s));
 }
 

@@ -46,4 +46,10 @@ cudaError_t launch_simt_bwd(const Problem& p, const void* q, const void* k, cons
                             const float* den, const void* dout, void* dq, void* dk, void* dv,
                             float* dW1, float* dW2, void* scratch, cudaStream_t s);
 
+// ---- tensor-core path (bf16 storage, d = 64, M in {64, 128}) ------------------------
+bool tc_fwd_supported(const Problem& p);
+cudaError_t launch_tc_fwd(const Problem& p, const void* q, const void* k, const void* v,
+                          const float* W1, const float* W2, void* out, float* den, int* status,
+                          cudaStream_t s);
+
 }  // namespace flex
