@@ -101,6 +101,25 @@ int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, cons
                      const float* den, const void* dout, void* dq, void* dk, void* dv,
                      float* dW1, float* dW2, void* ws, size_t ws_bytes, void* stream);
 
+/* flex_linattn_bwd without a workspace, for callers that cannot allocate device memory:
+ * for example a host framework whose memory pool owns all of the device's memory and
+ * passes its operators only input and output pointers, or a latency-critical path that
+ * must not call cudaMalloc/cudaFree, which can synchronise the device.  (The paper has
+ * no counterpart; this is a convenience of this library.)
+ * Same arguments, layouts and results as flex_linattn_bwd, minus ws and ws_bytes.  The
+ * scratch is one array of 4 MiB (2^20 floats) in the library's own device memory, which
+ * every GPU that loads the library keeps until the process exits; it must hold
+ * B * H * Mc * d floats (Mc = M, or 2M when W2 is given), else FLEX_EWORKSPACE is
+ * returned and nothing runs.  Nothing is allocated or freed.  All calls on a device
+ * share that array and it keeps the last call's contents, so two calls whose work may
+ * overlap on the GPU (different streams, or different host threads) race and must be
+ * ordered by the caller.  The first call on each device looks the array's address up
+ * (with that device current); make that first call before any stream capture. */
+int flex_linattn_bwd_noalloc(const flex_shape* shape, const void* q, const void* k,
+                             const void* v, const float* W1, const float* W2, int causal,
+                             const void* out, const float* den, const void* dout, void* dq,
+                             void* dk, void* dv, float* dW1, float* dW2, void* stream);
+
 /* Cumulative number of kernels this library has enqueued in this process (all entry
  * points, all devices).  Lets a caller count the launches inside a timed region. */
 unsigned long long flex_kernel_launches(void);
