@@ -7,20 +7,34 @@
 // tensor memory, the CUDA cores turn it into cos/sin features (Eq. phi_n, or the product
 // form of Eq. phi_non) and write them as bf16 MMA operands to shared memory.
 //
-// Features are processed in groups of 64 frequencies (128 features: 64 cos + 64 sin);
-// A, phi(Q) S and phi(Q) z accumulate over the groups, S and z are held per group.
-// Features are unscaled ([cos, sin] instead of M^{-1/2}[cos, sin]); the factor cancels in
-// the output and only the stored denominator is rescaled (den = den' / M).
+// Features are processed in groups of 64 frequencies (128 features: 64 cos + 64 sin); A,
+// phi(Q) S and phi(Q) z accumulate over the groups, S and z are held per group.  Features
+// are unscaled ([cos, sin] instead of M^{-1/2}[cos, sin]): the factor cancels in the
+// output, and only the stored denominator is rescaled (den = den' / M).
 //
-// One CTA (256 threads, 8 warps) per (b, h) sequence.  Thread 0 issues every MMA; all
-// threads take part in the CUDA-core phases.  Warps w and w+4 share TMEM lane quadrant
-// w % 4 and split the columns.
+// Warp roles (448 threads), handshakes on mbarriers:
+//   warp 0      TMA: q, k, v chunk tiles (128B swizzle) into shared memory
+//   warp 1      one thread issues every tcgen05.mma; owns the tensor-memory allocation
+//   warps 2-9   features: projection (TMEM) -> cos/sin -> bf16 phi tiles (shared memory);
+//               warps 2-5 take frequencies 0-31 of a group, warps 6-9 frequencies 32-63
+//   warps 10-13 epilogue: causal mask + bf16 of A (written back into TMEM as the A operand
+//               of A V), output rows, bf16 snapshot of S and z for the next chunk
+//
+// Sequence split: when there are SMs to spare, a sequence is cut into `splits` segments
+// handled by different CTAs with no waiting between them: the CTA of segment j first runs
+// a k-only pass over the chunks before its segment (projection + features of k and the
+// state update, no outputs) to build the state prefix, then its own chunks.  Segment
+// lengths halve from one segment to the next, which balances the work because a k-only
+// chunk costs about half a full chunk.
 //
 // Tensor memory (512 columns x 128 lanes, fp32):
 //   [0,128)    projection of one group (s: 64 cols a; n: 64 cols u, 64 cols w)
-//   [128,256)  A = phi(Q) phi(K)^T of the chunk (row = query, col = key)
+//   [128,256)  A = phi(Q) phi(K)^T (row = query, col = key); after the epilogue its first
+//              64 columns hold bf16(masked A), two keys per column
 //   [256,320)  numerator phi(Q) S + A V           [320,336) phi(Q) z (column 0)
 //   [336,336+64G)  S per group (lane = feature)   then 16 columns of z per group
+#include <cuda.h>
+
 #include "flex_internal.h"
 #include "tc_common.cuh"
 
@@ -28,24 +42,23 @@ namespace flex {
 namespace {
 using namespace tc;
 
-constexpr int kC = 128;   // tokens per chunk = MMA M
-constexpr int kThreadsTC = 256;
-constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz: a bounded wait
+constexpr int kC = 128;            // tokens per chunk = MMA M
+constexpr int kThreadsTC = 448;    // 14 warps
+constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kWarpEW = 10;
+constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz: every wait is bounded
+constexpr uint32_t kTileBytes = 128 * 128;       // one 128 x 64 bf16 tile
 
 template <bool NS, int G>
 struct Cfg {
     static constexpr int P = NS ? 128 : 64;  // projection columns per group
-    // shared memory offsets (bytes, 1024-aligned)
-    static constexpr uint32_t Q = 0, K = 16384, V = 32768;
-    static constexpr uint32_t W = 49152;
+    // shared memory offsets (bytes, 1024-aligned); X0/X1 hold q/k tiles
+    static constexpr uint32_t X0 = 0, X1 = 16384, V0 = 32768, V1 = 49152, ONES = 65536;
+    static constexpr uint32_t W = 69632;
     static constexpr uint32_t PQ = W + G * P * 128;
     static constexpr uint32_t PK = PQ + 32768;
     static constexpr uint32_t S = PK + 32768;
     static constexpr uint32_t Z = S + G * 16384;
-    static constexpr uint32_t ONES = Z + G * 4096;
-    static constexpr uint32_t A = ONES + 4096;
-    static constexpr uint32_t RS = A + 32768;
-    static constexpr uint32_t BYTES = RS + 1024;
+    static constexpr uint32_t BYTES = Z + G * 4096;
     // tensor memory columns
     static constexpr uint32_t T_P = 0, T_A = 128, T_O = 256, T_DN = 320, T_S = 336;
     static constexpr uint32_t T_Z = T_S + 64 * G;
@@ -53,11 +66,20 @@ struct Cfg {
     static_assert(BYTES + 1024 <= 232448, "shared memory budget");
 };
 
+struct Bars {
+    uint64_t x_full[2], x_free[2], v_full[2], v_free[2];
+    uint64_t p_full, p_free, phiq_full, phik_full, phi_free;
+    uint64_t attn_done, a_ready, o_ready, epi_done;
+};
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
 {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&v);
 }
+
+__device__ __forceinline__ float bf16_lo(uint32_t x) { return __uint_as_float(x << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t x) { return __uint_as_float(x & 0xFFFF0000u); }
 
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
                                              uint32_t d)
@@ -67,88 +89,38 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
                  : "memory");
 }
 
-// Waits for one MMA commit phase; the CTA agrees on the outcome (false = gave up).
-__device__ __forceinline__ bool wait_mma(uint64_t* mbar, uint32_t& phase, int* status)
+// Bounded wait on one mbarrier phase.  On a time-out the CTA is told to stop (abort flag)
+// and the status word records FLEX_ETIMEOUT; every other wait then returns at once.
+__device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                         int* status)
 {
-    bool ok = false;
+    if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     while (true) {
-        if (mbar_try_wait(mbar, phase)) { ok = true; break; }
-        if (clock64() - t0 > kWaitCycles) break;
-    }
-    phase ^= 1u;
-    if (!ok && (threadIdx.x & 31) == 0) atomicExch(status, (int)FLEX_ETIMEOUT);
-    const bool all_ok = !__syncthreads_or(!ok);
-    fence_after_sync();
-    return all_ok;
-}
-
-// Every thread: make its shared-memory writes visible to the tensor core and its tensor
-// memory reads complete, then meet the others.
-__device__ __forceinline__ void handoff_to_mma()
-{
-    fence_proxy_async();
-    fence_before_sync();
-    __syncthreads();
-}
-
-// Load rows [0, rows) of a [128 x 64] bf16 tile (row stride 64 elements) into a 128B-
-// swizzled shared tile; rows >= rows_valid are zero-filled.
-__device__ __forceinline__ void load_tile(const __nv_bfloat16* src, int rows_valid,
-                                          uint32_t dst)
-{
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int idx = threadIdx.x + kThreadsTC * i;
-        const int r = idx >> 3, c = idx & 7;
-        uint4 val = make_uint4(0, 0, 0, 0);
-        if (r < rows_valid) val = __ldg(reinterpret_cast<const uint4*>(src + r * 64 + c * 8));
-        st_shared_v4(dst + swz128(r, c * 8), val.x, val.y, val.z, val.w);
-    }
-}
-
-// Features of one group for one chunk: projection in TMEM -> bf16 phi tile (K-major,
-// block 0 = cos features, block 1 = sin features).  Thread: row t, frequencies
-// [32*wg, 32*wg + 32) of the group.
-template <bool NS>
-__device__ __forceinline__ void features_to_smem(uint32_t tm_row, int wg, int t, bool valid,
-                                                 uint32_t dst)
-{
-    float a[32], w[32];
-    tmem_ld16(tm_row + 32 * wg, *reinterpret_cast<float(*)[16]>(&a[0]));
-    tmem_ld16(tm_row + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
-    if (NS) {
-        tmem_ld16(tm_row + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]));
-        tmem_ld16(tm_row + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
-    }
-    tmem_wait_ld();
-    uint32_t pc[16], ps[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-        float s0, c0, s1, c1;
-        __sincosf(a[2 * i], &s0, &c0);
-        __sincosf(a[2 * i + 1], &s1, &c1);
-        if (NS) {
-            const float cw0 = __cosf(w[2 * i]), cw1 = __cosf(w[2 * i + 1]);
-            c0 *= cw0; s0 *= cw0; c1 *= cw1; s1 *= cw1;
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (clock64() - t0 > kWaitCycles) {
+            *abort_flag = 1;
+            atomicExch(status, (int)FLEX_ETIMEOUT);
+            return false;
         }
-        if (!valid) { c0 = s0 = c1 = s1 = 0.f; }
-        pc[i] = pack_bf16(c0, c1);
-        ps[i] = pack_bf16(s0, s1);
     }
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const uint32_t off = swz128(t, (4 * wg + j) * 8);
-        st_shared_v4(dst + off, pc[4 * j], pc[4 * j + 1], pc[4 * j + 2], pc[4 * j + 3]);
-        st_shared_v4(dst + 16384 + off, ps[4 * j], ps[4 * j + 1], ps[4 * j + 2], ps[4 * j + 3]);
-    }
+}
+
+// First chunk of segment j of `splits` (lengths proportional to 2^-j), rounded.
+__device__ __forceinline__ int segment_bound(int nch, int splits, int j)
+{
+    const long long den = (1LL << splits) - 1;
+    const long long num = (long long)nch * ((1LL << splits) - (1LL << (splits - j)));
+    return (int)((2 * num + den) / (2 * den));
 }
 
 template <bool NS, int G>
 __global__ void __launch_bounds__(kThreadsTC, 1)
-    tc_fwd_causal_kernel(int H, int N, int M, const __nv_bfloat16* __restrict__ q,
-                         const __nv_bfloat16* __restrict__ k,
-                         const __nv_bfloat16* __restrict__ v, const float* __restrict__ W1,
+    tc_fwd_causal_kernel(const __grid_constant__ CUtensorMap tmap_q,
+                         const __grid_constant__ CUtensorMap tmap_k,
+                         const __grid_constant__ CUtensorMap tmap_v, int H, int N, int M,
+                         int splits, const float* __restrict__ W1,
                          const float* __restrict__ W2, __nv_bfloat16* __restrict__ out,
                          float* __restrict__ den, int* status)
 {
@@ -156,16 +128,18 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const uint32_t sb = smem_u32(sm);
+    __shared__ Bars bars;
     __shared__ uint32_t tmem_base_sh;
-    __shared__ __align__(8) uint64_t mbar;
-    float* rs = reinterpret_cast<float*>(sm + L::RS);  // [2][128] row sums of bf16(A)
+    __shared__ volatile int abort_flag;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int wg = warp >> 2, quad = warp & 3, t = 32 * quad + lane;
-    const int bh = blockIdx.x, h = bh % H;
+    const int bh = blockIdx.x / splits, seg = blockIdx.x % splits, h = bh % H;
+    const int nch = (N + kC - 1) / kC;
+    const int cb = segment_bound(nch, splits, seg), ce = segment_bound(nch, splits, seg + 1);
+    if (cb >= ce) return;  // uniform over the CTA
     const size_t base = (size_t)bh * N * 64;
 
-    // ---- set-up: frequencies (bf16, K-major rows), zero state snapshots, ones ----
+    // ---- set-up: frequencies (bf16, K-major rows), ones, zero state snapshots ----
     for (int idx = tid; idx < G * L::P * 8; idx += kThreadsTC) {
         const int row = idx >> 3, c = idx & 7;
         const int g = row / L::P, r = row % L::P;
@@ -184,137 +158,320 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         st_shared_v4(sb + L::W + g * L::P * 128 + swz128(r, c * 8), pack_bf16(x[0], x[1]),
                      pack_bf16(x[2], x[3]), pack_bf16(x[4], x[5]), pack_bf16(x[6], x[7]));
     }
-    for (int idx = tid; idx < (G * (16384 + 4096)) / 16; idx += kThreadsTC)
-        st_shared_v4(sb + L::S + idx * 16, 0, 0, 0, 0);
     for (int idx = tid; idx < 4096 / 16; idx += kThreadsTC) {
         const uint32_t one2 = 0x3F803F80u;  // two bf16 ones
         st_shared_v4(sb + L::ONES + idx * 16, one2, one2, one2, one2);
     }
+    for (int idx = tid; idx < (G * (16384 + 4096)) / 16; idx += kThreadsTC)
+        st_shared_v4(sb + L::S + idx * 16, 0, 0, 0, 0);
     if (tid == 0) {
-        mbar_init(&mbar, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&bars.x_full[i], 1);
+            mbar_init(&bars.x_free[i], 1);
+            mbar_init(&bars.v_full[i], 1);
+            mbar_init(&bars.v_free[i], 1);
+        }
+        mbar_init(&bars.p_full, 1);
+        mbar_init(&bars.p_free, 8);
+        mbar_init(&bars.phiq_full, 8);
+        mbar_init(&bars.phik_full, 8);
+        mbar_init(&bars.phi_free, 1);
+        mbar_init(&bars.attn_done, 1);
+        mbar_init(&bars.a_ready, 4);
+        mbar_init(&bars.o_ready, 1);
+        mbar_init(&bars.epi_done, 4);
+        abort_flag = 0;
         fence_mbar_init();
     }
-    if (warp == 0) {
+    if (warp == kWarpMMA) {
         tmem_alloc(&tmem_base_sh, 512);
         tmem_relinquish();
     }
+    fence_proxy_async();
     fence_before_sync();
     __syncthreads();
     fence_after_sync();
     const uint32_t tm = tmem_base_sh;
-    const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);  // this warp's lane quadrant
-    uint32_t phase = 0;
 
-    constexpr uint32_t I_PROJ = idesc_bf16(128, L::P, 0, 0);
-    constexpr uint32_t I_QK = idesc_bf16(128, 128, 0, 0);
-    constexpr uint32_t I_QS = idesc_bf16(128, 64, 0, 1);
-    constexpr uint32_t I_QZ = idesc_bf16(128, 16, 0, 0);
-    constexpr uint32_t I_KV = idesc_bf16(128, 64, 1, 1);
-    constexpr uint32_t I_K1 = idesc_bf16(128, 16, 1, 0);
-    constexpr uint32_t I_AV = idesc_bf16(128, 64, 0, 1);
-
-    const int nchunks = (N + kC - 1) / kC;
-    for (int c = 0; c < nchunks; ++c) {
-        const int t0 = c * kC, CL = min(kC, N - t0);
-        const bool valid = t < CL;
-        load_tile(q + base + (size_t)t0 * 64, CL, sb + L::Q);
-        load_tile(k + base + (size_t)t0 * 64, CL, sb + L::K);
-        load_tile(v + base + (size_t)t0 * 64, CL, sb + L::V);
-        handoff_to_mma();
-
-        for (int g = 0; g < G; ++g) {
-            for (int which = 0; which < 2; ++which) {  // 0: q, 1: k
-                if (tid == 0) {
-                    fence_after_sync();
-                    const uint32_t x0 = sb + (which ? L::K : L::Q);
-                    const uint32_t w0 = sb + L::W + g * L::P * 128;
-#pragma unroll
-                    for (int ks = 0; ks < 4; ++ks)
-                        mma_bf16(tm + L::T_P, sdesc(x0 + ks * 32, 16, 1024),
-                                 sdesc(w0 + ks * 32, 16, 1024), I_PROJ, ks > 0);
-                    mma_commit(&mbar);
+    if (warp == kWarpTMA) {
+        // ================= TMA producer =================
+        // Main chunks: q -> X0, k -> X1.  k-only prefix chunks alternate k between X1 and
+        // X0, so the next tile loads while the current one is projected.
+        if (lane == 0) {
+            uint32_t ph_xfree[2] = {0, 0}, ph_vfree[2] = {0, 0};
+            bool used_x[2] = {false, false}, used_v[2] = {false, false};
+            auto load = [&](int b, const CUtensorMap* map, int t0) -> bool {
+                if (used_x[b]) {
+                    if (!bar_wait(&bars.x_free[b], ph_xfree[b], &abort_flag, status)) return false;
+                    ph_xfree[b] ^= 1;
                 }
-                if (!wait_mma(&mbar, phase, status)) goto done;
-                features_to_smem<NS>(tm_row + L::T_P, wg, t, valid,
-                                     sb + (which ? L::PK : L::PQ));
-                handoff_to_mma();
+                used_x[b] = true;
+                mbar_arrive_expect_tx(&bars.x_full[b], kTileBytes);
+                tma_load_3d(sb + (b ? L::X1 : L::X0), map, 0, t0, bh, &bars.x_full[b]);
+                return true;
+            };
+            for (int c = 0; c < ce; ++c) {
+                const int t0 = c * kC;
+                if (c >= cb) {
+                    if (!load(0, &tmap_q, t0) || !load(1, &tmap_k, t0)) break;
+                } else {
+                    if (!load((c & 1) ? 0 : 1, &tmap_k, t0)) break;
+                }
+                const int vb = c & 1;
+                if (used_v[vb]) {
+                    if (!bar_wait(&bars.v_free[vb], ph_vfree[vb], &abort_flag, status)) break;
+                    ph_vfree[vb] ^= 1;
+                }
+                used_v[vb] = true;
+                mbar_arrive_expect_tx(&bars.v_full[vb], kTileBytes);
+                tma_load_3d(sb + (vb ? L::V1 : L::V0), &tmap_v, 0, t0, bh, &bars.v_full[vb]);
             }
-            if (tid == 0) {
+        }
+    } else if (warp == kWarpMMA) {
+        // ================= MMA issue (one thread) =================
+        if (lane == 0) {
+            constexpr uint32_t I_PROJ = idesc_bf16(128, L::P, 0, 0);
+            constexpr uint32_t I_QK = idesc_bf16(128, 128, 0, 0);
+            constexpr uint32_t I_QS = idesc_bf16(128, 64, 0, 1);
+            constexpr uint32_t I_QZ = idesc_bf16(128, 16, 0, 0);
+            constexpr uint32_t I_KV = idesc_bf16(128, 64, 1, 1);
+            constexpr uint32_t I_K1 = idesc_bf16(128, 16, 1, 0);
+            constexpr uint32_t I_AV = idesc_bf16(128, 64, 0, 1);
+            uint32_t ph_xfull[2] = {0, 0}, ph_vfull[2] = {0, 0};
+            uint32_t ph_pfree = 0, ph_phiq = 0, ph_phik = 0, ph_aready = 0, ph_epi = 0;
+            int nproj = 0, pending_av = -1;
+            bool ok = true;
+
+            auto wait = [&](uint64_t* bar, uint32_t& ph) {
+                if (!ok) return;
+                ok = bar_wait(bar, ph, &abort_flag, status);
+                ph ^= 1;
+            };
+            auto proj = [&](int xb, int g) {
+                if (nproj > 0) wait(&bars.p_free, ph_pfree);
+                if (!ok) return;
+                fence_after_sync();
+                const uint32_t x0 = sb + (xb ? L::X1 : L::X0);
+                const uint32_t w0 = sb + L::W + g * L::P * 128;
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_bf16(tm + L::T_P, sdesc(x0 + ks * 32, 16, 1024),
+                             sdesc(w0 + ks * 32, 16, 1024), I_PROJ, ks > 0);
+                mma_commit(&bars.p_full);
+                ++nproj;
+            };
+            auto av = [&](int cc) {
+                wait(&bars.a_ready, ph_aready);
+                if (!ok) return;
+                fence_after_sync();
+                const uint32_t vb = sb + ((cc & 1) ? L::V1 : L::V0);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_bf16_tmem_a(tm + L::T_O, tm + L::T_A + 8 * ks,
+                                    sdesc(vb + ks * 2048, 16384, 1024), I_AV, 1u);
+                mma_commit(&bars.o_ready);
+                mma_commit(&bars.v_free[cc & 1]);
+            };
+            auto attn = [&](int c, int g, bool main) {
+                if (main) wait(&bars.phiq_full, ph_phiq);
+                wait(&bars.phik_full, ph_phik);
+                if (g == 0) {
+                    wait(&bars.v_full[c & 1], ph_vfull[c & 1]);
+                    if (main) wait(&bars.epi_done, ph_epi);
+                }
+                if (!ok) return;
                 fence_after_sync();
                 const uint32_t pq = sb + L::PQ, pk = sb + L::PK;
+                if (main) {
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) {  // K = 128 features of group g
-                    const uint32_t kofs = (ks >> 2) * 16384 + (ks & 3) * 32;
-                    const uint64_t aq = sdesc(pq + kofs, 16, 1024);
-                    const uint32_t acc = (g > 0 || ks > 0) ? 1u : 0u;
-                    mma_bf16(tm + L::T_A, aq, sdesc(pk + kofs, 16, 1024), I_QK, acc);
-                    mma_bf16(tm + L::T_O, aq, sdesc(sb + L::S + g * 16384 + ks * 2048, 16384, 1024),
-                             I_QS, acc);
-                    mma_bf16(tm + L::T_DN, aq,
-                             sdesc(sb + L::Z + g * 4096 + (ks >> 2) * 2048 + (ks & 3) * 32, 16,
-                                   1024),
-                             I_QZ, acc);
+                    for (int ks = 0; ks < 8; ++ks) {  // K = 128 features of group g
+                        const uint32_t kofs = (ks >> 2) * 16384 + (ks & 3) * 32;
+                        const uint64_t aq = sdesc(pq + kofs, 16, 1024);
+                        const uint32_t acc = (g > 0 || ks > 0) ? 1u : 0u;
+                        mma_bf16(tm + L::T_A, aq, sdesc(pk + kofs, 16, 1024), I_QK, acc);
+                        mma_bf16(tm + L::T_O, aq,
+                                 sdesc(sb + L::S + g * 16384 + ks * 2048, 16384, 1024), I_QS, acc);
+                        mma_bf16(tm + L::T_DN, aq,
+                                 sdesc(sb + L::Z + g * 4096 + (ks >> 2) * 2048 + (ks & 3) * 32,
+                                       16, 1024),
+                                 I_QZ, acc);
+                    }
                 }
+                const uint32_t vb = sb + ((c & 1) ? L::V1 : L::V0);
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) {  // K = 128 tokens of the chunk
                     const uint64_t ak = sdesc(pk + ks * 2048, 16384, 1024);
                     const uint32_t acc = (c > 0 || ks > 0) ? 1u : 0u;
-                    mma_bf16(tm + L::T_S + 64 * g, ak, sdesc(sb + L::V + ks * 2048, 16384, 1024),
-                             I_KV, acc);
+                    mma_bf16(tm + L::T_S + 64 * g, ak, sdesc(vb + ks * 2048, 16384, 1024), I_KV,
+                             acc);
                     mma_bf16(tm + L::T_Z + 16 * g, ak,
                              sdesc(sb + L::ONES + (ks >> 2) * 2048 + (ks & 3) * 32, 16, 1024),
                              I_K1, acc);
                 }
-                mma_commit(&mbar);
-            }
-            if (!wait_mma(&mbar, phase, status)) goto done;
-        }
+                mma_commit(&bars.phi_free);
+                if (g == G - 1) {
+                    if (main || c == cb - 1) mma_commit(&bars.attn_done);
+                    if (!main) mma_commit(&bars.v_free[c & 1]);
+                }
+            };
 
-        // ---- A: causal mask, bf16, row sums; written as the K-major A operand of A V ----
-        {
-            float a[64];
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-                tmem_ld16(tm_row + L::T_A + 64 * wg + 16 * j,
-                          *reinterpret_cast<float(*)[16]>(&a[16 * j]));
-            tmem_wait_ld();
-            float sum = 0.f;
-            uint32_t pk2[32];
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                const int j0 = 64 * wg + 2 * i;
-                const float x0 = (j0 <= t) ? a[2 * i] : 0.f;
-                const float x1 = (j0 + 1 <= t) ? a[2 * i + 1] : 0.f;
-                pk2[i] = pack_bf16(x0, x1);
-                const __nv_bfloat162 b2 = *reinterpret_cast<__nv_bfloat162*>(&pk2[i]);
-                sum += __bfloat162float(b2.x) + __bfloat162float(b2.y);
+            for (int c = 0; c < ce && ok; ++c) {
+                const bool main = c >= cb;
+                const int kb = main ? 1 : ((c & 1) ? 0 : 1);  // buffer holding k_c
+                if (main) wait(&bars.x_full[0], ph_xfull[0]);
+                wait(&bars.x_full[kb], ph_xfull[kb]);
+                for (int g = 0; g < G && ok; ++g) {
+                    if (main) {
+                        proj(0, g);
+                        if (g == G - 1) mma_commit(&bars.x_free[0]);
+                    }
+                    if (g == 0 && pending_av >= 0) {
+                        av(pending_av);
+                        pending_av = -1;
+                    }
+                    if (g >= 1) attn(c, g - 1, main);
+                    proj(kb, g);
+                    if (g == G - 1) mma_commit(&bars.x_free[kb]);
+                }
+                attn(c, G - 1, main);
+                if (main) pending_av = c;
             }
-#pragma unroll
-            for (int cc = 0; cc < 8; ++cc)
-                st_shared_v4(sb + L::A + wg * 16384 + swz128(t, cc * 8), pk2[4 * cc],
-                             pk2[4 * cc + 1], pk2[4 * cc + 2], pk2[4 * cc + 3]);
-            rs[wg * 128 + t] = sum;
+            if (ok && pending_av >= 0) av(pending_av);
         }
-        handoff_to_mma();
-        if (tid == 0) {
+    } else if (warp < kWarpEW) {
+        // ================= features =================
+        const int half = (warp - kWarpFW) >> 2, quad = warp & 3, t = 32 * quad + lane;
+        const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16) + L::T_P;
+        uint32_t ph_pfull = 0;
+        int n = 0;  // groups processed so far
+        for (int c = 0; c < ce; ++c) {
+            const bool main = c >= cb;
+            const bool valid = t < min(kC, N - c * kC);
+            for (int g = 0; g < G; ++g, ++n) {
+                for (int which = main ? 0 : 1; which < 2; ++which) {  // 0: q, 1: k
+                    if (!bar_wait(&bars.p_full, ph_pfull, &abort_flag, status)) goto fw_out;
+                    ph_pfull ^= 1;
+                    fence_after_sync();
+                    float a[32], w[32];
+                    tmem_ld16(tm_row + 32 * half, *reinterpret_cast<float(*)[16]>(&a[0]));
+                    tmem_ld16(tm_row + 32 * half + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+                    if (NS) {
+                        tmem_ld16(tm_row + 64 + 32 * half, *reinterpret_cast<float(*)[16]>(&w[0]));
+                        tmem_ld16(tm_row + 64 + 32 * half + 16,
+                                  *reinterpret_cast<float(*)[16]>(&w[16]));
+                    }
+                    tmem_wait_ld();
+                    fence_before_sync();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&bars.p_free);
+                    uint32_t pc[16], ps[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        float s0, c0, s1, c1;
+                        __sincosf(a[2 * i], &s0, &c0);
+                        __sincosf(a[2 * i + 1], &s1, &c1);
+                        if (NS) {
+                            const float cw0 = __cosf(w[2 * i]), cw1 = __cosf(w[2 * i + 1]);
+                            c0 *= cw0; s0 *= cw0; c1 *= cw1; s1 *= cw1;
+                        }
+                        if (!valid) { c0 = s0 = c1 = s1 = 0.f; }
+                        pc[i] = pack_bf16(c0, c1);
+                        ps[i] = pack_bf16(s0, s1);
+                    }
+                    if (n > 0 && !bar_wait(&bars.phi_free, (n - 1) & 1, &abort_flag, status))
+                        goto fw_out;
+                    const uint32_t dst = sb + (which ? L::PK : L::PQ);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const uint32_t off = swz128(t, (4 * half + j) * 8);
+                        st_shared_v4(dst + off, pc[4 * j], pc[4 * j + 1], pc[4 * j + 2],
+                                     pc[4 * j + 3]);
+                        st_shared_v4(dst + 16384 + off, ps[4 * j], ps[4 * j + 1], ps[4 * j + 2],
+                                     ps[4 * j + 3]);
+                    }
+                    fence_proxy_async();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(which ? &bars.phik_full : &bars.phiq_full);
+                }
+            }
+        }
+    fw_out:;
+    } else {
+        // ================= epilogue =================
+        const int quad = warp & 3, t = 32 * quad + lane;
+        const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
+        uint32_t ph_attn = 0, ph_o = 0;
+        auto snapshot = [&]() {
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
+                float s[64], zz[16];
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    tmem_ld16(tm_row + L::T_S + 64 * g + 16 * j,
+                              *reinterpret_cast<float(*)[16]>(&s[16 * j]));
+                tmem_ld16(tm_row + L::T_Z + 16 * g, zz);
+                tmem_wait_ld();
+#pragma unroll
+                for (int cc = 0; cc < 8; ++cc)
+                    st_shared_v4(sb + L::S + g * 16384 + swz128(t, cc * 8),
+                                 pack_bf16(s[8 * cc], s[8 * cc + 1]),
+                                 pack_bf16(s[8 * cc + 2], s[8 * cc + 3]),
+                                 pack_bf16(s[8 * cc + 4], s[8 * cc + 5]),
+                                 pack_bf16(s[8 * cc + 6], s[8 * cc + 7]));
+                *reinterpret_cast<__nv_bfloat16*>(sm + L::Z + g * 4096 + (t >> 6) * 2048 +
+                                                  swz128(0, t & 63)) = __float2bfloat16_rn(zz[0]);
+            }
+        };
+        auto signal = [&](uint64_t* bar) {
+            fence_proxy_async();
+            fence_before_sync();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar);
+        };
+        if (cb > 0) {  // the k-only prefix ends here: snapshot its state
+            if (!bar_wait(&bars.attn_done, ph_attn, &abort_flag, status)) goto ew_out;
+            ph_attn ^= 1;
             fence_after_sync();
-#pragma unroll
-            for (int ks = 0; ks < 8; ++ks)
-                mma_bf16(tm + L::T_O, sdesc(sb + L::A + (ks >> 2) * 16384 + (ks & 3) * 32, 16, 1024),
-                         sdesc(sb + L::V + ks * 2048, 16384, 1024), I_AV, 1u);
-            mma_commit(&mbar);
+            snapshot();
         }
-        if (!wait_mma(&mbar, phase, status)) goto done;
+        signal(&bars.epi_done);
+        for (int c = cb; c < ce; ++c) {
+            const int t0 = c * kC;
+            const bool valid = t < min(kC, N - t0);
+            if (!bar_wait(&bars.attn_done, ph_attn, &abort_flag, status)) goto ew_out;
+            ph_attn ^= 1;
+            fence_after_sync();
+            // causal mask, bf16, row sum; bf16 A written in place (keys 32b..32b+31 of
+            // block b go to columns 16b..16b+15, which block b has already read)
+            float rowsum = 0.f;
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                float a[32];
+                tmem_ld16(tm_row + L::T_A + 32 * b, *reinterpret_cast<float(*)[16]>(&a[0]));
+                tmem_ld16(tm_row + L::T_A + 32 * b + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+                tmem_wait_ld();
+                uint32_t pk2[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int j0 = 32 * b + 2 * i;
+                    pk2[i] = pack_bf16(j0 <= t ? a[2 * i] : 0.f, j0 + 1 <= t ? a[2 * i + 1] : 0.f);
+                    rowsum += bf16_lo(pk2[i]) + bf16_hi(pk2[i]);
+                }
+                tmem_st16(tm_row + L::T_A + 16 * b, pk2);
+            }
+            tmem_wait_st();
+            signal(&bars.a_ready);
 
-        if (wg == 0) {
-            // ---- output rows: out = num / den ----
+            if (!bar_wait(&bars.o_ready, ph_o, &abort_flag, status)) goto ew_out;
+            ph_o ^= 1;
+            fence_after_sync();
             float o[64], dn[16];
 #pragma unroll
             for (int j = 0; j < 4; ++j)
                 tmem_ld16(tm_row + L::T_O + 16 * j, *reinterpret_cast<float(*)[16]>(&o[16 * j]));
             tmem_ld16(tm_row + L::T_DN, dn);
             tmem_wait_ld();
-            const float dd = dn[0] + rs[t] + rs[128 + t];
+            const float dd = dn[0] + rowsum;
             if (valid) {
                 const float inv = 1.f / dd;
                 uint4* dst = reinterpret_cast<uint4*>(out + base + (size_t)(t0 + t) * 64);
@@ -326,36 +483,60 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                                          pack_bf16(o[8 * cc + 6] * inv, o[8 * cc + 7] * inv));
                 if (den) den[(size_t)bh * N + t0 + t] = dd / (float)M;
             }
-        } else {
-            // ---- state snapshot for the next chunk: S (MN-major rows) and z (K-major row 0) ----
-#pragma unroll
-            for (int g = 0; g < G; ++g) {
-                float s[64], zz[16];
-#pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    tmem_ld16(tm_row + L::T_S + 64 * g + 16 * j,
-                              *reinterpret_cast<float(*)[16]>(&s[16 * j]));
-                tmem_ld16(tm_row + L::T_Z + 16 * g, zz);
-                tmem_wait_ld();
-                const int f = t;  // feature within the group
-#pragma unroll
-                for (int cc = 0; cc < 8; ++cc)
-                    st_shared_v4(sb + L::S + g * 16384 + swz128(f, cc * 8),
-                                 pack_bf16(s[8 * cc], s[8 * cc + 1]),
-                                 pack_bf16(s[8 * cc + 2], s[8 * cc + 3]),
-                                 pack_bf16(s[8 * cc + 4], s[8 * cc + 5]),
-                                 pack_bf16(s[8 * cc + 6], s[8 * cc + 7]));
-                *reinterpret_cast<__nv_bfloat16*>(sm + L::Z + g * 4096 + (f >> 6) * 2048 +
-                                                  swz128(0, f & 63)) = __float2bfloat16_rn(zz[0]);
-            }
+            if (c + 1 < ce) snapshot();
+            signal(&bars.epi_done);
         }
-        handoff_to_mma();
+    ew_out:;
     }
-done:
+
     fence_before_sync();
     __syncthreads();
     fence_after_sync();
-    if (warp == 0) tmem_dealloc(tm, 512);
+    if (warp == kWarpMMA) tmem_dealloc(tm, 512);
+}
+
+// ---- host side ---------------------------------------------------------------------------
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return (EncodeTiledFn) nullptr;
+        return (EncodeTiledFn)p;
+    }();
+    return fn;
+}
+
+// [B*H][N][64] bf16 as a 3-D tensor; 128 x 64 boxes, 128-byte swizzle; rows past N read 0.
+bool make_act_map(CUtensorMap* m, const void* base, int BH, int N)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {64, (cuuint64_t)N, (cuuint64_t)BH};
+    cuuint64_t strides[2] = {128, (cuuint64_t)N * 128};
+    cuuint32_t box[3] = {64, 128, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+               box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
+}
+
+int sm_count()
+{
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    return n;
 }
 
 template <bool NS, int G>
@@ -363,17 +544,31 @@ cudaError_t launch_one(const Problem& p, const void* q, const void* k, const voi
                        const float* W1, const float* W2, void* out, float* den, int* status,
                        cudaStream_t s)
 {
+    CUtensorMap mq, mk, mv;
+    const int BH = p.B * p.H;
+    if (!make_act_map(&mq, q, BH, p.N) || !make_act_map(&mk, k, BH, p.N) ||
+        !make_act_map(&mv, v, BH, p.N))
+        return cudaErrorInvalidValue;
+    const int splits = tc_fwd_splits(p, sm_count());
     auto kern = tc_fwd_causal_kernel<NS, G>;
     const int smem = (int)Cfg<NS, G>::BYTES + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    kern<<<p.B * p.H, kThreadsTC, smem, s>>>(p.H, p.N, p.M, (const __nv_bfloat16*)q,
-                                              (const __nv_bfloat16*)k, (const __nv_bfloat16*)v,
-                                              W1, W2, (__nv_bfloat16*)out, den, status);
+    kern<<<BH * splits, kThreadsTC, smem, s>>>(mq, mk, mv, p.H, p.N, p.M, splits, W1, W2,
+                                               (__nv_bfloat16*)out, den, status);
     return cudaGetLastError();
 }
 
 }  // namespace
+
+int tc_fwd_splits(const Problem& p, int sms)
+{
+    const long long BH = (long long)p.B * p.H;
+    const int nch = (p.N + kC - 1) / kC;
+    if (sms > 0 && 3 * BH <= sms && nch >= 14) return 3;
+    if (sms > 0 && 2 * BH <= sms && nch >= 6) return 2;
+    return 1;
+}
 
 bool tc_fwd_supported(const Problem& p)
 {

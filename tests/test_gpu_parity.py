@@ -148,3 +148,16 @@ def test_backward_full_size_head0():
     r = oracle.bwd(sub["q"], sub["k"], sub["v"], sub["W1"], sub["W2"], w.causal, sub["dO"])
     g0 = [t[:, 0:1] for t in g[:3]] + [g[3][0:1], None]
     _compare_grads(w, g0, r)
+
+
+@pytest.mark.parametrize("N", [700, 1800, 2000, 4097])
+@pytest.mark.parametrize("w", [WL[1], WL[2]], ids=["stationary", "nonstationary"])
+def test_forward_sequence_splits(w, N):
+    """Few sequences and many chunks: the causal tensor-core path splits each sequence
+    over 2 or 3 CTAs (k-only prefix pass + own segment); every position must match."""
+    ws_ = w.replace(B=1, H=2, N=N)
+    ins = workloads.make_inputs(ws_)
+    out, den = _gpu_fwd(ws_, ins, True)
+    ro, rd = _oracle_fwd(ins, True)
+    assert_close(to_host(out), ro, w.dtype, f"out N={N}")
+    assert_close(to_host(den), rd, w.dtype, "den", max_abs_scale=float(np.abs(rd).max()))
