@@ -12,13 +12,14 @@
 // are unscaled ([cos, sin] instead of M^{-1/2}[cos, sin]): the factor cancels in the
 // output, and only the stored denominator is rescaled (den = den' / M).
 //
-// Warp roles (448 threads), handshakes on mbarriers:
+// Warp roles (576 threads), handshakes on mbarriers:
 //   warp 0      TMA: q, k, v chunk tiles (128B swizzle) into shared memory
 //   warp 1      one thread issues every tcgen05.mma; owns the tensor-memory allocation
 //   warps 2-9   features: projection (TMEM) -> cos/sin -> bf16 phi tiles (shared memory);
 //               warps 2-5 take frequencies 0-31 of a group, warps 6-9 frequencies 32-63
-//   warps 10-13 epilogue: causal mask + bf16 of A (written back into TMEM as the A operand
-//               of A V), output rows, bf16 snapshot of S and z for the next chunk
+//   warps 10-17 epilogue, two halves of 4 warps: causal mask + bf16 of A (written back
+//               into TMEM as the A operand of A V), output rows, bf16 snapshot of S and z
+//               for the next chunk; each half takes half of the columns (or one group)
 //
 // Sequence split: when there are SMs to spare, a sequence is cut into `splits` segments
 // handled by different CTAs with no waiting between them: the CTA of segment j first runs
@@ -27,12 +28,16 @@
 // lengths halve from one segment to the next, which balances the work because a k-only
 // chunk costs about half a full chunk.
 //
+// z rides in S as an extra column: the state update multiplies phi(K)^T by [V | 1], and
+// the output MMAs multiply by [S | z] and [V | 1], so column 64 of the output accumulator
+// is the denominator, built from exactly the bf16 values that build the numerator.
+//
 // Tensor memory (512 columns x 128 lanes, fp32):
 //   [0,128)    projection of one group (s: 64 cols a; n: 64 cols u, 64 cols w)
-//   [128,256)  A = phi(Q) phi(K)^T (row = query, col = key); after the epilogue its first
-//              64 columns hold bf16(masked A), two keys per column
-//   [256,320)  numerator phi(Q) S + A V           [320,336) phi(Q) z (column 0)
-//   [336,336+64G)  S per group (lane = feature)   then 16 columns of z per group
+//   [128,256)  A = phi(Q) phi(K)^T (row = query, col = key); after the epilogue, columns
+//              [0,32) and [64,96) hold bf16(masked A) of keys 0-63 and 64-127, two per column
+//   [256,336)  phi(Q) [S | z] + A [V | 1]: numerator in 0-63, denominator in 64
+//   [336,336+80G)  [S | z] per group (lane = feature), z in column 64 of each
 #include <cuda.h>
 
 #include "flex_internal.h"
@@ -43,26 +48,29 @@ namespace {
 using namespace tc;
 
 constexpr int kC = 128;            // tokens per chunk = MMA M
-constexpr int kThreadsTC = 448;    // 14 warps
-constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kWarpEW = 10;
+constexpr int kThreadsTC = 576;    // 18 warps
+constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kWarpEW = 10, kEpiWarps = 8;
 constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz: every wait is bounded
 constexpr uint32_t kTileBytes = 128 * 128;       // one 128 x 64 bf16 tile
 
 template <bool NS, int G>
 struct Cfg {
     static constexpr int P = NS ? 128 : 64;  // projection columns per group
-    // shared memory offsets (bytes, 1024-aligned); X0/X1 hold q/k tiles
-    static constexpr uint32_t X0 = 0, X1 = 16384, V0 = 32768, V1 = 49152, ONES = 65536;
-    static constexpr uint32_t W = 69632;
+    // shared memory offsets (bytes, 1024-aligned); X0/X1 hold q/k tiles.  VONE is the
+    // second 64-column block of [V | 1] (column 0 = 1, the rest 0), reached from either V
+    // buffer through the descriptor's leading byte offset.
+    static constexpr uint32_t X0 = 0, X1 = 16384, V0 = 32768, V1 = 49152, VONE = 65536;
+    static constexpr uint32_t W = 81920;
     static constexpr uint32_t PQ = W + G * P * 128;
     static constexpr uint32_t PK = PQ + 32768;
-    static constexpr uint32_t S = PK + 32768;
-    static constexpr uint32_t Z = S + G * 16384;
-    static constexpr uint32_t BYTES = Z + G * 4096;
+    // [S | z] snapshot per group, K-major: 80 rows (64 dcols, z, 15 zero rows) x 128
+    // features = two 64-feature blocks of 80 x 128 bytes
+    static constexpr uint32_t SX = PK + 32768;
+    static constexpr uint32_t SX_BLOCK = 80 * 128, SX_GROUP = 2 * SX_BLOCK;
+    static constexpr uint32_t BYTES = SX + G * SX_GROUP;
     // tensor memory columns
-    static constexpr uint32_t T_P = 0, T_A = 128, T_O = 256, T_DN = 320, T_S = 336;
-    static constexpr uint32_t T_Z = T_S + 64 * G;
-    static_assert(T_Z + 16 * G <= 512, "tensor memory budget");
+    static constexpr uint32_t T_P = 0, T_A = 128, T_O = 256, T_S = 336;
+    static_assert(T_S + 80 * G <= 512, "tensor memory budget");
     static_assert(BYTES + 1024 <= 232448, "shared memory budget");
 };
 
@@ -77,9 +85,6 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&v);
 }
-
-__device__ __forceinline__ float bf16_lo(uint32_t x) { return __uint_as_float(x << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t x) { return __uint_as_float(x & 0xFFFF0000u); }
 
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
                                              uint32_t d)
@@ -116,7 +121,7 @@ __device__ __forceinline__ int segment_bound(int nch, int splits, int j)
 }
 
 template <bool NS, int G>
-__global__ void __launch_bounds__(kThreadsTC, 1)
+__global__ void __maxnreg__(96)
     tc_fwd_causal_kernel(const __grid_constant__ CUtensorMap tmap_q,
                          const __grid_constant__ CUtensorMap tmap_k,
                          const __grid_constant__ CUtensorMap tmap_v, int H, int N, int M,
@@ -158,12 +163,13 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         st_shared_v4(sb + L::W + g * L::P * 128 + swz128(r, c * 8), pack_bf16(x[0], x[1]),
                      pack_bf16(x[2], x[3]), pack_bf16(x[4], x[5]), pack_bf16(x[6], x[7]));
     }
-    for (int idx = tid; idx < 4096 / 16; idx += kThreadsTC) {
-        const uint32_t one2 = 0x3F803F80u;  // two bf16 ones
-        st_shared_v4(sb + L::ONES + idx * 16, one2, one2, one2, one2);
-    }
-    for (int idx = tid; idx < (G * (16384 + 4096)) / 16; idx += kThreadsTC)
-        st_shared_v4(sb + L::S + idx * 16, 0, 0, 0, 0);
+    for (int idx = tid; idx < 16384 / 16; idx += kThreadsTC)  // [1, 0, ..., 0] rows
+        st_shared_v4(sb + L::VONE + idx * 16, 0, 0, 0, 0);
+    for (int idx = tid; idx < G * L::SX_GROUP / 16; idx += kThreadsTC)
+        st_shared_v4(sb + L::SX + idx * 16, 0, 0, 0, 0);
+    __syncthreads();
+    for (int r = tid; r < kC; r += kThreadsTC)
+        *reinterpret_cast<uint16_t*>(sm + L::VONE + swz128(r, 0)) = 0x3F80u;  // bf16 1.0
     if (tid == 0) {
         for (int i = 0; i < 2; ++i) {
             mbar_init(&bars.x_full[i], 1);
@@ -177,9 +183,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         mbar_init(&bars.phik_full, 8);
         mbar_init(&bars.phi_free, 1);
         mbar_init(&bars.attn_done, 1);
-        mbar_init(&bars.a_ready, 4);
+        mbar_init(&bars.a_ready, kEpiWarps);
         mbar_init(&bars.o_ready, 1);
-        mbar_init(&bars.epi_done, 4);
+        mbar_init(&bars.epi_done, kEpiWarps);
         abort_flag = 0;
         fence_mbar_init();
     }
@@ -232,11 +238,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         if (lane == 0) {
             constexpr uint32_t I_PROJ = idesc_bf16(128, L::P, 0, 0);
             constexpr uint32_t I_QK = idesc_bf16(128, 128, 0, 0);
-            constexpr uint32_t I_QS = idesc_bf16(128, 64, 0, 1);
-            constexpr uint32_t I_QZ = idesc_bf16(128, 16, 0, 0);
-            constexpr uint32_t I_KV = idesc_bf16(128, 64, 1, 1);
-            constexpr uint32_t I_K1 = idesc_bf16(128, 16, 1, 0);
-            constexpr uint32_t I_AV = idesc_bf16(128, 64, 0, 1);
+            constexpr uint32_t I_QS = idesc_bf16(128, 80, 0, 0);
+            constexpr uint32_t I_KV = idesc_bf16(128, 80, 1, 1);
+            constexpr uint32_t I_AV = idesc_bf16(128, 80, 0, 1);
             uint32_t ph_xfull[2] = {0, 0}, ph_vfull[2] = {0, 0};
             uint32_t ph_pfree = 0, ph_phiq = 0, ph_phik = 0, ph_aready = 0, ph_epi = 0;
             int nproj = 0, pending_av = -1;
@@ -247,16 +251,25 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 ok = bar_wait(bar, ph, &abort_flag, status);
                 ph ^= 1;
             };
+            // Descriptors are built once; an operand K step adds its byte offset / 16 to
+            // the start-address field (addresses stay below 256 KB: no carry out).
+            const uint64_t d_x[2] = {sdesc(sb + L::X0, 16, 1024), sdesc(sb + L::X1, 16, 1024)};
+            const uint64_t d_w = sdesc(sb + L::W, 16, 1024);
+            const uint64_t d_pq = sdesc(sb + L::PQ, 16, 1024);
+            const uint64_t d_pk = sdesc(sb + L::PK, 16, 1024);
+            const uint64_t d_pk_mn = sdesc(sb + L::PK, 16384, 1024);
+            const uint64_t d_sx = sdesc(sb + L::SX, 16, 1024);
+            const uint64_t d_v[2] = {sdesc(sb + L::V0, L::VONE - L::V0, 1024),
+                                     sdesc(sb + L::V1, L::VONE - L::V1, 1024)};
+            auto adv = [](uint64_t d, uint32_t bytes) { return d + (bytes >> 4); };
             auto proj = [&](int xb, int g) {
                 if (nproj > 0) wait(&bars.p_free, ph_pfree);
                 if (!ok) return;
                 fence_after_sync();
-                const uint32_t x0 = sb + (xb ? L::X1 : L::X0);
-                const uint32_t w0 = sb + L::W + g * L::P * 128;
+                const uint64_t wd = adv(d_w, g * L::P * 128);
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
-                    mma_bf16(tm + L::T_P, sdesc(x0 + ks * 32, 16, 1024),
-                             sdesc(w0 + ks * 32, 16, 1024), I_PROJ, ks > 0);
+                    mma_bf16(tm + L::T_P, adv(d_x[xb], ks * 32), adv(wd, ks * 32), I_PROJ, ks > 0);
                 mma_commit(&bars.p_full);
                 ++nproj;
             };
@@ -264,11 +277,11 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 wait(&bars.a_ready, ph_aready);
                 if (!ok) return;
                 fence_after_sync();
-                const uint32_t vb = sb + ((cc & 1) ? L::V1 : L::V0);
+                const uint64_t vd = d_v[cc & 1];
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks)
-                    mma_bf16_tmem_a(tm + L::T_O, tm + L::T_A + 8 * ks,
-                                    sdesc(vb + ks * 2048, 16384, 1024), I_AV, 1u);
+                for (int ks = 0; ks < 8; ++ks)  // keys 16ks..16ks+15: bf16 A columns
+                    mma_bf16_tmem_a(tm + L::T_O, tm + L::T_A + 64 * (ks >> 2) + 8 * (ks & 3),
+                                    adv(vd, ks * 2048), I_AV, 1u);
                 mma_commit(&bars.o_ready);
                 mma_commit(&bars.v_free[cc & 1]);
             };
@@ -281,33 +294,24 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 }
                 if (!ok) return;
                 fence_after_sync();
-                const uint32_t pq = sb + L::PQ, pk = sb + L::PK;
+                const uint64_t vd = d_v[c & 1];
+                const uint64_t sxd = adv(d_sx, g * L::SX_GROUP);
+                const uint32_t acc_s = c > 0 ? 1u : 0u;
                 if (main) {
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks) {  // K = 128 features of group g
                         const uint32_t kofs = (ks >> 2) * 16384 + (ks & 3) * 32;
-                        const uint64_t aq = sdesc(pq + kofs, 16, 1024);
+                        const uint64_t aq = adv(d_pq, kofs);
                         const uint32_t acc = (g > 0 || ks > 0) ? 1u : 0u;
-                        mma_bf16(tm + L::T_A, aq, sdesc(pk + kofs, 16, 1024), I_QK, acc);
+                        mma_bf16(tm + L::T_A, aq, adv(d_pk, kofs), I_QK, acc);
                         mma_bf16(tm + L::T_O, aq,
-                                 sdesc(sb + L::S + g * 16384 + ks * 2048, 16384, 1024), I_QS, acc);
-                        mma_bf16(tm + L::T_DN, aq,
-                                 sdesc(sb + L::Z + g * 4096 + (ks >> 2) * 2048 + (ks & 3) * 32,
-                                       16, 1024),
-                                 I_QZ, acc);
+                                 adv(sxd, (ks >> 2) * L::SX_BLOCK + (ks & 3) * 32), I_QS, acc);
                     }
                 }
-                const uint32_t vb = sb + ((c & 1) ? L::V1 : L::V0);
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) {  // K = 128 tokens of the chunk
-                    const uint64_t ak = sdesc(pk + ks * 2048, 16384, 1024);
-                    const uint32_t acc = (c > 0 || ks > 0) ? 1u : 0u;
-                    mma_bf16(tm + L::T_S + 64 * g, ak, sdesc(vb + ks * 2048, 16384, 1024), I_KV,
-                             acc);
-                    mma_bf16(tm + L::T_Z + 16 * g, ak,
-                             sdesc(sb + L::ONES + (ks >> 2) * 2048 + (ks & 3) * 32, 16, 1024),
-                             I_K1, acc);
-                }
+                for (int ks = 0; ks < 8; ++ks)  // K = 128 tokens of the chunk
+                    mma_bf16(tm + L::T_S + 80 * g, adv(d_pk_mn, ks * 2048), adv(vd, ks * 2048),
+                             I_KV, (acc_s | (ks > 0)) ? 1u : 0u);
                 mma_commit(&bars.phi_free);
                 if (g == G - 1) {
                     if (main || c == cb - 1) mma_commit(&bars.attn_done);
@@ -315,27 +319,38 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 }
             };
 
+            // Job stream: per chunk, for each group, a q job (main chunks) and a k job.  The
+            // projection of a job is issued before the attention MMAs of the group the
+            // previous job completed, so the tensor pipe (in order) never makes the feature
+            // warps wait for a projection stuck behind a long attention step.
+            int pa_c = -1, pa_g = 0;
+            bool pa_main = false;
             for (int c = 0; c < ce && ok; ++c) {
                 const bool main = c >= cb;
-                const int kb = main ? 1 : ((c & 1) ? 0 : 1);  // buffer holding k_c
-                if (main) wait(&bars.x_full[0], ph_xfull[0]);
-                wait(&bars.x_full[kb], ph_xfull[kb]);
                 for (int g = 0; g < G && ok; ++g) {
-                    if (main) {
-                        proj(0, g);
-                        if (g == G - 1) mma_commit(&bars.x_free[0]);
+                    for (int which = main ? 0 : 1; which < 2 && ok; ++which) {
+                        const int buf = which == 0 ? 0 : (main ? 1 : ((c & 1) ? 0 : 1));
+                        if (g == 0) wait(&bars.x_full[buf], ph_xfull[buf]);
+                        proj(buf, g);
+                        if (g == G - 1) mma_commit(&bars.x_free[buf]);
+                        if (pa_c >= 0) {
+                            attn(pa_c, pa_g, pa_main);
+                            pa_c = -1;
+                        }
+                        if (which == 1) {
+                            if (g == 0 && main && pending_av >= 0) {
+                                av(pending_av);
+                                pending_av = -1;
+                            }
+                            pa_c = c;  // this k job completes group g
+                            pa_g = g;
+                            pa_main = main;
+                            if (g == G - 1 && main) pending_av = c;
+                        }
                     }
-                    if (g == 0 && pending_av >= 0) {
-                        av(pending_av);
-                        pending_av = -1;
-                    }
-                    if (g >= 1) attn(c, g - 1, main);
-                    proj(kb, g);
-                    if (g == G - 1) mma_commit(&bars.x_free[kb]);
                 }
-                attn(c, G - 1, main);
-                if (main) pending_av = c;
             }
+            if (ok && pa_c >= 0) attn(pa_c, pa_g, pa_main);
             if (ok && pending_av >= 0) av(pending_av);
         }
     } else if (warp < kWarpEW) {
@@ -398,29 +413,34 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     fw_out:;
     } else {
         // ================= epilogue =================
-        const int quad = warp & 3, t = 32 * quad + lane;
+        // Two halves of 4 warps (one warp per lane quadrant each): half eh takes keys
+        // [64eh, 64eh+64) of A, output columns [32eh, 32eh+32), and group eh of the state
+        // (G = 2) or its state columns [32eh, 32eh+32) (G = 1).
+        const int eh = (warp - kWarpEW) >> 2, quad = warp & 3, t = 32 * quad + lane;
         const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
         uint32_t ph_attn = 0, ph_o = 0;
         auto snapshot = [&]() {
+            // K-major [S | z]: row e holds S[f][e] over the features f of one group
+            constexpr int NCOL = G == 2 ? 64 : 32;
+            const int g = G == 2 ? eh : 0, e0 = G == 2 ? 0 : 32 * eh;
+            float s_[NCOL];
 #pragma unroll
-            for (int g = 0; g < G; ++g) {
-                float s[64], zz[16];
+            for (int j = 0; j < NCOL / 16; ++j)
+                tmem_ld16(tm_row + L::T_S + 80 * g + e0 + 16 * j,
+                          *reinterpret_cast<float(*)[16]>(&s_[16 * j]));
+            float zz[16];
+            const bool with_z = G == 2 || eh == 0;
+            if (with_z) tmem_ld16(tm_row + L::T_S + 80 * g + 64, zz);
+            tmem_wait_ld();
+            uint8_t* blk = sm + L::SX + g * L::SX_GROUP + (t >> 6) * L::SX_BLOCK;
+            const uint32_t col = t & 63;
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    tmem_ld16(tm_row + L::T_S + 64 * g + 16 * j,
-                              *reinterpret_cast<float(*)[16]>(&s[16 * j]));
-                tmem_ld16(tm_row + L::T_Z + 16 * g, zz);
-                tmem_wait_ld();
-#pragma unroll
-                for (int cc = 0; cc < 8; ++cc)
-                    st_shared_v4(sb + L::S + g * 16384 + swz128(t, cc * 8),
-                                 pack_bf16(s[8 * cc], s[8 * cc + 1]),
-                                 pack_bf16(s[8 * cc + 2], s[8 * cc + 3]),
-                                 pack_bf16(s[8 * cc + 4], s[8 * cc + 5]),
-                                 pack_bf16(s[8 * cc + 6], s[8 * cc + 7]));
-                *reinterpret_cast<__nv_bfloat16*>(sm + L::Z + g * 4096 + (t >> 6) * 2048 +
-                                                  swz128(0, t & 63)) = __float2bfloat16_rn(zz[0]);
-            }
+            for (int e = 0; e < NCOL; ++e)
+                *reinterpret_cast<__nv_bfloat16*>(blk + swz128(e0 + e, col)) =
+                    __float2bfloat16_rn(s_[e]);
+            if (with_z)
+                *reinterpret_cast<__nv_bfloat16*>(blk + swz128(64, col)) =
+                    __float2bfloat16_rn(zz[0]);
         };
         auto signal = [&](uint64_t* bar) {
             fence_proxy_async();
@@ -441,23 +461,22 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             if (!bar_wait(&bars.attn_done, ph_attn, &abort_flag, status)) goto ew_out;
             ph_attn ^= 1;
             fence_after_sync();
-            // causal mask, bf16, row sum; bf16 A written in place (keys 32b..32b+31 of
-            // block b go to columns 16b..16b+15, which block b has already read)
-            float rowsum = 0.f;
+            // causal mask + bf16; keys 32b..32b+31 of this half (columns 64eh + 32b ..) go
+            // to columns 64eh + 16b .., which this thread has already read
 #pragma unroll
-            for (int b = 0; b < 4; ++b) {
+            for (int b = 0; b < 2; ++b) {
+                const uint32_t col = L::T_A + 64 * eh + 32 * b;
                 float a[32];
-                tmem_ld16(tm_row + L::T_A + 32 * b, *reinterpret_cast<float(*)[16]>(&a[0]));
-                tmem_ld16(tm_row + L::T_A + 32 * b + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+                tmem_ld16(tm_row + col, *reinterpret_cast<float(*)[16]>(&a[0]));
+                tmem_ld16(tm_row + col + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
                 tmem_wait_ld();
                 uint32_t pk2[16];
 #pragma unroll
                 for (int i = 0; i < 16; ++i) {
-                    const int j0 = 32 * b + 2 * i;
+                    const int j0 = 64 * eh + 32 * b + 2 * i;
                     pk2[i] = pack_bf16(j0 <= t ? a[2 * i] : 0.f, j0 + 1 <= t ? a[2 * i + 1] : 0.f);
-                    rowsum += bf16_lo(pk2[i]) + bf16_hi(pk2[i]);
                 }
-                tmem_st16(tm_row + L::T_A + 16 * b, pk2);
+                tmem_st16(tm_row + L::T_A + 64 * eh + 16 * b, pk2);
             }
             tmem_wait_st();
             signal(&bars.a_ready);
@@ -465,23 +484,21 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             if (!bar_wait(&bars.o_ready, ph_o, &abort_flag, status)) goto ew_out;
             ph_o ^= 1;
             fence_after_sync();
-            float o[64], dn[16];
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-                tmem_ld16(tm_row + L::T_O + 16 * j, *reinterpret_cast<float(*)[16]>(&o[16 * j]));
-            tmem_ld16(tm_row + L::T_DN, dn);
+            float o[32], dn[16];
+            tmem_ld16(tm_row + L::T_O + 32 * eh, *reinterpret_cast<float(*)[16]>(&o[0]));
+            tmem_ld16(tm_row + L::T_O + 32 * eh + 16, *reinterpret_cast<float(*)[16]>(&o[16]));
+            tmem_ld16(tm_row + L::T_O + 64, dn);
             tmem_wait_ld();
-            const float dd = dn[0] + rowsum;
             if (valid) {
-                const float inv = 1.f / dd;
-                uint4* dst = reinterpret_cast<uint4*>(out + base + (size_t)(t0 + t) * 64);
+                const float inv = 1.f / dn[0];
+                uint4* dst = reinterpret_cast<uint4*>(out + base + (size_t)(t0 + t) * 64 + 32 * eh);
 #pragma unroll
-                for (int cc = 0; cc < 8; ++cc)
+                for (int cc = 0; cc < 4; ++cc)
                     dst[cc] = make_uint4(pack_bf16(o[8 * cc] * inv, o[8 * cc + 1] * inv),
                                          pack_bf16(o[8 * cc + 2] * inv, o[8 * cc + 3] * inv),
                                          pack_bf16(o[8 * cc + 4] * inv, o[8 * cc + 5] * inv),
                                          pack_bf16(o[8 * cc + 6] * inv, o[8 * cc + 7] * inv));
-                if (den) den[(size_t)bh * N + t0 + t] = dd / (float)M;
+                if (den && eh == 0) den[(size_t)bh * N + t0 + t] = dn[0] / (float)M;
             }
             if (c + 1 < ce) snapshot();
             signal(&bars.epi_done);
