@@ -41,8 +41,9 @@ int check_ws(void* ws, size_t ws_bytes, size_t need)
 
 size_t fwd_ws_bytes(const Problem& p)
 {
-    (void)p;
-    return header_bytes();
+    size_t n = header_bytes();
+    if (flex::tc_nc_supported(p)) n += flex::align_up(flex::tc_nc_ws_bytes(p), 256);
+    return n;
 }
 
 size_t bwd_ws_bytes(const Problem& p)
@@ -81,7 +82,7 @@ size_t flex_workspace_bytes(const flex_shape* shape, int causal, int backward)
 {
     Problem p;
     if (make_problem(shape, nullptr, causal, &p) != FLEX_OK) return 0;
-    // The nonstationary variant needs the larger scratch; size for it.
+    // Size for the larger of the two variants' scratch.
     p.nonstat = 1;
     return backward ? bwd_ws_bytes(p) : fwd_ws_bytes(p);
 }
@@ -114,6 +115,9 @@ int flex_linattn_fwd(const flex_shape* shape, const void* q, const void* k, cons
     int* status = &((flex::WsHeader*)ws)->status;
     if (flex::tc_fwd_supported(p))
         return count(1, flex::launch_tc_fwd(p, q, k, v, W1, W2, out, den, status, s));
+    if (flex::tc_nc_supported(p))
+        return count(3, flex::launch_tc_nc(p, q, k, v, W1, W2, out, den,
+                                           (char*)ws + header_bytes(), status, s));
     if (flex::simt_pick_chunk_fwd(p) == 0) return FLEX_EUNSUPPORTED;
     return count(1, flex::launch_simt_fwd(p, q, k, v, W1, W2, out, den, s));
 }

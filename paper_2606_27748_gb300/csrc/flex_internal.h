@@ -53,4 +53,11 @@ cudaError_t launch_tc_fwd(const Problem& p, const void* q, const void* k, const 
                           const float* W1, const float* W2, void* out, float* den, int* status,
                           cudaStream_t s);
 
+bool tc_nc_supported(const Problem& p);
+int tc_nc_splits(const Problem& p);
+size_t tc_nc_ws_bytes(const Problem& p);
+cudaError_t launch_tc_nc(const Problem& p, const void* q, const void* k, const void* v,
+                         const float* W1, const float* W2, void* out, float* den, void* scratch,
+                         int* status, cudaStream_t s);
+
 }  // namespace flex

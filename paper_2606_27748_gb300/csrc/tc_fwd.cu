@@ -42,6 +42,7 @@
 
 #include "flex_internal.h"
 #include "tc_common.cuh"
+#include "tc_util.cuh"
 
 namespace flex {
 namespace {
@@ -50,8 +51,6 @@ using namespace tc;
 constexpr int kC = 128;            // tokens per chunk = MMA M
 constexpr int kThreadsTC = 576;    // 18 warps
 constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kWarpEW = 10, kEpiWarps = 8;
-constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz: every wait is bounded
-constexpr uint32_t kTileBytes = 128 * 128;       // one 128 x 64 bf16 tile
 
 template <bool NS, int G>
 struct Cfg {
@@ -79,38 +78,6 @@ struct Bars {
     uint64_t p_full, p_free, phiq_full, phik_full, phi_free;
     uint64_t attn_done, a_ready, o_ready, epi_done;
 };
-
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi)
-{
-    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<uint32_t*>(&v);
-}
-
-__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
-                                             uint32_t d)
-{
-    asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
-                 "r"(d)
-                 : "memory");
-}
-
-// Bounded wait on one mbarrier phase.  On a time-out the CTA is told to stop (abort flag)
-// and the status word records FLEX_ETIMEOUT; every other wait then returns at once.
-__device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                         int* status)
-{
-    if (mbar_try_wait(bar, parity)) return true;
-    const long long t0 = clock64();
-    while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if (*abort_flag) return false;
-        if (clock64() - t0 > kWaitCycles) {
-            *abort_flag = 1;
-            atomicExch(status, (int)FLEX_ETIMEOUT);
-            return false;
-        }
-    }
-}
 
 // First chunk of segment j of `splits` (lengths proportional to 2^-j), rounded.
 __device__ __forceinline__ int segment_bound(int nch, int splits, int j)
@@ -510,50 +477,6 @@ __global__ void __maxnreg__(96)
     __syncthreads();
     fence_after_sync();
     if (warp == kWarpMMA) tmem_dealloc(tm, 512);
-}
-
-// ---- host side ---------------------------------------------------------------------------
-
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn()
-{
-    static EncodeTiledFn fn = [] {
-        void* p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
-                                             cudaEnableDefault, &q) != cudaSuccess ||
-            q != cudaDriverEntryPointSuccess)
-            return (EncodeTiledFn) nullptr;
-        return (EncodeTiledFn)p;
-    }();
-    return fn;
-}
-
-// [B*H][N][64] bf16 as a 3-D tensor; 128 x 64 boxes, 128-byte swizzle; rows past N read 0.
-bool make_act_map(CUtensorMap* m, const void* base, int BH, int N)
-{
-    EncodeTiledFn enc = encode_fn();
-    if (!enc) return false;
-    cuuint64_t dims[3] = {64, (cuuint64_t)N, (cuuint64_t)BH};
-    cuuint64_t strides[2] = {128, (cuuint64_t)N * 128};
-    cuuint32_t box[3] = {64, 128, 1};
-    cuuint32_t es[3] = {1, 1, 1};
-    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
-               box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
-           CUDA_SUCCESS;
-}
-
-int sm_count()
-{
-    int dev = 0, n = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    return n;
 }
 
 template <bool NS, int G>
