@@ -32,6 +32,7 @@ sys.path.insert(0, ROOT)
 from paper_2606_27748_gb300 import workloads  # noqa: E402
 
 METRIC = "RFF linear-attn fwd tokens/s (N=16K causal) & % of bf16 tensor/HBM roofline"
+METRIC_TRAIN = "RFF linear-attn fwd+bwd training-step tokens/s & % of HBM roofline"
 L2_BYTES = 129e6
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
@@ -256,8 +257,16 @@ def run_ours(args, w):
     ws = flexattn.workspace(shape, w.causal, False, dev)
     stream = torch.cuda.current_stream()
 
+    if w.backward:  # a training step: forward, then backward of sum(dO * out)
+        dO = torch.from_numpy(workloads.draw_activation(w, workloads.DO)).to(tdt).to(dev)
+        grads = [torch.empty_like(q), torch.empty_like(k), torch.empty_like(v),
+                 torch.empty_like(W1), None if W2 is None else torch.empty_like(W2)]
+        ws_b = flexattn.workspace(shape, w.causal, True, dev)
+
     def step():
         flexattn.linattn_fwd(q, k, v, W1, W2, w.causal, out=out, den=den, ws=ws)
+        if w.backward:
+            flexattn.linattn_bwd(q, k, v, W1, W2, w.causal, out, den, dO, *grads, ws=ws_b)
 
     for _ in range(max(3, args.warmup)):
         step()
@@ -329,6 +338,8 @@ def run_ours(args, w):
 
     peaks, peaks_src = load_peaks()
     nbytes = algorithmic_bytes(w)
+    if w.backward:  # + backward: read q, k, v, out, dO; write dq, dk, dv
+        nbytes += w.token_heads * 8 * w.d * elem_bytes(w)
     achieved = nbytes / (kernel_ms * 1e-3) / 1e9
     roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
             "frac": achieved / peaks["hbm_gbs"], "traffic": recorded_traffic(w, source_digest()),
@@ -345,7 +356,8 @@ def run_ours(args, w):
 
     if rank == 0:
         line = {
-            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "metric": METRIC_TRAIN if w.backward else METRIC, "value": value,
+            "unit": "tokens/s", "n_gpus": world,
             "steps": K, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": w.dtype, "data": "synthetic",

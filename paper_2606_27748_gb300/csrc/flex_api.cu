@@ -5,6 +5,7 @@
 
 #include <stdint.h>
 
+#include <algorithm>
 #include <atomic>
 
 using flex::Problem;
@@ -48,7 +49,9 @@ size_t fwd_ws_bytes(const Problem& p)
 
 size_t bwd_ws_bytes(const Problem& p)
 {
-    return header_bytes() + flex::align_up(flex::simt_bwd_ws_bytes(p), 256);
+    size_t scratch = flex::simt_bwd_ws_bytes(p);
+    if (flex::tc_bwd_supported(p)) scratch = std::max(scratch, flex::tc_bwd_ws_bytes(p));
+    return header_bytes() + flex::align_up(scratch, 256);
 }
 
 std::atomic<unsigned long long> g_launches{0};
@@ -138,9 +141,12 @@ int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, cons
         if (!aligned(t, 16)) return FLEX_EINVAL;
     if ((W2 && !aligned(W2, 16)) || (dW2 && !aligned(dW2, 16))) return FLEX_EINVAL;
     if ((rc = check_ws(ws, ws_bytes, bwd_ws_bytes(p)))) return rc;
-    if (flex::simt_pick_chunk_bwd(p) == 0) return FLEX_EUNSUPPORTED;
     cudaStream_t s = (cudaStream_t)stream;
     void* scratch = (char*)ws + header_bytes();
+    if (flex::tc_bwd_supported(p))
+        return count(4, flex::launch_tc_bwd(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1,
+                                            dW2, scratch, &((flex::WsHeader*)ws)->status, s));
+    if (flex::simt_pick_chunk_bwd(p) == 0) return FLEX_EUNSUPPORTED;
     return count(2, flex::launch_simt_bwd(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1,
                                           dW2, scratch, s));
 }

@@ -1,0 +1,620 @@
+// Backward of RFF linear attention on the tensor cores (tcgen05).
+//
+// Gradient of L = sum(dout * out) for Eq. (linear att).  With unscaled features phi'
+// (the M^{-1/2} cancels), den' = M den, g_i = dout_i / den'_i, c_i = -(dout_i . out_i)/den'_i:
+//   dA_ij    = g_i . v_j + c_i                      (j <= i when causal)
+//   dphi(q_i) = sum_j dA_ij phi(k_j)   = [intra-chunk] + S_i g_i + c_i z_i
+//   dphi(k_j) = sum_i dA_ij phi(q_i)   = [intra-chunk] + R_j v_j + r_j
+//   dv_j      = sum_i A_ij g_i         = [intra-chunk] + R_j^T phi(k_j)
+// with S = sum phi(k) v^T, z = sum phi(k) (forward running sums) and R = sum phi(q) g^T,
+// r = sum c phi(q) (reverse running sums), then through the feature map (Eq. phi_n /
+// phi_non) by the chain rule: dx = da W, dW += da^T x.
+//
+// Every term splits over feature groups (64 frequencies = 128 features), and A enters dv
+// linearly, so one CTA handles one (sequence, group) pair and the group results are summed:
+// dq, dk, dv by fp32 adds onto zeroed accumulators (at most two groups, so the sum does not
+// depend on the order), dW through per-(sequence, group) partials reduced over the batch in
+// a fixed order.  Two launches: pass F runs the chunks forward (dq and the q part of dW,
+// state S, z), pass R runs them backward (dk, dv and the k part of dW, state R, r).
+//
+// Phases are serialised: all 256 threads load, compute features and run the CUDA-core
+// epilogues; thread 0 issues the MMAs; one mbarrier tracks their completion (bounded waits).
+//
+// Tensor memory (512 columns): [0,128) projection, [128,256) A / dA (bf16 in place) then
+// dx (0-63) and the chunk's dW (64-127), [256,384) dphi, [384,464) S|z or R|r.
+#include <algorithm>
+
+#include "flex_internal.h"
+#include "tc_common.cuh"
+#include "tc_util.cuh"
+
+namespace flex {
+namespace {
+using namespace tc;
+
+constexpr int kC = 128;
+constexpr int kThreadsB = 256;
+enum { kPassF = 0, kPassR = 1 };
+
+template <bool NS>
+struct BwCfg {
+    static constexpr int P = NS ? 128 : 64;  // projection rows (and dW rows) per group
+    // shared memory (bytes).  Pass R keeps bf16(dA) in [Q | DA2] and bf16(A) in [DO | O].
+    static constexpr uint32_t Q = 0, DA2 = 16384, K = 32768, V = 49152, DO = 65536, O = 81920;
+    static constexpr uint32_t GT = 98304;     // g tile [token][dcol], bf16
+    static constexpr uint32_t C16 = 114688;   // K-major [16][128 tokens]: ones (F) / c (R)
+    static constexpr uint32_t W = 118784;     // this group's projection rows
+    static constexpr uint32_t PQ = 135168, PK = 167936;  // features (then da in place)
+    static constexpr uint32_t SN = 200704;    // state snapshot [feature][64 dcol], bf16
+    static constexpr uint32_t ZR = 217088;    // z or r [128] fp32
+    static constexpr uint32_t CROW = 217600;  // c_t [128] fp32
+    static constexpr uint32_t BYTES = 218112;
+    static constexpr uint32_t T_P = 0, T_A = 128, T_D = 256, T_S = 384;
+    static_assert(BYTES + 1024 <= 232448, "shared memory budget");
+};
+
+__device__ __forceinline__ float bf16_at(const uint8_t* tile, int row, int col)
+{
+    return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(tile + swz128(row, col)));
+}
+
+template <int PASS, bool NS>
+__global__ void __launch_bounds__(kThreadsB, 1)
+    tc_bwd_kernel(int H, int N, int M, int G, int causal, const __nv_bfloat16* __restrict__ q,
+                  const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __restrict__ v,
+                  const float* __restrict__ W1, const float* __restrict__ W2,
+                  const __nv_bfloat16* __restrict__ outp, const float* __restrict__ den,
+                  const __nv_bfloat16* __restrict__ dout, float* __restrict__ acc_x,
+                  float* __restrict__ acc_v, float* __restrict__ dw_part, int* status)
+{
+    using L = BwCfg<NS>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const uint32_t sb = smem_u32(sm);
+    __shared__ uint32_t tmem_base_sh;
+    __shared__ __align__(8) uint64_t mbar;
+    __shared__ volatile int abort_flag;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int wg = warp >> 2, quad = warp & 3, t = 32 * quad + lane;
+    const int bh = blockIdx.x / G, g = blockIdx.x % G, h = bh % H;
+    const size_t base = (size_t)bh * N * 64;
+    float* zr = reinterpret_cast<float*>(sm + L::ZR);
+    float* crow = reinterpret_cast<float*>(sm + L::CROW);
+
+    // ---- set-up: this group's projection rows, zero state, C16 ----
+    for (int idx = tid; idx < L::P * 8; idx += kThreadsB) {
+        const int r = idx >> 3, c = idx & 7, f = 64 * g + (r & 63);
+        const float* w1 = W1 + ((size_t)h * M + f) * 64 + c * 8;
+        float x[8];
+        if (!NS) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[e] = w1[e];
+        } else {
+            const float* w2 = W2 + ((size_t)h * M + f) * 64 + c * 8;
+            const float sgn = r < 64 ? 1.f : -1.f;  // U = (W1+W2)/2, V = (W1-W2)/2
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[e] = 0.5f * (w1[e] + sgn * w2[e]);
+        }
+        st_shared_v4(sb + L::W + swz128(r, c * 8), pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]),
+                     pack_bf16(x[4], x[5]), pack_bf16(x[6], x[7]));
+    }
+    for (int idx = tid; idx < 16384 / 16; idx += kThreadsB) st_shared_v4(sb + L::SN + idx * 16, 0, 0, 0, 0);
+    for (int idx = tid; idx < 4096 / 16; idx += kThreadsB) {
+        const uint32_t fill = PASS == kPassF ? 0x3F803F80u : 0u;  // ones (z) or zeros (c rows)
+        st_shared_v4(sb + L::C16 + idx * 16, fill, fill, fill, fill);
+    }
+    for (int idx = tid; idx < 128; idx += kThreadsB) zr[idx] = 0.f;
+    if (tid == 0) {
+        mbar_init(&mbar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(&tmem_base_sh, 512);
+        tmem_relinquish();
+    }
+    fence_proxy_async();
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    const uint32_t tm = tmem_base_sh;
+    const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
+    uint32_t phase = 0;
+
+    auto handoff = [&]() {
+        fence_proxy_async();
+        fence_before_sync();
+        __syncthreads();
+    };
+    auto commit_wait = [&]() -> bool {  // thread 0 has issued MMAs: commit, all wait
+        if (tid == 0) mma_commit(&mbar);
+        bool ok = bar_wait(&mbar, phase, &abort_flag, status);
+        phase ^= 1;
+        ok = !__syncthreads_or(!ok);
+        fence_after_sync();
+        return ok;
+    };
+    auto adv = [](uint64_t d, uint32_t bytes) { return d + (bytes >> 4); };
+    const uint64_t dQ = sdesc(sb + L::Q, 16, 1024), dK = sdesc(sb + L::K, 16, 1024);
+    const uint64_t dV = sdesc(sb + L::V, 16, 1024), dG = sdesc(sb + L::GT, 16, 1024);
+    const uint64_t dW = sdesc(sb + L::W, 16, 1024), dWmn = sdesc(sb + L::W, 16384, 1024);
+    const uint64_t dPQ = sdesc(sb + L::PQ, 16, 1024), dPK = sdesc(sb + L::PK, 16, 1024);
+    const uint64_t dPQmn = sdesc(sb + L::PQ, 16384, 1024), dPKmn = sdesc(sb + L::PK, 16384, 1024);
+    const uint64_t dVmn = sdesc(sb + L::V, 16384, 1024), dGmn = sdesc(sb + L::GT, 16384, 1024);
+    const uint64_t dQmn = sdesc(sb + L::Q, 16384, 1024), dKmn = sdesc(sb + L::K, 16384, 1024);
+    const uint64_t dSN = sdesc(sb + L::SN, 16, 1024), dSNmn = sdesc(sb + L::SN, 16384, 1024);
+    const uint64_t dC16 = sdesc(sb + L::C16, 16, 1024);
+    const uint64_t dDAmn = sdesc(sb + L::Q, L::DA2 - L::Q, 1024);  // bf16(dA) as [query][key]
+    const uint64_t dAmn = sdesc(sb + L::DO, L::O - L::DO, 1024);   // bf16(A)  as [query][key]
+    constexpr uint32_t I_PROJ = idesc_bf16(128, L::P, 0, 0);
+    constexpr uint32_t I_KK128 = idesc_bf16(128, 128, 0, 0);   // K-major A, K-major B, N=128
+    constexpr uint32_t I_KM128 = idesc_bf16(128, 128, 0, 1);   // K-major A, MN-major B, N=128
+    constexpr uint32_t I_MM128 = idesc_bf16(128, 128, 1, 1);   // MN-major A and B, N=128
+    constexpr uint32_t I_KM64 = idesc_bf16(128, 64, 0, 1);
+    constexpr uint32_t I_MM64 = idesc_bf16(128, 64, 1, 1);
+    constexpr uint32_t I_M16 = idesc_bf16(128, 16, 1, 0);      // MN-major A, K-major B, N=16
+
+    // projection of a tile into T_P, then features of this group into dst (K-major rows)
+    auto project = [&](uint64_t dx) {
+        if (tid == 0) {
+            fence_after_sync();
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks)
+                mma_bf16(tm + L::T_P, adv(dx, ks * 32), adv(dW, ks * 32), I_PROJ, ks > 0);
+        }
+        return commit_wait();
+    };
+    auto features = [&](uint32_t dst, bool valid) {
+        float a[32], w[32];
+        tmem_ld16(tm_row + L::T_P + 32 * wg, *reinterpret_cast<float(*)[16]>(&a[0]));
+        tmem_ld16(tm_row + L::T_P + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+        if (NS) {
+            tmem_ld16(tm_row + L::T_P + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]));
+            tmem_ld16(tm_row + L::T_P + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
+        }
+        tmem_wait_ld();
+        uint32_t pc[16], ps[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            float s0, c0, s1, c1;
+            __sincosf(a[2 * i], &s0, &c0);
+            __sincosf(a[2 * i + 1], &s1, &c1);
+            if (NS) {
+                const float cw0 = __cosf(w[2 * i]), cw1 = __cosf(w[2 * i + 1]);
+                c0 *= cw0; s0 *= cw0; c1 *= cw1; s1 *= cw1;
+            }
+            if (!valid) { c0 = s0 = c1 = s1 = 0.f; }
+            pc[i] = pack_bf16(c0, c1);
+            ps[i] = pack_bf16(s0, s1);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint32_t off = swz128(t, (4 * wg + j) * 8);
+            st_shared_v4(dst + off, pc[4 * j], pc[4 * j + 1], pc[4 * j + 2], pc[4 * j + 3]);
+            st_shared_v4(dst + 16384 + off, ps[4 * j], ps[4 * j + 1], ps[4 * j + 2], ps[4 * j + 3]);
+        }
+    };
+    // Chain rule through the features of this thread's 32 frequencies: dphi from T_D plus
+    // the per-feature term zr * scale, then da written over the feature tile in place
+    // (s: da in the cos columns, zeros in the sin columns; n: du | dw).
+    auto feature_backward = [&](uint32_t tile, float scale, bool valid) {
+        float dc[32], ds[32];
+        tmem_ld16(tm_row + L::T_D + 32 * wg, *reinterpret_cast<float(*)[16]>(&dc[0]));
+        tmem_ld16(tm_row + L::T_D + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&dc[16]));
+        tmem_ld16(tm_row + L::T_D + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&ds[0]));
+        tmem_ld16(tm_row + L::T_D + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&ds[16]));
+        float a[32], w[32];
+        if (NS) {  // u, w recomputed by a fresh projection in T_P
+            tmem_ld16(tm_row + L::T_P + 32 * wg, *reinterpret_cast<float(*)[16]>(&a[0]));
+            tmem_ld16(tm_row + L::T_P + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+            tmem_ld16(tm_row + L::T_P + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]));
+            tmem_ld16(tm_row + L::T_P + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
+        }
+        tmem_wait_ld();
+        const uint8_t* tp = sm + (tile - sb);
+        uint32_t o1[16], o2[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            float r1[2], r2[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int fi = 2 * i + e, f = 32 * wg + fi;
+                const float dphic = dc[fi] + scale * zr[f], dphis = ds[fi] + scale * zr[64 + f];
+                if (!NS) {
+                    const float pc = bf16_at(tp, t, f), psn = bf16_at(tp + 16384, t, f);
+                    r1[e] = -psn * dphic + pc * dphis;
+                    r2[e] = 0.f;
+                } else {
+                    float su, cu, sw, cw;
+                    __sincosf(a[fi], &su, &cu);
+                    __sincosf(w[fi], &sw, &cw);
+                    r1[e] = cw * (-su * dphic + cu * dphis);
+                    r2[e] = -sw * (cu * dphic + su * dphis);
+                }
+                if (!valid) r1[e] = r2[e] = 0.f;
+            }
+            o1[i] = pack_bf16(r1[0], r1[1]);
+            o2[i] = pack_bf16(r2[0], r2[1]);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const uint32_t off = swz128(t, (4 * wg + j) * 8);
+            st_shared_v4(tile + off, o1[4 * j], o1[4 * j + 1], o1[4 * j + 2], o1[4 * j + 3]);
+            st_shared_v4(tile + 16384 + off, o2[4 * j], o2[4 * j + 1], o2[4 * j + 2], o2[4 * j + 3]);
+        }
+    };
+    // dx = da W (T_A[0,64)) and this chunk's dW = da^T x (T_A[64,128))
+    auto project_back = [&](uint64_t d_da, uint64_t d_da_mn, uint64_t d_x_mn) {
+        if (tid == 0) {
+            fence_after_sync();
+            const int kst = NS ? 8 : 4;  // K = P rows of W (s: the cos half only)
+            for (int ks = 0; ks < kst; ++ks)
+                mma_bf16(tm + L::T_A, adv(d_da, (ks >> 2) * 16384 + (ks & 3) * 32),
+                         adv(dWmn, ks * 2048), I_KM64, ks > 0);
+#pragma unroll
+            for (int ks = 0; ks < 8; ++ks)
+                mma_bf16(tm + L::T_A + 64, adv(d_da_mn, ks * 2048), adv(d_x_mn, ks * 2048), I_MM64,
+                         ks > 0);
+        }
+        return commit_wait();
+    };
+    // dW rows of this chunk (lane = row of this group's projection) into the partial slot
+    auto dw_accumulate = [&](bool first) {
+        float v_[64];
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            tmem_ld16(tm_row + L::T_A + 64 + 16 * j, *reinterpret_cast<float(*)[16]>(&v_[16 * j]));
+        tmem_wait_ld();
+        if (t < L::P && wg == 1) {
+            float4* dst = reinterpret_cast<float4*>(dw_part + ((size_t)blockIdx.x * 128 + t) * 64);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+                float4 old = first ? make_float4(0.f, 0.f, 0.f, 0.f) : dst[j];
+                dst[j] = make_float4(old.x + v_[4 * j], old.y + v_[4 * j + 1],
+                                     old.z + v_[4 * j + 2], old.w + v_[4 * j + 3]);
+            }
+        }
+    };
+    // state snapshot [feature][64] bf16 + column 64 (z or r) fp32, from T_S (lane = feature)
+    auto snapshot = [&]() {
+        float s_[32], zz[16];
+        tmem_ld16(tm_row + L::T_S + 32 * wg, *reinterpret_cast<float(*)[16]>(&s_[0]));
+        tmem_ld16(tm_row + L::T_S + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&s_[16]));
+        tmem_ld16(tm_row + L::T_S + 64, zz);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            st_shared_v4(sb + L::SN + swz128(t, (4 * wg + j) * 8),
+                         pack_bf16(s_[8 * j], s_[8 * j + 1]), pack_bf16(s_[8 * j + 2], s_[8 * j + 3]),
+                         pack_bf16(s_[8 * j + 4], s_[8 * j + 5]), pack_bf16(s_[8 * j + 6], s_[8 * j + 7]));
+        if (wg == 0) zr[t] = zz[0];
+    };
+    // rows of a [128 x 64] TMEM block (T_A[0,64)) added into an fp32 [token][64] accumulator
+    auto add_rows = [&](float* acc, int t0, bool valid) {
+        float v_[32];
+        tmem_ld16(tm_row + L::T_A + 32 * wg, *reinterpret_cast<float(*)[16]>(&v_[0]));
+        tmem_ld16(tm_row + L::T_A + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&v_[16]));
+        tmem_wait_ld();
+        if (valid) {
+            float* dst = acc + base + (size_t)(t0 + t) * 64 + 32 * wg;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) atomicAdd(dst + j, v_[j]);
+        }
+    };
+
+    const int nch = (N + kC - 1) / kC;
+    const float dscale = 1.0f / (float)M;  // den' = M den
+    for (int it = 0; it < nch; ++it) {
+        const int c = PASS == kPassF ? it : nch - 1 - it;
+        const int t0 = c * kC, CL = min(kC, N - t0);
+        const bool valid = t < CL;
+        // ---- loads: q, k, v tiles; g tile and c_t from dout, out, den ----
+        for (int i = tid; i < 3 * 1024; i += kThreadsB) {
+            const int tile = i >> 10, idx = i & 1023, r = idx >> 3, cc = idx & 7;
+            const __nv_bfloat16* src = tile == 0 ? q : (tile == 1 ? k : v);
+            uint4 val = make_uint4(0, 0, 0, 0);
+            if (r < CL) val = __ldg(reinterpret_cast<const uint4*>(src + base + (size_t)(t0 + r) * 64 + cc * 8));
+            const uint32_t dst = tile == 0 ? L::Q : (tile == 1 ? L::K : L::V);
+            st_shared_v4(sb + dst + swz128(r, cc * 8), val.x, val.y, val.z, val.w);
+        }
+        if (wg == 0) {
+            float gsc = 0.f, cval = 0.f;
+            uint32_t gp[32];
+            if (valid) {
+                const size_t row = base + (size_t)(t0 + t) * 64;
+                gsc = dscale / den[(size_t)bh * N + t0 + t];
+                float dot = 0.f;
+#pragma unroll
+                for (int cc = 0; cc < 8; ++cc) {
+                    const uint4 a4 = __ldg(reinterpret_cast<const uint4*>(dout + row + cc * 8));
+                    const uint4 o4 = __ldg(reinterpret_cast<const uint4*>(outp + row + cc * 8));
+                    const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w}, ow[4] = {o4.x, o4.y, o4.z, o4.w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float a0 = __uint_as_float(aw[e] << 16), a1 = __uint_as_float(aw[e] & 0xFFFF0000u);
+                        const float b0 = __uint_as_float(ow[e] << 16), b1 = __uint_as_float(ow[e] & 0xFFFF0000u);
+                        // c uses the same bf16-rounded g as the MMAs, so g.v_j + c_i cancels
+                        // exactly where out_i = v_j (e.g. the first causal position)
+                        const uint32_t gw = pack_bf16(a0 * gsc, a1 * gsc);
+                        gp[cc * 4 + e] = gw;
+                        dot = fmaf(__uint_as_float(gw << 16), b0,
+                                   fmaf(__uint_as_float(gw & 0xFFFF0000u), b1, dot));
+                    }
+                }
+                cval = -dot;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 32; ++e) gp[e] = 0u;
+            }
+#pragma unroll
+            for (int cc = 0; cc < 8; ++cc)
+                st_shared_v4(sb + L::GT + swz128(t, cc * 8), gp[4 * cc], gp[4 * cc + 1],
+                             gp[4 * cc + 2], gp[4 * cc + 3]);
+            crow[t] = cval;
+            if (PASS == kPassR)  // row 0 of the K-major [16][tokens] c operand
+                *reinterpret_cast<__nv_bfloat16*>(sm + L::C16 + (t >> 6) * 2048 + swz128(0, t & 63)) =
+                    __float2bfloat16_rn(cval);
+        }
+        handoff();
+        // ---- features of q and k for this group ----
+        if (!project(dQ)) goto done;
+        features(sb + L::PQ, valid);
+        handoff();
+        if (!project(dK)) goto done;
+        features(sb + L::PK, valid);
+        handoff();
+
+        if (PASS == kPassF) {
+            // dA = g v^T, then + c, mask, bf16 in place (A operand of dphi(q) = dA phi(K))
+            if (tid == 0) {
+                fence_after_sync();
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_bf16(tm + L::T_A, adv(dG, ks * 32), adv(dV, ks * 32), I_KK128, ks > 0);
+            }
+            if (!commit_wait()) goto done;
+            {
+                const float cv = crow[t];
+#pragma unroll
+                for (int b = 0; b < 2; ++b) {
+                    const uint32_t col = L::T_A + 64 * wg + 32 * b;
+                    float a[32];
+                    tmem_ld16(tm_row + col, *reinterpret_cast<float(*)[16]>(&a[0]));
+                    tmem_ld16(tm_row + col + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+                    tmem_wait_ld();
+                    uint32_t pk2[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const int j0 = 64 * wg + 32 * b + 2 * i;
+                        const bool m0 = (!causal || j0 <= t) && j0 < CL && valid;
+                        const bool m1 = (!causal || j0 + 1 <= t) && j0 + 1 < CL && valid;
+                        pk2[i] = pack_bf16(m0 ? a[2 * i] + cv : 0.f, m1 ? a[2 * i + 1] + cv : 0.f);
+                    }
+                    tmem_st16(tm_row + L::T_A + 64 * wg + 16 * b, pk2);
+                }
+                tmem_wait_st();
+            }
+            handoff();
+            // dphi(q) = dA phi(K) + g S^T; S += phi(K)^T v; z += phi(K)^T 1
+            if (tid == 0) {
+                fence_after_sync();
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_bf16_tmem_a(tm + L::T_D, tm + L::T_A + 64 * (ks >> 2) + 8 * (ks & 3),
+                                    adv(dPKmn, ks * 2048), I_KM128, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_bf16(tm + L::T_D, adv(dG, ks * 32), adv(dSN, ks * 32), I_KK128, 1u);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t acc = (it > 0 || ks > 0) ? 1u : 0u;
+                    mma_bf16(tm + L::T_S, adv(dPKmn, ks * 2048), adv(dVmn, ks * 2048), I_MM64, acc);
+                    mma_bf16(tm + L::T_S + 64, adv(dPKmn, ks * 2048),
+                             adv(dC16, (ks >> 2) * 2048 + (ks & 3) * 32), I_M16, acc);
+                }
+            }
+            if (!commit_wait()) goto done;
+            if (NS && !project(dQ)) goto done;  // u, w of q for the chain rule
+            feature_backward(sb + L::PQ, crow[t], valid);
+            handoff();
+            if (!project_back(dPQ, dPQmn, dQmn)) goto done;
+            add_rows(acc_x, t0, valid);
+            dw_accumulate(it == 0);
+            snapshot();
+            handoff();
+        } else {
+            // A = phi(Q) phi(K)^T -> mask -> bf16 [query][key] in [DO | O]
+            if (tid == 0) {
+                fence_after_sync();
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t kofs = (ks >> 2) * 16384 + (ks & 3) * 32;
+                    mma_bf16(tm + L::T_A, adv(dPQ, kofs), adv(dPK, kofs), I_KK128, ks > 0);
+                }
+            }
+            if (!commit_wait()) goto done;
+            auto mask_to_smem = [&](uint32_t blk0, float add) {
+#pragma unroll
+                for (int b = 0; b < 2; ++b) {
+                    float a[32];
+                    tmem_ld16(tm_row + L::T_A + 64 * wg + 32 * b, *reinterpret_cast<float(*)[16]>(&a[0]));
+                    tmem_ld16(tm_row + L::T_A + 64 * wg + 32 * b + 16,
+                              *reinterpret_cast<float(*)[16]>(&a[16]));
+                    tmem_wait_ld();
+                    uint32_t pk2[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const int j0 = 64 * wg + 32 * b + 2 * i;
+                        const bool m0 = (!causal || j0 <= t) && j0 < CL && valid;
+                        const bool m1 = (!causal || j0 + 1 <= t) && j0 + 1 < CL && valid;
+                        pk2[i] = pack_bf16(m0 ? a[2 * i] + add : 0.f, m1 ? a[2 * i + 1] + add : 0.f);
+                    }
+                    const uint32_t dst = blk0 + wg * 16384;  // key block wg
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        st_shared_v4(dst + swz128(t, (4 * b + j) * 8), pk2[4 * j], pk2[4 * j + 1],
+                                     pk2[4 * j + 2], pk2[4 * j + 3]);
+                }
+            };
+            mask_to_smem(sb + L::DO, 0.f);
+            fence_before_sync();
+            __syncthreads();
+            // dA = g v^T -> + c, mask -> bf16 [query][key] in [Q | DA2]
+            if (tid == 0) {
+                fence_after_sync();
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_bf16(tm + L::T_A, adv(dG, ks * 32), adv(dV, ks * 32), I_KK128, ks > 0);
+            }
+            if (!commit_wait()) goto done;
+            mask_to_smem(sb + L::Q, crow[t]);
+            handoff();
+            // dphi(k) = dA^T phi(Q) + v R^T;  dv = A^T g + phi(K) R;  R += phi(Q)^T g;
+            // r += phi(Q)^T c
+            if (tid == 0) {
+                fence_after_sync();
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_bf16(tm + L::T_D, adv(dDAmn, ks * 2048), adv(dPQmn, ks * 2048), I_MM128, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_bf16(tm + L::T_D, adv(dV, ks * 32), adv(dSN, ks * 32), I_KK128, 1u);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_bf16(tm + L::T_A, adv(dAmn, ks * 2048), adv(dGmn, ks * 2048), I_MM64, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_bf16(tm + L::T_A, adv(dPK, (ks >> 2) * 16384 + (ks & 3) * 32),
+                             adv(dSNmn, ks * 2048), I_KM64, 1u);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) {
+                    const uint32_t acc = (it > 0 || ks > 0) ? 1u : 0u;
+                    mma_bf16(tm + L::T_S, adv(dPQmn, ks * 2048), adv(dGmn, ks * 2048), I_MM64, acc);
+                    mma_bf16(tm + L::T_S + 64, adv(dPQmn, ks * 2048),
+                             adv(dC16, (ks >> 2) * 2048 + (ks & 3) * 32), I_M16, acc);
+                }
+            }
+            if (!commit_wait()) goto done;
+            add_rows(acc_v, t0, valid);  // dv of this group
+            fence_before_sync();
+            __syncthreads();
+            if (NS && !project(dK)) goto done;  // u, w of k for the chain rule
+            feature_backward(sb + L::PK, 1.0f, valid);
+            handoff();
+            if (!project_back(dPK, dPKmn, dKmn)) goto done;
+            add_rows(acc_x, t0, valid);
+            dw_accumulate(false);
+            snapshot();
+            handoff();
+        }
+    }
+done:
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    if (warp == 0) tmem_dealloc(tm, 512);
+}
+
+// dW over the batch in a fixed order.  Partial slots [bh * G + g][row][64]; s: rows < 64
+// are frequencies 64g + row; n: rows < 64 are dU, rows >= 64 are dV of frequency 64g + row%64.
+__global__ void tc_dw_reduce_kernel(int B, int H, int M, int G, int nonstat,
+                                    const float* __restrict__ part, float* __restrict__ dW1,
+                                    float* __restrict__ dW2)
+{
+    const size_t total = (size_t)H * M * 64;
+    for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int h = (int)(idx / ((size_t)M * 64));
+        const int f = (int)((idx / 64) % M), e = (int)(idx % 64);
+        const int g = f / 64, r = f % 64;
+        float a = 0.f, b2 = 0.f;
+        for (int b = 0; b < B; ++b) {
+            const float* p = part + ((size_t)((b * H + h) * G + g) * 128) * 64;
+            a += p[(size_t)r * 64 + e];
+            if (nonstat) b2 += p[(size_t)(64 + r) * 64 + e];
+        }
+        if (!nonstat) {
+            dW1[idx] = a;
+        } else {
+            dW1[idx] = 0.5f * (a + b2);
+            dW2[idx] = 0.5f * (a - b2);
+        }
+    }
+}
+
+__global__ void tc_to_bf16_kernel(size_t n, const float* __restrict__ a, const float* __restrict__ b,
+                                  const float* __restrict__ c, __nv_bfloat16* __restrict__ oa,
+                                  __nv_bfloat16* __restrict__ ob, __nv_bfloat16* __restrict__ oc)
+{
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (size_t)gridDim.x * blockDim.x) {
+        oa[i] = __float2bfloat16_rn(a[i]);
+        ob[i] = __float2bfloat16_rn(b[i]);
+        oc[i] = __float2bfloat16_rn(c[i]);
+    }
+}
+
+template <bool NS>
+cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const void* v,
+                       const float* W1, const float* W2, const void* out, const float* den,
+                       const void* dout, void* dq, void* dk, void* dv, float* dW1, float* dW2,
+                       void* scratch, int* status, cudaStream_t s)
+{
+    const int BH = p.B * p.H, G = p.M / 64;
+    const size_t n = (size_t)BH * p.N * 64;
+    float* acc_q = static_cast<float*>(scratch);
+    float* acc_k = acc_q + n;
+    float* acc_v = acc_k + n;
+    float* part = acc_v + n;
+    cudaError_t e = cudaMemsetAsync(acc_q, 0, 3 * n * sizeof(float), s);
+    if (e != cudaSuccess) return e;
+    const int smem = (int)BwCfg<NS>::BYTES + 1024;
+    auto kf = tc_bwd_kernel<kPassF, NS>;
+    auto kr = tc_bwd_kernel<kPassR, NS>;
+    if ((e = cudaFuncSetAttribute(kf, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return e;
+    if ((e = cudaFuncSetAttribute(kr, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return e;
+    typedef const __nv_bfloat16* CB;
+    kf<<<BH * G, kThreadsB, smem, s>>>(p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k, (CB)v, W1, W2,
+                                       (CB)out, den, (CB)dout, acc_q, acc_v, part, status);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    kr<<<BH * G, kThreadsB, smem, s>>>(p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k, (CB)v, W1, W2,
+                                       (CB)out, den, (CB)dout, acc_k, acc_v, part, status);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const size_t work = (size_t)p.H * p.M * 64;
+    tc_dw_reduce_kernel<<<(int)std::min<size_t>((work + 255) / 256, 152 * 8), 256, 0, s>>>(
+        p.B, p.H, p.M, G, p.nonstat, part, dW1, dW2);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    tc_to_bf16_kernel<<<152 * 8, 256, 0, s>>>(n, acc_q, acc_k, acc_v, (__nv_bfloat16*)dq,
+                                               (__nv_bfloat16*)dk, (__nv_bfloat16*)dv);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+// Causal only: the running prefix (pass F) and suffix (pass R) states are exactly the
+// inter-chunk terms of the causal gradient.
+bool tc_bwd_supported(const Problem& p)
+{
+    return p.bf16 && p.causal && p.d == 64 && (p.M == 64 || p.M == 128);
+}
+
+size_t tc_bwd_ws_bytes(const Problem& p)
+{
+    const size_t BH = (size_t)p.B * p.H, G = (size_t)p.M / 64;
+    return (3 * BH * p.N * 64 + BH * G * 128 * 64) * sizeof(float);
+}
+
+cudaError_t launch_tc_bwd(const Problem& p, const void* q, const void* k, const void* v,
+                          const float* W1, const float* W2, const void* out, const float* den,
+                          const void* dout, void* dq, void* dk, void* dv, float* dW1, float* dW2,
+                          void* scratch, int* status, cudaStream_t s)
+{
+    if (p.nonstat)
+        return launch_bwd<true>(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1, dW2, scratch,
+                                status, s);
+    return launch_bwd<false>(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1, dW2, scratch,
+                             status, s);
+}
+
+}  // namespace flex
