@@ -221,6 +221,15 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const void* tmap, int 
         : "memory");
 }
 
+// TMA: prefetch a 3-D tile into L2 (no shared memory, no completion tracking).
+__device__ __forceinline__ void tma_prefetch_3d(const void* tmap, int c0, int c1, int c2)
+{
+    asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
+                     (uint64_t)tmap),
+                 "r"(c0), "r"(c1), "r"(c2)
+                 : "memory");
+}
+
 // Waits for the phase with the given parity to complete.  Gives up after `limit` polls
 // (each poll itself blocks for a hardware-defined time slice) and returns false.
 __device__ __forceinline__ bool mbar_wait(void* mbar, uint32_t parity, uint32_t limit)

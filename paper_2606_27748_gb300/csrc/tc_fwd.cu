@@ -12,9 +12,13 @@
 // are unscaled ([cos, sin] instead of M^{-1/2}[cos, sin]): the factor cancels in the
 // output, and only the stored denominator is rescaled (den = den' / M).
 //
-// Warp roles (576 threads), handshakes on mbarriers:
+// Warp roles (608 threads), handshakes on mbarriers:
 //   warp 0      TMA: q, k, v chunk tiles (128B swizzle) into shared memory
-//   warp 1      one thread issues every tcgen05.mma; owns the tensor-memory allocation
+//   warp 1      one thread issues the attention MMAs (QK, numerator, state, A V); owns the
+//               tensor-memory allocation
+//   warp 18     one thread issues the projection MMAs.  A thread that issues an MMA blocks
+//               while the tensor core's queue is full, so projections get their own issuer
+//               and never wait behind a long attention step
 //   warps 2-9   features: projection (TMEM) -> cos/sin -> bf16 phi tiles (shared memory);
 //               warps 2-5 take frequencies 0-31 of a group, warps 6-9 frequencies 32-63
 //   warps 10-17 epilogue, two halves of 4 warps: causal mask + bf16 of A (written back
@@ -49,8 +53,9 @@ namespace {
 using namespace tc;
 
 constexpr int kC = 128;            // tokens per chunk = MMA M
-constexpr int kThreadsTC = 576;    // 18 warps
+constexpr int kThreadsTC = 608;    // 19 warps
 constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kWarpEW = 10, kEpiWarps = 8;
+constexpr int kWarpProj = 18;
 
 template <bool NS, int G>
 struct Cfg {
@@ -75,7 +80,7 @@ struct Cfg {
 
 struct Bars {
     uint64_t x_full[2], x_free[2], v_full[2], v_free[2];
-    uint64_t p_full, p_free, phiq_full, phik_full, phi_free;
+    uint64_t p_full, p_free, phiq_full, phik_full, phiq_free, phik_free;
     uint64_t attn_done, a_ready, o_ready, epi_done;
 };
 
@@ -148,7 +153,8 @@ __global__ void __maxnreg__(96)
         mbar_init(&bars.p_free, 8);
         mbar_init(&bars.phiq_full, 8);
         mbar_init(&bars.phik_full, 8);
-        mbar_init(&bars.phi_free, 1);
+        mbar_init(&bars.phiq_free, 1);
+        mbar_init(&bars.phik_free, 1);
         mbar_init(&bars.attn_done, 1);
         mbar_init(&bars.a_ready, kEpiWarps);
         mbar_init(&bars.o_ready, 1);
@@ -185,6 +191,11 @@ __global__ void __maxnreg__(96)
             };
             for (int c = 0; c < ce; ++c) {
                 const int t0 = c * kC;
+                if (c + 1 < ce) {  // the next chunk's tiles into L2 while this one is used
+                    if (c + 1 >= cb) tma_prefetch_3d(&tmap_q, 0, t0 + kC, bh);
+                    tma_prefetch_3d(&tmap_k, 0, t0 + kC, bh);
+                    tma_prefetch_3d(&tmap_v, 0, t0 + kC, bh);
+                }
                 if (c >= cb) {
                     if (!load(0, &tmap_q, t0) || !load(1, &tmap_k, t0)) break;
                 } else {
@@ -200,19 +211,15 @@ __global__ void __maxnreg__(96)
                 tma_load_3d(sb + (vb ? L::V1 : L::V0), &tmap_v, 0, t0, bh, &bars.v_full[vb]);
             }
         }
-    } else if (warp == kWarpMMA) {
-        // ================= MMA issue (one thread) =================
+    } else if (warp == kWarpMMA || warp == kWarpProj) {
+        // ================= MMA issue (one thread per role) =================
         if (lane == 0) {
             constexpr uint32_t I_PROJ = idesc_bf16(128, L::P, 0, 0);
             constexpr uint32_t I_QK = idesc_bf16(128, 128, 0, 0);
             constexpr uint32_t I_QS = idesc_bf16(128, 80, 0, 0);
             constexpr uint32_t I_KV = idesc_bf16(128, 80, 1, 1);
             constexpr uint32_t I_AV = idesc_bf16(128, 80, 0, 1);
-            uint32_t ph_xfull[2] = {0, 0}, ph_vfull[2] = {0, 0};
-            uint32_t ph_pfree = 0, ph_phiq = 0, ph_phik = 0, ph_aready = 0, ph_epi = 0;
-            int nproj = 0, pending_av = -1;
             bool ok = true;
-
             auto wait = [&](uint64_t* bar, uint32_t& ph) {
                 if (!ok) return;
                 ok = bar_wait(bar, ph, &abort_flag, status);
@@ -220,116 +227,104 @@ __global__ void __maxnreg__(96)
             };
             // Descriptors are built once; an operand K step adds its byte offset / 16 to
             // the start-address field (addresses stay below 256 KB: no carry out).
-            const uint64_t d_x[2] = {sdesc(sb + L::X0, 16, 1024), sdesc(sb + L::X1, 16, 1024)};
-            const uint64_t d_w = sdesc(sb + L::W, 16, 1024);
-            const uint64_t d_pq = sdesc(sb + L::PQ, 16, 1024);
-            const uint64_t d_pk = sdesc(sb + L::PK, 16, 1024);
-            const uint64_t d_pk_mn = sdesc(sb + L::PK, 16384, 1024);
-            const uint64_t d_sx = sdesc(sb + L::SX, 16, 1024);
-            const uint64_t d_v[2] = {sdesc(sb + L::V0, L::VONE - L::V0, 1024),
-                                     sdesc(sb + L::V1, L::VONE - L::V1, 1024)};
             auto adv = [](uint64_t d, uint32_t bytes) { return d + (bytes >> 4); };
-            auto proj = [&](int xb, int g) {
-                if (nproj > 0) wait(&bars.p_free, ph_pfree);
-                if (!ok) return;
-                fence_after_sync();
-                const uint64_t wd = adv(d_w, g * L::P * 128);
+            if (warp == kWarpProj) {
+                // projections: per chunk, per group, q (main chunks) then k
+                const uint64_t d_x[2] = {sdesc(sb + L::X0, 16, 1024), sdesc(sb + L::X1, 16, 1024)};
+                const uint64_t d_w = sdesc(sb + L::W, 16, 1024);
+                uint32_t ph_xfull[2] = {0, 0}, ph_pfree = 0;
+                int nproj = 0;
+                for (int c = 0; c < ce && ok; ++c) {
+                    const bool main = c >= cb;
+                    for (int g = 0; g < G && ok; ++g) {
+                        for (int which = main ? 0 : 1; which < 2 && ok; ++which) {
+                            const int buf = which == 0 ? 0 : (main ? 1 : ((c & 1) ? 0 : 1));
+                            if (g == 0) wait(&bars.x_full[buf], ph_xfull[buf]);
+                            if (nproj > 0) wait(&bars.p_free, ph_pfree);
+                            if (!ok) break;
+                            fence_after_sync();
+                            const uint64_t wd = adv(d_w, g * L::P * 128);
 #pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    mma_bf16(tm + L::T_P, adv(d_x[xb], ks * 32), adv(wd, ks * 32), I_PROJ, ks > 0);
-                mma_commit(&bars.p_full);
-                ++nproj;
-            };
-            auto av = [&](int cc) {
-                wait(&bars.a_ready, ph_aready);
-                if (!ok) return;
-                fence_after_sync();
-                const uint64_t vd = d_v[cc & 1];
-#pragma unroll
-                for (int ks = 0; ks < 8; ++ks)  // keys 16ks..16ks+15: bf16 A columns
-                    mma_bf16_tmem_a(tm + L::T_O, tm + L::T_A + 64 * (ks >> 2) + 8 * (ks & 3),
-                                    adv(vd, ks * 2048), I_AV, 1u);
-                mma_commit(&bars.o_ready);
-                mma_commit(&bars.v_free[cc & 1]);
-            };
-            auto attn = [&](int c, int g, bool main) {
-                if (main) wait(&bars.phiq_full, ph_phiq);
-                wait(&bars.phik_full, ph_phik);
-                if (g == 0) {
-                    wait(&bars.v_full[c & 1], ph_vfull[c & 1]);
-                    if (main) wait(&bars.epi_done, ph_epi);
-                }
-                if (!ok) return;
-                fence_after_sync();
-                const uint64_t vd = d_v[c & 1];
-                const uint64_t sxd = adv(d_sx, g * L::SX_GROUP);
-                const uint32_t acc_s = c > 0 ? 1u : 0u;
-                if (main) {
-#pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) {  // K = 128 features of group g
-                        const uint32_t kofs = (ks >> 2) * 16384 + (ks & 3) * 32;
-                        const uint64_t aq = adv(d_pq, kofs);
-                        const uint32_t acc = (g > 0 || ks > 0) ? 1u : 0u;
-                        mma_bf16(tm + L::T_A, aq, adv(d_pk, kofs), I_QK, acc);
-                        mma_bf16(tm + L::T_O, aq,
-                                 adv(sxd, (ks >> 2) * L::SX_BLOCK + (ks & 3) * 32), I_QS, acc);
+                            for (int ks = 0; ks < 4; ++ks)
+                                mma_bf16(tm + L::T_P, adv(d_x[buf], ks * 32), adv(wd, ks * 32),
+                                         I_PROJ, ks > 0);
+                            mma_commit(&bars.p_full);
+                            if (g == G - 1) mma_commit(&bars.x_free[buf]);
+                            ++nproj;
+                        }
                     }
                 }
+            } else {
+                // attention MMAs of each group, then A V of each main chunk
+                const uint64_t d_pq = sdesc(sb + L::PQ, 16, 1024);
+                const uint64_t d_pk = sdesc(sb + L::PK, 16, 1024);
+                const uint64_t d_pk_mn = sdesc(sb + L::PK, 16384, 1024);
+                const uint64_t d_sx = sdesc(sb + L::SX, 16, 1024);
+                const uint64_t d_v[2] = {sdesc(sb + L::V0, L::VONE - L::V0, 1024),
+                                         sdesc(sb + L::V1, L::VONE - L::V1, 1024)};
+                uint32_t ph_vfull[2] = {0, 0};
+                uint32_t ph_phiq = 0, ph_phik = 0, ph_aready = 0, ph_epi = 0;
+                for (int c = 0; c < ce && ok; ++c) {
+                    const bool main = c >= cb;
+                    const uint64_t vd = d_v[c & 1];
+                    for (int g = 0; g < G && ok; ++g) {
+                        if (main) wait(&bars.phiq_full, ph_phiq);
+                        wait(&bars.phik_full, ph_phik);
+                        if (g == 0) {
+                            wait(&bars.v_full[c & 1], ph_vfull[c & 1]);
+                            if (main) wait(&bars.epi_done, ph_epi);
+                        }
+                        if (!ok) break;
+                        fence_after_sync();
+                        if (main) {
+                            const uint64_t sxd = adv(d_sx, g * L::SX_GROUP);
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks)  // K = 128 tokens of the chunk
-                    mma_bf16(tm + L::T_S + 80 * g, adv(d_pk_mn, ks * 2048), adv(vd, ks * 2048),
-                             I_KV, (acc_s | (ks > 0)) ? 1u : 0u);
-                mma_commit(&bars.phi_free);
-                if (g == G - 1) {
-                    if (main || c == cb - 1) mma_commit(&bars.attn_done);
-                    if (!main) mma_commit(&bars.v_free[c & 1]);
-                }
-            };
-
-            // Job stream: per chunk, for each group, a q job (main chunks) and a k job.  The
-            // projection of a job is issued before the attention MMAs of the group the
-            // previous job completed, so the tensor pipe (in order) never makes the feature
-            // warps wait for a projection stuck behind a long attention step.
-            int pa_c = -1, pa_g = 0;
-            bool pa_main = false;
-            for (int c = 0; c < ce && ok; ++c) {
-                const bool main = c >= cb;
-                for (int g = 0; g < G && ok; ++g) {
-                    for (int which = main ? 0 : 1; which < 2 && ok; ++which) {
-                        const int buf = which == 0 ? 0 : (main ? 1 : ((c & 1) ? 0 : 1));
-                        if (g == 0) wait(&bars.x_full[buf], ph_xfull[buf]);
-                        proj(buf, g);
-                        if (g == G - 1) mma_commit(&bars.x_free[buf]);
-                        if (pa_c >= 0) {
-                            attn(pa_c, pa_g, pa_main);
-                            pa_c = -1;
-                        }
-                        if (which == 1) {
-                            if (g == 0 && main && pending_av >= 0) {
-                                av(pending_av);
-                                pending_av = -1;
+                            for (int ks = 0; ks < 8; ++ks) {  // K = 128 features of group g
+                                const uint32_t kofs = (ks >> 2) * 16384 + (ks & 3) * 32;
+                                const uint64_t aq = adv(d_pq, kofs);
+                                const uint32_t acc = (g > 0 || ks > 0) ? 1u : 0u;
+                                mma_bf16(tm + L::T_A, aq, adv(d_pk, kofs), I_QK, acc);
+                                mma_bf16(tm + L::T_O, aq,
+                                         adv(sxd, (ks >> 2) * L::SX_BLOCK + (ks & 3) * 32), I_QS,
+                                         acc);
                             }
-                            pa_c = c;  // this k job completes group g
-                            pa_g = g;
-                            pa_main = main;
-                            if (g == G - 1 && main) pending_av = c;
+                            mma_commit(&bars.phiq_free);  // phi(Q) no longer read
                         }
+                        const uint32_t acc_s = c > 0 ? 1u : 0u;
+#pragma unroll
+                        for (int ks = 0; ks < 8; ++ks)  // K = 128 tokens of the chunk
+                            mma_bf16(tm + L::T_S + 80 * g, adv(d_pk_mn, ks * 2048),
+                                     adv(vd, ks * 2048), I_KV, (acc_s | (ks > 0)) ? 1u : 0u);
+                        mma_commit(&bars.phik_free);  // phi(K) no longer read
+                        if (g == G - 1) {
+                            if (main || c == cb - 1) mma_commit(&bars.attn_done);
+                            if (!main) mma_commit(&bars.v_free[c & 1]);
+                        }
+                    }
+                    if (main && ok) {
+                        wait(&bars.a_ready, ph_aready);
+                        if (!ok) break;
+                        fence_after_sync();
+#pragma unroll
+                        for (int ks = 0; ks < 8; ++ks)  // keys 16ks..16ks+15: bf16 A columns
+                            mma_bf16_tmem_a(tm + L::T_O, tm + L::T_A + 64 * (ks >> 2) + 8 * (ks & 3),
+                                            adv(vd, ks * 2048), I_AV, 1u);
+                        mma_commit(&bars.o_ready);
+                        mma_commit(&bars.v_free[c & 1]);
                     }
                 }
             }
-            if (ok && pa_c >= 0) attn(pa_c, pa_g, pa_main);
-            if (ok && pending_av >= 0) av(pending_av);
         }
     } else if (warp < kWarpEW) {
         // ================= features =================
         const int half = (warp - kWarpFW) >> 2, quad = warp & 3, t = 32 * quad + lane;
         const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16) + L::T_P;
         uint32_t ph_pfull = 0;
-        int n = 0;  // groups processed so far
+        int n = 0, nq = 0;  // groups processed so far (all / main chunks)
         for (int c = 0; c < ce; ++c) {
             const bool main = c >= cb;
             const bool valid = t < min(kC, N - c * kC);
-            for (int g = 0; g < G; ++g, ++n) {
+            for (int g = 0; g < G; ++g, ++n, nq += main ? 1 : 0) {
                 for (int which = main ? 0 : 1; which < 2; ++which) {  // 0: q, 1: k
                     if (!bar_wait(&bars.p_full, ph_pfull, &abort_flag, status)) goto fw_out;
                     ph_pfull ^= 1;
@@ -360,7 +355,11 @@ __global__ void __maxnreg__(96)
                         pc[i] = pack_bf16(c0, c1);
                         ps[i] = pack_bf16(s0, s1);
                     }
-                    if (n > 0 && !bar_wait(&bars.phi_free, (n - 1) & 1, &abort_flag, status))
+                    // the tile is free once the previous group's MMAs that read it are done
+                    if (which == 0 ? (nq > 0 && !bar_wait(&bars.phiq_free, (nq - 1) & 1,
+                                                          &abort_flag, status))
+                                   : (n > 0 && !bar_wait(&bars.phik_free, (n - 1) & 1,
+                                                         &abort_flag, status)))
                         goto fw_out;
                     const uint32_t dst = sb + (which ? L::PK : L::PQ);
 #pragma unroll

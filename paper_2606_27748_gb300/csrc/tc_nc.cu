@@ -154,6 +154,10 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
             uint32_t ph_x[2] = {0, 0}, ph_v[2] = {0, 0};
             for (int i = 0; i < nc; ++i) {
                 const int b = i & 1, t0 = (c0 + i) * kC;
+                if (i + 2 < nc) {  // two chunks ahead into L2
+                    tma_prefetch_3d(&tmap_x, 0, t0 + 2 * kC, bh);
+                    if (MODE == kState) tma_prefetch_3d(&tmap_v, 0, t0 + 2 * kC, bh);
+                }
                 if (i >= 2) {
                     if (!bar_wait(&bars.x_free[b], ph_x[b], &abort_flag, status)) break;
                     ph_x[b] ^= 1;
