@@ -48,7 +48,7 @@ cudaError_t launch_simt_bwd(const Problem& p, const void* q, const void* k, cons
 
 // ---- tensor-core path (bf16 storage, d = 64, M in {64, 128}) ------------------------
 bool tc_fwd_supported(const Problem& p);
-int tc_fwd_splits(const Problem& p, int sms);  // CTAs per sequence (1-3)
+int tc_fwd_splits(const Problem& p, int sms);  // segments per sequence (1-3)
 cudaError_t launch_tc_fwd(const Problem& p, const void* q, const void* k, const void* v,
                           const float* W1, const float* W2, void* out, float* den, int* status,
                           cudaStream_t s);

@@ -46,6 +46,22 @@ __device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity, volatil
     }
 }
 
+// bar_wait for a barrier that other CTAs of the cluster arrive on (acquire at cluster scope).
+__device__ __forceinline__ bool bar_wait_cluster(uint64_t* bar, uint32_t parity,
+                                                 volatile int* abort_flag, int* status)
+{
+    const long long t0 = clock64();
+    while (true) {
+        if (mbar_try_wait_cluster(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (clock64() - t0 > kWaitCycles) {
+            *abort_flag = 1;
+            atomicExch(status, (int)FLEX_ETIMEOUT);
+            return false;
+        }
+    }
+}
+
 
 // ---- host side ----------------------------------------------------------------------------
 
