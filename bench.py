@@ -32,7 +32,7 @@ sys.path.insert(0, ROOT)
 from paper_2606_27748_gb300 import workloads  # noqa: E402
 
 METRIC = "RFF linear-attn fwd tokens/s (N=16K causal) & % of bf16 tensor/HBM roofline"
-METRIC_TRAIN = "RFF linear-attn fwd+bwd training-step tokens/s & % of HBM roofline"
+METRIC_TRAIN = "RFF linear-attn fwd+bwd training-step tokens/s & % of roofline"
 L2_BYTES = 129e6
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
@@ -65,15 +65,62 @@ def algorithmic_bytes(w):
 
 
 def algorithmic_flops(w):
+    """Forward: the two projections and the state read and update; a training step counts
+    the backward as twice the forward."""
     mc = 2 * w.M if w.variant == "n" else w.M
     per = 2 * (2 * w.d * mc) + 2 * (2 * (2 * w.M) * w.d)
+    return w.token_heads * per * (3 if w.backward else 1)
+
+
+def sincos_count(w):
+    """sin/cos evaluations on the path: per feature vector 2M (s: cos a, sin a) or 3M (n:
+    cos u, sin u, cos w); the forward builds phi(q) and phi(k); the backward rebuilds both
+    and, for n, also needs sin w (4M per vector)."""
+    fwd = (3 if w.variant == "n" else 2) * w.M
+    bwd = (4 if w.variant == "n" else 2) * w.M
+    per = 2 * fwd + (2 * bwd if w.backward else 0)
     return w.token_heads * per
 
 
-def source_digest():
+SFU_PER_CLK_PER_SM = 16  # sin/cos results per clock per SM (measured 15.9 by a probe)
+
+
+def roofline(w, kernel_ms, peaks, sms, traffic):
+    """The three roofs of the path; `bound` is the unit with the longest time at peak."""
+    sec = kernel_ms * 1e-3
+    nbytes = algorithmic_bytes(w)
+    if w.backward:  # + backward: read q, k, v, out, dO; write dq, dk, dv
+        nbytes += w.token_heads * 8 * w.d * elem_bytes(w)
+    flops, ops = algorithmic_flops(w), sincos_count(w)
+    sfu_peak = SFU_PER_CLK_PER_SM * sms * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e9  # G/s
+    roofs = {
+        "hbm": (nbytes / sec / 1e9, peaks["hbm_gbs"], "GB/s", nbytes / (peaks["hbm_gbs"] * 1e9)),
+        "tensor": (flops / sec / 1e12, peaks["bf16_tflops"], "TFLOP/s",
+                   flops / (peaks["bf16_tflops"] * 1e12)),
+        "alu": (ops / sec / 1e9, sfu_peak, "Gsincos/s", ops / (sfu_peak * 1e9)),
+    }
+    bound = max(roofs, key=lambda k: roofs[k][3])
+    a, pk, unit, _ = roofs[bound]
+    return {"bound": bound, "achieved": a, "peak": pk, "unit": unit, "frac": a / pk,
+            "traffic": traffic,
+            "algorithmic_bytes_per_launch": nbytes, "algorithmic_flops_per_launch": flops,
+            "sincos_per_launch": ops,
+            "time_at_peak_us": {k: v[3] * 1e6 for k, v in roofs.items()},
+            "fracs": {k: v[0] / v[1] for k, v in roofs.items()},
+            "alu_peak_note": f"{SFU_PER_CLK_PER_SM} sin/cos per clock per SM x {sms} SMs x "
+                             f"{peaks.get('sm_max_mhz', 2070.0):.0f} MHz",
+            "kernel_ms": kernel_ms}
+
+
+def source_digest(files=None):
+    """sha256 over the given kernel sources (paths relative to the repository root), or
+    over every file of csrc/."""
+    if files is None:
+        files = sorted(os.path.relpath(f, ROOT) for f in
+                       glob.glob(os.path.join(ROOT, "paper_2606_27748_gb300", "csrc", "*")))
     h = hashlib.sha256()
-    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2606_27748_gb300", "csrc", "*"))):
-        h.update(open(f, "rb").read())
+    for f in files:
+        h.update(open(os.path.join(ROOT, f), "rb").read())
     return h.hexdigest()
 
 
@@ -83,15 +130,16 @@ def load_peaks():
     return FALLBACK_PEAKS, "fallback"
 
 
-def recorded_traffic(w, kernel_digest):
-    """DRAM bytes per launch from the committed ncu summary, if it is for this source."""
+def recorded_traffic(w):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel sources it was
+    taken from are unchanged."""
     if not os.path.exists(TRAFFIC_FILE):
         return None
     try:
         t = json.load(open(TRAFFIC_FILE)).get(w.name)
-    except ValueError:
-        return None
-    if not t or t.get("source_sha256") != kernel_digest:
+        if not t or t.get("source_sha256") != source_digest(t.get("sources")):
+            return None
+    except (ValueError, OSError):
         return None
     return t.get("dram_bytes_per_launch")
 
@@ -218,6 +266,26 @@ def run_reference(args, w):
 
 
 # ---------------------------------------------------------------------------------------
+# Multi-rank bookkeeping: every rank runs a full replica; the step time of the job is the
+# maximum over ranks and the value counts the work of all ranks.
+# ---------------------------------------------------------------------------------------
+def max_over_ranks(values, world, device="cpu"):
+    """Element-wise maximum of a list of floats over all ranks (identity when world = 1)."""
+    if world <= 1:
+        return list(values)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(list(values), dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def job_value(world, tokens_per_rank, ms_per_step):
+    """Whole-job tokens/s: the tokens all ranks processed over the slowest rank's time."""
+    return world * tokens_per_rank / (ms_per_step * 1e-3)
+
+
+# ---------------------------------------------------------------------------------------
 # Our arm.
 # ---------------------------------------------------------------------------------------
 def run_ours(args, w):
@@ -296,12 +364,9 @@ def run_ours(args, w):
     flexattn.check_status(ws)
     total_ms = t_start.elapsed_time(t_end)
     kernel_ms = sum(a.elapsed_time(b) for a, b in ev) / K
-    if world > 1:
-        t = torch.tensor([total_ms, kernel_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms, kernel_ms = t.tolist()
+    total_ms, kernel_ms = max_over_ranks([total_ms, kernel_ms], world, dev)
     ms_per_step = total_ms / K
-    value = world * w.tokens / (ms_per_step * 1e-3)
+    value = job_value(world, w.tokens, ms_per_step)
 
     # End to end through the same C-ABI call with host buffers: H2D of q, k, v from pinned
     # memory, the forward, D2H of out, every step.
@@ -327,28 +392,16 @@ def run_ours(args, w):
         torch.cuda.synchronize()
         barrier()
         e2e_ms = a.elapsed_time(b) / K
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = t.item()
+        e2e_ms = max_over_ranks([e2e_ms], world, dev)[0]
         h2d = sum(host[n].numel() * host[n].element_size() for n in "qkv")
-        e2e = {"value": world * w.tokens / (e2e_ms * 1e-3), "unit": "tokens/s",
+        e2e = {"value": job_value(world, w.tokens, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": host_out.numel() * host_out.element_size()}
 
     peaks, peaks_src = load_peaks()
-    nbytes = algorithmic_bytes(w)
-    if w.backward:  # + backward: read q, k, v, out, dO; write dq, dk, dv
-        nbytes += w.token_heads * 8 * w.d * elem_bytes(w)
-    achieved = nbytes / (kernel_ms * 1e-3) / 1e9
-    roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-            "frac": achieved / peaks["hbm_gbs"], "traffic": recorded_traffic(w, source_digest()),
-            "peak_source": peaks_src,
-            "algorithmic_bytes_per_launch": nbytes,
-            "algorithmic_tflops": algorithmic_flops(w) / (kernel_ms * 1e-3) / 1e12,
-            "tensor_frac_of_burst_peak": algorithmic_flops(w) / (kernel_ms * 1e-3) / 1e12
-            / peaks["bf16_tflops"],
-            "kernel_ms": kernel_ms}
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    roof = roofline(w, kernel_ms, peaks, sms, recorded_traffic(w))
+    roof["peak_source"] = peaks_src
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
