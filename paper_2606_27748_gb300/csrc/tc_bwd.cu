@@ -13,9 +13,10 @@
 // Every term splits over feature groups (64 frequencies = 128 features), and A enters dv
 // linearly, so one CTA handles one (sequence, group) pair and the group results are summed:
 // dq, dk, dv by fp32 adds onto zeroed accumulators (at most two groups, so the sum does not
-// depend on the order), dW through per-(sequence, group) partials reduced over the batch in
-// a fixed order.  Two launches: pass F runs the chunks forward (dq and the q part of dW,
-// state S, z), pass R runs them backward (dk, dv and the k part of dW, state R, r).
+// depend on the order), dW through per-(pass, sequence, group) partials reduced over the
+// batch in a fixed order.  Pass F runs the chunks forward (dq and the q part of dW, state
+// S, z), pass R runs them backward (dk, dv and the k part of dW, state R, r); the two are
+// independent and run as the two halves of one grid.
 //
 // Phases are serialised: all 256 threads load, compute features and run the CUDA-core
 // epilogues; thread 0 issues the MMAs; one mbarrier tracks their completion (bounded waits).
@@ -58,16 +59,33 @@ __device__ __forceinline__ float bf16_at(const uint8_t* tile, int row, int col)
     return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(tile + swz128(row, col)));
 }
 
-template <int PASS, bool NS>
+__device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d)
+{
+    asm volatile("red.global.add.v4.f32 [%0], {%1,%2,%3,%4};" ::"l"(addr), "f"(a), "f"(b),
+                 "f"(c), "f"(d)
+                 : "memory");
+}
+
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+template <bool NS>
 __global__ void __launch_bounds__(kThreadsB, 1)
     tc_bwd_kernel(int H, int N, int M, int G, int causal, const __nv_bfloat16* __restrict__ q,
                   const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __restrict__ v,
                   const float* __restrict__ W1, const float* __restrict__ W2,
                   const __nv_bfloat16* __restrict__ outp, const float* __restrict__ den,
-                  const __nv_bfloat16* __restrict__ dout, float* __restrict__ acc_x,
-                  float* __restrict__ acc_v, float* __restrict__ dw_part, int* status)
+                  const __nv_bfloat16* __restrict__ dout, float* __restrict__ acc_q,
+                  float* __restrict__ acc_k, float* __restrict__ acc_v, float* __restrict__ dw_part,
+                  int units, int* status)
 {
     using L = BwCfg<NS>;
+    // blocks [0, units): pass F, [units, 2 units): pass R; unit = (sequence, group)
+    const int PASS = (int)blockIdx.x >= units ? kPassR : kPassF;
+    const int unit = (int)blockIdx.x % units;
+    float* const acc_x = PASS == kPassF ? acc_q : acc_k;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const uint32_t sb = smem_u32(sm);
@@ -77,7 +95,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int wg = warp >> 2, quad = warp & 3, t = 32 * quad + lane;
-    const int bh = blockIdx.x / G, g = blockIdx.x % G, h = bh % H;
+    const int bh = unit / G, g = unit % G, h = bh % H;
     const size_t base = (size_t)bh * N * 64;
     float* zr = reinterpret_cast<float*>(sm + L::ZR);
     float* crow = reinterpret_cast<float*>(sm + L::CROW);
@@ -268,6 +286,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         tmem_wait_ld();
         if (t < L::P && wg == 1) {
             float4* dst = reinterpret_cast<float4*>(dw_part + ((size_t)blockIdx.x * 128 + t) * 64);
+            // slot blockIdx.x = pass * units + unit
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
                 float4 old = first ? make_float4(0.f, 0.f, 0.f, 0.f) : dst[j];
@@ -299,7 +318,8 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         if (valid) {
             float* dst = acc + base + (size_t)(t0 + t) * 64 + 32 * wg;
 #pragma unroll
-            for (int j = 0; j < 32; ++j) atomicAdd(dst + j, v_[j]);
+            for (int j = 0; j < 8; ++j)
+                red_add_v4(dst + 4 * j, v_[4 * j], v_[4 * j + 1], v_[4 * j + 2], v_[4 * j + 3]);
         }
     };
 
@@ -309,6 +329,18 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         const int c = PASS == kPassF ? it : nch - 1 - it;
         const int t0 = c * kC, CL = min(kC, N - t0);
         const bool valid = t < CL;
+        if (tid == 0) {  // the next chunk's tiles into L2 while this one is worked on
+            const int cn = PASS == kPassF ? c + 1 : c - 1;
+            if (cn >= 0 && cn < nch) {
+                const size_t off = base + (size_t)cn * kC * 64;
+                const uint32_t bytes = (uint32_t)min(kC, N - cn * kC) * 128;
+                prefetch_l2(q + off, bytes);
+                prefetch_l2(k + off, bytes);
+                prefetch_l2(v + off, bytes);
+                prefetch_l2(dout + off, bytes);
+                prefetch_l2(outp + off, bytes);
+            }
+        }
         // ---- loads: q, k, v tiles; g tile and c_t from dout, out, den ----
         for (int i = tid; i < 3 * 1024; i += kThreadsB) {
             const int tile = i >> 10, idx = i & 1023, r = idx >> 3, cc = idx & 7;
@@ -504,7 +536,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             handoff();
             if (!project_back(dPK, dPKmn, dKmn)) goto done;
             add_rows(acc_x, t0, valid);
-            dw_accumulate(false);
+            dw_accumulate(it == 0);
             snapshot();
             handoff();
         }
@@ -516,8 +548,9 @@ done:
     if (warp == 0) tmem_dealloc(tm, 512);
 }
 
-// dW over the batch in a fixed order.  Partial slots [bh * G + g][row][64]; s: rows < 64
-// are frequencies 64g + row; n: rows < 64 are dU, rows >= 64 are dV of frequency 64g + row%64.
+// dW over the batch in a fixed order.  Partial slots [pass][bh * G + g][row][64]; s: rows
+// < 64 are frequencies 64g + row; n: rows < 64 are dU, rows >= 64 are dV of frequency
+// 64g + row%64.
 __global__ void tc_dw_reduce_kernel(int B, int H, int M, int G, int nonstat,
                                     const float* __restrict__ part, float* __restrict__ dW1,
                                     float* __restrict__ dW2)
@@ -529,10 +562,11 @@ __global__ void tc_dw_reduce_kernel(int B, int H, int M, int G, int nonstat,
         const int f = (int)((idx / 64) % M), e = (int)(idx % 64);
         const int g = f / 64, r = f % 64;
         float a = 0.f, b2 = 0.f;
+        const size_t pass_stride = (size_t)B * H * G * 128 * 64;  // pass R slots follow pass F's
         for (int b = 0; b < B; ++b) {
             const float* p = part + ((size_t)((b * H + h) * G + g) * 128) * 64;
-            a += p[(size_t)r * 64 + e];
-            if (nonstat) b2 += p[(size_t)(64 + r) * 64 + e];
+            a += p[(size_t)r * 64 + e] + p[pass_stride + (size_t)r * 64 + e];
+            if (nonstat) b2 += p[(size_t)(64 + r) * 64 + e] + p[pass_stride + (size_t)(64 + r) * 64 + e];
         }
         if (!nonstat) {
             dW1[idx] = a;
@@ -570,16 +604,13 @@ cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const voi
     cudaError_t e = cudaMemsetAsync(acc_q, 0, 3 * n * sizeof(float), s);
     if (e != cudaSuccess) return e;
     const int smem = (int)BwCfg<NS>::BYTES + 1024;
-    auto kf = tc_bwd_kernel<kPassF, NS>;
-    auto kr = tc_bwd_kernel<kPassR, NS>;
-    if ((e = cudaFuncSetAttribute(kf, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return e;
-    if ((e = cudaFuncSetAttribute(kr, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return e;
+    auto kb = tc_bwd_kernel<NS>;
+    if ((e = cudaFuncSetAttribute(kb, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return e;
     typedef const __nv_bfloat16* CB;
-    kf<<<BH * G, kThreadsB, smem, s>>>(p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k, (CB)v, W1, W2,
-                                       (CB)out, den, (CB)dout, acc_q, acc_v, part, status);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    kr<<<BH * G, kThreadsB, smem, s>>>(p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k, (CB)v, W1, W2,
-                                       (CB)out, den, (CB)dout, acc_k, acc_v, part, status);
+    const int units = BH * G;
+    kb<<<2 * units, kThreadsB, smem, s>>>(p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k, (CB)v, W1,
+                                          W2, (CB)out, den, (CB)dout, acc_q, acc_k, acc_v, part,
+                                          units, status);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const size_t work = (size_t)p.H * p.M * 64;
     tc_dw_reduce_kernel<<<(int)std::min<size_t>((work + 255) / 256, 152 * 8), 256, 0, s>>>(
@@ -602,7 +633,7 @@ bool tc_bwd_supported(const Problem& p)
 size_t tc_bwd_ws_bytes(const Problem& p)
 {
     const size_t BH = (size_t)p.B * p.H, G = (size_t)p.M / 64;
-    return (3 * BH * p.N * 64 + BH * G * 128 * 64) * sizeof(float);
+    return (3 * BH * p.N * 64 + 2 * BH * G * 128 * 64) * sizeof(float);
 }
 
 cudaError_t launch_tc_bwd(const Problem& p, const void* q, const void* k, const void* v,
