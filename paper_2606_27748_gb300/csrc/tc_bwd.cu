@@ -54,10 +54,6 @@ struct BwCfg {
     static_assert(BYTES + 1024 <= 232448, "shared memory budget");
 };
 
-__device__ __forceinline__ float bf16_at(const uint8_t* tile, int row, int col)
-{
-    return __bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(tile + swz128(row, col)));
-}
 
 __device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d)
 {
@@ -73,7 +69,10 @@ __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes)
 
 template <bool NS>
 __global__ void __launch_bounds__(kThreadsB, 1)
-    tc_bwd_kernel(int H, int N, int M, int G, int causal, const __nv_bfloat16* __restrict__ q,
+    tc_bwd_kernel(const __grid_constant__ CUtensorMap tmap_q,
+                  const __grid_constant__ CUtensorMap tmap_k,
+                  const __grid_constant__ CUtensorMap tmap_v, int H, int N, int M, int G, int causal,
+                  const __nv_bfloat16* __restrict__ q,
                   const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __restrict__ v,
                   const float* __restrict__ W1, const float* __restrict__ W2,
                   const __nv_bfloat16* __restrict__ outp, const float* __restrict__ den,
@@ -90,7 +89,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const uint32_t sb = smem_u32(sm);
     __shared__ uint32_t tmem_base_sh;
-    __shared__ __align__(8) uint64_t mbar;
+    __shared__ __align__(8) uint64_t mbar, tma_bar;
     __shared__ volatile int abort_flag;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -125,6 +124,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     for (int idx = tid; idx < 128; idx += kThreadsB) zr[idx] = 0.f;
     if (tid == 0) {
         mbar_init(&mbar, 1);
+        mbar_init(&tma_bar, 1);
         abort_flag = 0;
         fence_mbar_init();
     }
@@ -138,7 +138,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     fence_after_sync();
     const uint32_t tm = tmem_base_sh;
     const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
-    uint32_t phase = 0;
+    uint32_t phase = 0, tma_phase = 0;
 
     auto handoff = [&]() {
         fence_proxy_async();
@@ -230,17 +230,36 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             tmem_ld16(tm_row + L::T_P + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
         }
         tmem_wait_ld();
-        const uint8_t* tp = sm + (tile - sb);
+        uint32_t cpair[16], spair[16];  // s: this thread's cos / sin features, bf16 pairs
+        if (!NS) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint4 c4 = *reinterpret_cast<const uint4*>(sm + (tile - sb) + swz128(t, (4 * wg + j) * 8));
+                const uint4 s4 =
+                    *reinterpret_cast<const uint4*>(sm + (tile - sb) + 16384 + swz128(t, (4 * wg + j) * 8));
+                cpair[4 * j] = c4.x; cpair[4 * j + 1] = c4.y; cpair[4 * j + 2] = c4.z; cpair[4 * j + 3] = c4.w;
+                spair[4 * j] = s4.x; spair[4 * j + 1] = s4.y; spair[4 * j + 2] = s4.z; spair[4 * j + 3] = s4.w;
+            }
+        }
+        float zc[32], zs[32];  // the per-feature term, z (pass F) or r (pass R)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const float4 a4 = reinterpret_cast<const float4*>(zr + 32 * wg)[j];
+            const float4 b4 = reinterpret_cast<const float4*>(zr + 64 + 32 * wg)[j];
+            zc[4 * j] = a4.x; zc[4 * j + 1] = a4.y; zc[4 * j + 2] = a4.z; zc[4 * j + 3] = a4.w;
+            zs[4 * j] = b4.x; zs[4 * j + 1] = b4.y; zs[4 * j + 2] = b4.z; zs[4 * j + 3] = b4.w;
+        }
         uint32_t o1[16], o2[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
             float r1[2], r2[2];
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
-                const int fi = 2 * i + e, f = 32 * wg + fi;
-                const float dphic = dc[fi] + scale * zr[f], dphis = ds[fi] + scale * zr[64 + f];
+                const int fi = 2 * i + e;
+                const float dphic = dc[fi] + scale * zc[fi], dphis = ds[fi] + scale * zs[fi];
                 if (!NS) {
-                    const float pc = bf16_at(tp, t, f), psn = bf16_at(tp + 16384, t, f);
+                    const float pc = __uint_as_float(e ? cpair[i] & 0xFFFF0000u : cpair[i] << 16);
+                    const float psn = __uint_as_float(e ? spair[i] & 0xFFFF0000u : spair[i] << 16);
                     r1[e] = -psn * dphic + pc * dphis;
                     r2[e] = 0.f;
                 } else {
@@ -262,8 +281,10 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             st_shared_v4(tile + 16384 + off, o2[4 * j], o2[4 * j + 1], o2[4 * j + 2], o2[4 * j + 3]);
         }
     };
-    // dx = da W (T_A[0,64)) and this chunk's dW = da^T x (T_A[64,128))
-    auto project_back = [&](uint64_t d_da, uint64_t d_da_mn, uint64_t d_x_mn) {
+    // dx = da W (T_A[0,64)) and dW = da^T x: n: this chunk's in T_A[64,128); s: summed
+    // over the chunks in the projection's unused half, T_P[64,128)
+    constexpr uint32_t T_DW = NS ? L::T_A + 64 : L::T_P + 64;
+    auto project_back = [&](uint64_t d_da, uint64_t d_da_mn, uint64_t d_x_mn, bool first) {
         if (tid == 0) {
             fence_after_sync();
             const int kst = NS ? 8 : 4;  // K = P rows of W (s: the cos half only)
@@ -272,8 +293,8 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                          adv(dWmn, ks * 2048), I_KM64, ks > 0);
 #pragma unroll
             for (int ks = 0; ks < 8; ++ks)
-                mma_bf16(tm + L::T_A + 64, adv(d_da_mn, ks * 2048), adv(d_x_mn, ks * 2048), I_MM64,
-                         ks > 0);
+                mma_bf16(tm + T_DW, adv(d_da_mn, ks * 2048), adv(d_x_mn, ks * 2048), I_MM64,
+                         (NS ? ks > 0 : (!first || ks > 0)) ? 1u : 0u);
         }
         return commit_wait();
     };
@@ -282,7 +303,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         float v_[64];
 #pragma unroll
         for (int j = 0; j < 4; ++j)
-            tmem_ld16(tm_row + L::T_A + 64 + 16 * j, *reinterpret_cast<float(*)[16]>(&v_[16 * j]));
+            tmem_ld16(tm_row + T_DW + 16 * j, *reinterpret_cast<float(*)[16]>(&v_[16 * j]));
         tmem_wait_ld();
         if (t < L::P && wg == 1) {
             float4* dst = reinterpret_cast<float4*>(dw_part + ((size_t)blockIdx.x * 128 + t) * 64);
@@ -341,14 +362,13 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 prefetch_l2(outp + off, bytes);
             }
         }
-        // ---- loads: q, k, v tiles; g tile and c_t from dout, out, den ----
-        for (int i = tid; i < 3 * 1024; i += kThreadsB) {
-            const int tile = i >> 10, idx = i & 1023, r = idx >> 3, cc = idx & 7;
-            const __nv_bfloat16* src = tile == 0 ? q : (tile == 1 ? k : v);
-            uint4 val = make_uint4(0, 0, 0, 0);
-            if (r < CL) val = __ldg(reinterpret_cast<const uint4*>(src + base + (size_t)(t0 + r) * 64 + cc * 8));
-            const uint32_t dst = tile == 0 ? L::Q : (tile == 1 ? L::K : L::V);
-            st_shared_v4(sb + dst + swz128(r, cc * 8), val.x, val.y, val.z, val.w);
+        // ---- loads: q, k, v tiles (TMA; rows past N read as zero); g tile and c_t from
+        // dout, out, den ----
+        if (tid == 0) {
+            mbar_arrive_expect_tx(&tma_bar, 3 * kTileBytes);
+            tma_load_3d(sb + L::Q, &tmap_q, 0, t0, bh, &tma_bar);
+            tma_load_3d(sb + L::K, &tmap_k, 0, t0, bh, &tma_bar);
+            tma_load_3d(sb + L::V, &tmap_v, 0, t0, bh, &tma_bar);
         }
         if (wg == 0) {
             float gsc = 0.f, cval = 0.f;
@@ -388,6 +408,8 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 *reinterpret_cast<__nv_bfloat16*>(sm + L::C16 + (t >> 6) * 2048 + swz128(0, t & 63)) =
                     __float2bfloat16_rn(cval);
         }
+        if (!bar_wait(&tma_bar, tma_phase, &abort_flag, status)) goto done;
+        tma_phase ^= 1;
         handoff();
         // ---- features of q and k for this group ----
         if (!project(dQ)) goto done;
@@ -450,9 +472,9 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             if (NS && !project(dQ)) goto done;  // u, w of q for the chain rule
             feature_backward(sb + L::PQ, crow[t], valid);
             handoff();
-            if (!project_back(dPQ, dPQmn, dQmn)) goto done;
+            if (!project_back(dPQ, dPQmn, dQmn, it == 0)) goto done;
             add_rows(acc_x, t0, valid);
-            dw_accumulate(it == 0);
+            if (NS) dw_accumulate(it == 0);
             snapshot();
             handoff();
         } else {
@@ -534,13 +556,14 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             if (NS && !project(dK)) goto done;  // u, w of k for the chain rule
             feature_backward(sb + L::PK, 1.0f, valid);
             handoff();
-            if (!project_back(dPK, dPKmn, dKmn)) goto done;
+            if (!project_back(dPK, dPKmn, dKmn, it == 0)) goto done;
             add_rows(acc_x, t0, valid);
-            dw_accumulate(it == 0);
+            if (NS) dw_accumulate(it == 0);
             snapshot();
             handoff();
         }
     }
+    if (!NS) dw_accumulate(true);  // s: the sum over all chunks, from T_P[64,128)
 done:
     fence_before_sync();
     __syncthreads();
@@ -604,11 +627,16 @@ cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const voi
     cudaError_t e = cudaMemsetAsync(acc_q, 0, 3 * n * sizeof(float), s);
     if (e != cudaSuccess) return e;
     const int smem = (int)BwCfg<NS>::BYTES + 1024;
+    CUtensorMap mq, mk, mv;
+    if (!make_act_map(&mq, q, BH, p.N) || !make_act_map(&mk, k, BH, p.N) ||
+        !make_act_map(&mv, v, BH, p.N))
+        return cudaErrorInvalidValue;
     auto kb = tc_bwd_kernel<NS>;
     if ((e = cudaFuncSetAttribute(kb, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return e;
     typedef const __nv_bfloat16* CB;
     const int units = BH * G;
-    kb<<<2 * units, kThreadsB, smem, s>>>(p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k, (CB)v, W1,
+    kb<<<2 * units, kThreadsB, smem, s>>>(mq, mk, mv, p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k,
+                                          (CB)v, W1,
                                           W2, (CB)out, den, (CB)dout, acc_q, acc_k, acc_v, part,
                                           units, status);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
