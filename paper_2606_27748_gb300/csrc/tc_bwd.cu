@@ -174,22 +174,34 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     constexpr uint32_t I_M16 = idesc_bf16(128, 16, 1, 0);      // MN-major A, K-major B, N=16
 
     // projection of a tile into T_P, then features of this group into dst (K-major rows)
+    auto issue_projection = [&](uint64_t dx, uint32_t col) {
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks)
+            mma_bf16(tm + col, adv(dx, ks * 32), adv(dW, ks * 32), I_PROJ, ks > 0);
+    };
     auto project = [&](uint64_t dx) {
         if (tid == 0) {
             fence_after_sync();
-#pragma unroll
-            for (int ks = 0; ks < 4; ++ks)
-                mma_bf16(tm + L::T_P, adv(dx, ks * 32), adv(dW, ks * 32), I_PROJ, ks > 0);
+            issue_projection(dx, L::T_P);
         }
         return commit_wait();
     };
-    auto features = [&](uint32_t dst, bool valid) {
+    // q into T_P and k into T_A (free until the attention MMAs), one round trip
+    auto project_qk = [&]() {
+        if (tid == 0) {
+            fence_after_sync();
+            issue_projection(dQ, L::T_P);
+            issue_projection(dK, L::T_A);
+        }
+        return commit_wait();
+    };
+    auto features = [&](uint32_t dst, uint32_t tcol, bool valid) {
         float a[32], w[32];
-        tmem_ld16(tm_row + L::T_P + 32 * wg, *reinterpret_cast<float(*)[16]>(&a[0]));
-        tmem_ld16(tm_row + L::T_P + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+        tmem_ld16(tm_row + tcol + 32 * wg, *reinterpret_cast<float(*)[16]>(&a[0]));
+        tmem_ld16(tm_row + tcol + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
         if (NS) {
-            tmem_ld16(tm_row + L::T_P + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]));
-            tmem_ld16(tm_row + L::T_P + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
+            tmem_ld16(tm_row + tcol + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]));
+            tmem_ld16(tm_row + tcol + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
         }
         tmem_wait_ld();
         uint32_t pc[16], ps[16];
@@ -412,11 +424,9 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         tma_phase ^= 1;
         handoff();
         // ---- features of q and k for this group ----
-        if (!project(dQ)) goto done;
-        features(sb + L::PQ, valid);
-        handoff();
-        if (!project(dK)) goto done;
-        features(sb + L::PK, valid);
+        if (!project_qk()) goto done;
+        features(sb + L::PQ, L::T_P, valid);
+        features(sb + L::PK, L::T_A, valid);
         handoff();
 
         if (PASS == kPassF) {
@@ -469,7 +479,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 }
             }
             if (!commit_wait()) goto done;
-            if (NS && !project(dQ)) goto done;  // u, w of q for the chain rule
+            // n: u, w of q for the chain rule are still in T_P
             feature_backward(sb + L::PQ, crow[t], valid);
             handoff();
             if (!project_back(dPQ, dPQmn, dQmn, it == 0)) goto done;

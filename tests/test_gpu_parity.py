@@ -162,3 +162,27 @@ def test_forward_sequence_splits(w, N):
     ro, rd = _oracle_fwd(ins, True)
     assert_close(to_host(out), ro, w.dtype, f"out N={N}")
     assert_close(to_host(den), rd, w.dtype, "den", max_abs_scale=float(np.abs(rd).max()))
+
+
+@pytest.mark.parametrize("w", [WL[1], WL[2]], ids=["stationary", "nonstationary"])
+def test_dispatch_launch_counts_and_determinism(w):
+    """The tensor-core entry points run (launch counts per call: causal forward 1, non-causal
+    forward 3, causal backward 3), and the backward is bit-for-bit repeatable (dq, dk, dv
+    are sums of at most two groups, dW is reduced in a fixed order)."""
+    ws_ = w.replace(B=2, H=2, N=700, backward=True)
+    ins = workloads.make_inputs(ws_)
+    n0 = flexattn.kernel_launches()
+    _gpu_fwd(ws_, ins, True)
+    assert flexattn.kernel_launches() - n0 == 1
+    n0 = flexattn.kernel_launches()
+    _gpu_fwd(ws_, ins, False)
+    assert flexattn.kernel_launches() - n0 == 3
+    n0 = flexattn.kernel_launches()
+    g1 = _gpu_bwd(ws_, ins, True)
+    assert flexattn.kernel_launches() - n0 == 1 + 3  # the forward it runs first + backward
+    g2 = _gpu_bwd(ws_, ins, True)
+    for a, b in zip(g1, g2):
+        if a is None:
+            assert b is None
+        else:
+            assert np.array_equal(a, b)
