@@ -326,7 +326,8 @@ def run_ours(args, w):
     stream = torch.cuda.current_stream()
 
     if w.backward:  # a training step: forward, then backward of sum(dO * out)
-        dO = torch.from_numpy(workloads.draw_activation(w, workloads.DO)).to(tdt).to(dev)
+        host["dO"] = torch.from_numpy(workloads.draw_activation(w, workloads.DO)).to(tdt).pin_memory()
+        dO = host["dO"].to(dev)
         grads = [torch.empty_like(q), torch.empty_like(k), torch.empty_like(v),
                  torch.empty_like(W1), None if W2 is None else torch.empty_like(W2)]
         ws_b = flexattn.workspace(shape, w.causal, True, dev)
@@ -372,13 +373,17 @@ def run_ours(args, w):
     # memory, the forward, D2H of out, every step.
     e2e = None
     if not args.no_e2e:
-        host_out = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+        # inference: the output comes back; training: the frequency gradient (dq, dk, dv
+        # feed the layers below on the device)
+        result = grads[3] if w.backward else out
+        host_out = torch.empty(result.shape, dtype=result.dtype).pin_memory()
+        inputs = (("q", q), ("k", k), ("v", v)) + ((("dO", dO),) if w.backward else ())
 
         def e2e_step():
-            for n, t in (("q", q), ("k", k), ("v", v)):
+            for n, t in inputs:
                 t.copy_(host[n], non_blocking=True)
             step()
-            host_out.copy_(out, non_blocking=True)
+            host_out.copy_(result, non_blocking=True)
 
         for _ in range(max(3, args.warmup)):
             e2e_step()
@@ -393,7 +398,7 @@ def run_ours(args, w):
         barrier()
         e2e_ms = a.elapsed_time(b) / K
         e2e_ms = max_over_ranks([e2e_ms], world, dev)[0]
-        h2d = sum(host[n].numel() * host[n].element_size() for n in "qkv")
+        h2d = sum(host[n].numel() * host[n].element_size() for n, _ in inputs)
         e2e = {"value": job_value(world, w.tokens, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": host_out.numel() * host_out.element_size()}

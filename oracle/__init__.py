@@ -68,8 +68,9 @@ class Oracle:
         lib.oracle_linattn_fwd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, i, dp, dp, i]
         lib.oracle_linattn_bwd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, i, dp, dp, dp,
                                            dp, dp, dp, i]
+        lib.oracle_linattn_decode.argtypes = [i, i, i, i, dp, dp, dp, dp, dp, dp, dp, dp, dp]
         for fn in (lib.oracle_featmap, lib.oracle_featmap_sumform, lib.oracle_linattn_fwd,
-                   lib.oracle_linattn_bwd):
+                   lib.oracle_linattn_bwd, lib.oracle_linattn_decode):
             fn.restype = ctypes.c_int
         self._lib = lib
         self.path = path
@@ -140,6 +141,24 @@ class Oracle:
             raise ValueError("oracle_linattn_bwd: bad shape")
         return dq, dk, dv, dW1, dW2
 
+    def decode(self, q, k, v, W1, W2, S, z):
+        """One causal decode step (Eq. linear att as running sums, inclusive of the new
+        token): q, k, v [B, H, d]; state S [B, H, 2M, d], z [B, H, 2M] (not modified).
+        Returns (out [B, H, d], den [B, H], S', z')."""
+        q, k, v, W1, W2 = (self._f64(a) for a in (q, k, v, W1, W2))
+        S = np.array(S, dtype=np.float64, copy=True, order="C")
+        z = np.array(z, dtype=np.float64, copy=True, order="C")
+        B, H, d = q.shape
+        M = W1.shape[1]
+        out = np.empty_like(q)
+        den = np.empty((B, H))
+        rc = self._lib.oracle_linattn_decode(B, H, d, M, self._p(q), self._p(k), self._p(v),
+                                             self._p(W1), self._p(W2), self._p(S), self._p(z),
+                                             self._p(out), self._p(den))
+        if rc != 0:
+            raise ValueError("oracle_linattn_decode: bad shape")
+        return out, den, S, z
+
 
 def load() -> Oracle:
     """The oracle built from ``flex_oracle.c`` (compiled on first use if needed)."""
@@ -162,3 +181,7 @@ def fwd(q, k, v, W1, W2=None, causal=True, nthreads=None):
 
 def bwd(q, k, v, W1, W2, causal, dout, nthreads=None):
     return load().bwd(q, k, v, W1, W2, causal, dout, nthreads)
+
+
+def decode(q, k, v, W1, W2, S, z):
+    return load().decode(q, k, v, W1, W2, S, z)

@@ -407,3 +407,42 @@ int oracle_linattn_bwd(int B, int H, int N, int d, int M, const double* q, const
     free(dA); free(dB); free(jobs);
     return 0;
 }
+
+/* One step of the causal recurrence behind Eq. (linear att) with j <= i: the running sums
+ * S = sum_j phi(k_j) v_j^T and z = sum_j phi(k_j) absorb the new token (inclusive), then
+ * out = phi(q)^T S / den with den = phi(q)^T z.  Per (b, h): q, k, v, out [d]; S [2M][d]
+ * and z [2M] are updated in place; den [1]. */
+int oracle_linattn_decode(int B, int H, int d, int M, const double* q, const double* k,
+                          const double* v, const double* W1, const double* W2, double* S,
+                          double* z, double* out, double* den)
+{
+    if (bad_shape(B, H, 1, d, M)) return -1;
+    const int F = 2 * M;
+    double* pq = malloc((size_t)F * sizeof(double));
+    double* pk = malloc((size_t)F * sizeof(double));
+    for (int b = 0; b < B; ++b)
+        for (int h = 0; h < H; ++h) {
+            const size_t u = (size_t)b * H + h;
+            const double* w1 = W1 + (size_t)h * M * d;
+            const double* w2 = W2 ? W2 + (size_t)h * M * d : NULL;
+            feature(d, M, q + u * d, w1, w2, pq);
+            feature(d, M, k + u * d, w1, w2, pk);
+            double* Su = S + u * F * d;
+            double* zu = z + u * F;
+            for (int f = 0; f < F; ++f) {
+                for (int e = 0; e < d; ++e) Su[(size_t)f * d + e] += pk[f] * v[u * d + e];
+                zu[f] += pk[f];
+            }
+            double dn = 0.0;
+            for (int f = 0; f < F; ++f) dn += pq[f] * zu[f];
+            for (int e = 0; e < d; ++e) {
+                double num = 0.0;
+                for (int f = 0; f < F; ++f) num += pq[f] * Su[(size_t)f * d + e];
+                out[u * d + e] = num / dn;
+            }
+            den[u] = dn;
+        }
+    free(pq);
+    free(pk);
+    return 0;
+}

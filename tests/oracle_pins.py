@@ -15,7 +15,8 @@ Facts used (none is the oracle's own formula retyped):
   * Yaglom (Thm. yaglom) with independent Gaussian W1, W2:
       E = 1/2 exp(-|x-y|^2 / 2 s^2) + 1/2 exp(-(|x|^2 + |y|^2) / 2 s^2).
   * Eq. (linear att) is an exact reassociation of Eq. (attention): the C linear form
-    equals the numpy N x N form (different module, different feature form).
+    equals the numpy N x N form (different module, different feature form); so does the
+    C decode recurrence run token by token, and its state equals the numpy running sums.
   * d = 1, M = 1: phi_s(q).phi_s(k) = cos(w (q - k)) in closed form.
   * causal output at the last position equals the non-causal output.
   * causal O_0 = v_0; constant v = c gives O = c (rows of weights sum to one).
@@ -119,6 +120,25 @@ def pin_linear_equals_brute(orc):
                 assert _rel(out, bo) < 1e-11, f"out {variant} causal={causal} N={N}"
 
 
+def pin_decode_equals_brute(orc):
+    """Token-by-token decode from the zero state reproduces every row of the causal N x N
+    form, and the state it carries is sum_j phi(k_j) v_j^T, sum_j phi(k_j) with the numpy
+    features (sum form for n)."""
+    for variant in ("s", "n"):
+        B, H, N, d, M = 2, 2, 9, 5, 7
+        q, k, v, W1, W2 = _case(40, B, H, N, d, M, variant)
+        bo, bd = brute.attention(q, k, v, W1, W2, True)
+        S = np.zeros((B, H, 2 * M, d))
+        z = np.zeros((B, H, 2 * M))
+        for i in range(N):
+            out, den, S, z = orc.decode(q[:, :, i], k[:, :, i], v[:, :, i], W1, W2, S, z)
+            assert _rel(den, bd[:, :, i]) < 1e-12, f"decode den {variant} i={i}"
+            assert _rel(out, bo[:, :, i]) < 1e-11, f"decode out {variant} i={i}"
+        pk = brute.features(k, W1, W2)
+        assert _rel(S, np.einsum("bhnf,bhne->bhfe", pk, v)) < 1e-12, f"decode S {variant}"
+        assert _rel(z, pk.sum(axis=2)) < 1e-12, f"decode z {variant}"
+
+
 def pin_closed_form_d1(orc):
     q = np.array([0.3, -1.1, 0.7]).reshape(1, 1, 3, 1)
     k = np.array([0.1, 0.5, -0.4]).reshape(1, 1, 3, 1)
@@ -197,7 +217,8 @@ def pin_gradient_invariants(orc):
 
 ALL_PINS = [
     pin_origin_features, pin_stationary_unit_norm, pin_sum_to_product, pin_w2_equals_w1,
-    pin_bochner, pin_yaglom, pin_linear_equals_brute, pin_closed_form_d1,
+    pin_bochner, pin_yaglom, pin_linear_equals_brute, pin_decode_equals_brute,
+    pin_closed_form_d1,
     pin_causal_last_equals_noncausal, pin_first_and_constant, pin_finite_differences,
     pin_gradient_invariants,
 ]

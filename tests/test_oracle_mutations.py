@@ -39,6 +39,9 @@ MUTATIONS = [
     ("reverse_scan_exclusive",
      "for (int j = N - 1; j >= 0; --j) {\n        if (J->causal)",
      "for (int j = N - 1; j >= 0; --j) {\n        if (J->causal && 0)", 0),
+    ("decode_drops_new_value", "Su[(size_t)f * d + e] += pk[f] * v[u * d + e];",
+     "Su[(size_t)f * d + e] += 0.0 * v[u * d + e];", 0),
+    ("decode_forgets_z_update", "zu[f] += pk[f];", "zu[f] += 0.0;", 0),
 ]
 
 
