@@ -33,6 +33,8 @@ from paper_2606_27748_gb300 import workloads  # noqa: E402
 
 METRIC = "RFF linear-attn fwd tokens/s (N=16K causal) & % of bf16 tensor/HBM roofline"
 METRIC_TRAIN = "RFF linear-attn fwd+bwd training-step tokens/s & % of roofline"
+METRIC_DECODE = ("RFF linear-attn recurrent decode tokens/s (one new token per sequence, fp32 "
+                 "running state) & % of HBM roofline")
 L2_BYTES = 129e6
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
@@ -243,6 +245,23 @@ def run_reference(args, w):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
+    if w.decode:
+        for _ in range(args.warmup):
+            oracle_decode_sample(w, 1)
+        step = sum(oracle_decode_sample(w, 1) for _ in range(args.steps)) / args.steps
+        value = w.B / step
+        print(json.dumps({
+            "metric": METRIC_DECODE, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "d": w.d, "M": w.M,
+                       "variant": w.variant, "causal": True},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                             "sample": f"one decode step of all {w.B}x{w.H} sequences per step"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}), flush=True)
+        return
     cores = cpu_cores()
     nseq = min(w.B * w.H, cores)
     for _ in range(args.warmup):
@@ -432,11 +451,178 @@ def run_ours(args, w):
         dist.destroy_process_group()
 
 
+# ---------------------------------------------------------------------------------------
+# Recurrent decode workload: a step gives every sequence one new token (its q, k, v), which
+# updates the fp32 running state (S, z) and yields its output.
+# ---------------------------------------------------------------------------------------
+def decode_work(w):
+    """(bytes, flops, sin/cos) per decode step: the state read and written once, the new
+    tokens' q, k, v read and out written, the frequencies read once."""
+    F, bh = 2 * w.M, w.B * w.H
+    mc = 2 * w.M if w.variant == "n" else w.M
+    nbytes = (bh * (F * w.d + F) * 4 * 2 + bh * 4 * w.d * elem_bytes(w)
+              + w.H * w.M * w.d * 4 * (2 if w.variant == "n" else 1))
+    flops = bh * (2 * (2 * w.d * mc) + 3 * (2 * F * w.d))
+    ops = bh * 2 * (3 if w.variant == "n" else 2) * w.M
+    return nbytes, flops, ops
+
+
+def oracle_decode_sample(w, steps):
+    """Seconds per oracle decode step of all B x H sequences (the first token)."""
+    import numpy as np
+    import oracle
+    ins = workloads.make_inputs(w, N=1)
+    q, k, v = (ins[n][:, :, 0] for n in "qkv")
+    W1, W2 = ins["W1"], ins["W2"]
+    S = np.zeros((w.B, w.H, 2 * w.M, w.d))
+    z = np.zeros((w.B, w.H, 2 * w.M))
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        _, _, S, z = oracle.decode(q, k, v, W1, W2, S, z)
+    return (time.perf_counter() - t0) / steps
+
+
+def run_decode(args, w):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2606_27748_gb300 import build, flexattn
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if rank == 0 or not os.path.exists(flexattn.LIBRARY):
+        build.build()
+    if world > 1:
+        dist.barrier()
+    flexattn.load()
+    tdt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    ins = workloads.make_inputs(w)
+    toks = [[torch.from_numpy(np.ascontiguousarray(ins[n][:, :, i])).to(tdt).to(dev)
+             for n in "qkv"] for i in range(w.N)]
+    host = [[t.cpu().pin_memory() for t in tk] for tk in toks]
+    W1 = torch.from_numpy(ins["W1"]).to(dev)
+    W2 = None if ins["W2"] is None else torch.from_numpy(ins["W2"]).to(dev)
+    del ins
+    S, z = flexattn.decode_state(w.B, w.H, w.M, w.d, dev)
+    ws = flexattn.decode_workspace(w.B, w.H, w.M, w.d, dev)
+    out = torch.empty_like(toks[0][0])
+    den = torch.empty(w.B, w.H, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    it = [0]
+
+    def step(tk=None):
+        q, k, v = tk if tk is not None else toks[it[0] % w.N]
+        it[0] += 1
+        flexattn.linattn_decode(q, k, v, W1, W2, S, z, out=out, den=den, ws=ws)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
+    clocks = Clocks(torch.cuda.current_device()) if rank == 0 else None
+    if clocks:
+        clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    launches0 = flexattn.kernel_launches()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(K):
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = flexattn.kernel_launches() - launches0
+    clk = clocks.stop() if clocks else None
+    total_ms = t_start.elapsed_time(t_end)
+    kernel_ms = sum(a.elapsed_time(b) for a, b in ev) / K
+    total_ms, kernel_ms = max_over_ranks([total_ms, kernel_ms], world, dev)
+    ms_per_step = total_ms / K
+    value = job_value(world, w.B, ms_per_step)
+
+    e2e = None
+    if not args.no_e2e:  # the new tokens from pinned host memory, the outputs back
+        host_out = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+        dev_tok = [torch.empty_like(t) for t in toks[0]]
+
+        def e2e_step():
+            for t, hsrc in zip(dev_tok, host[it[0] % w.N]):
+                t.copy_(hsrc, non_blocking=True)
+            step(dev_tok)
+            host_out.copy_(out, non_blocking=True)
+
+        for _ in range(max(3, args.warmup)):
+            e2e_step()
+        barrier()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(K):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e2e_ms = max_over_ranks([a.elapsed_time(b) / K], world, dev)[0]
+        e2e = {"value": job_value(world, w.B, e2e_ms), "unit": "tokens/s",
+               "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in host[0]),
+               "d2h_bytes_per_step": host_out.numel() * host_out.element_size()}
+
+    peaks, peaks_src = load_peaks()
+    nbytes, flops, ops = decode_work(w)
+    sec = kernel_ms * 1e-3
+    roof = {"bound": "hbm", "achieved": nbytes / sec / 1e9, "peak": peaks["hbm_gbs"],
+            "unit": "GB/s", "frac": nbytes / sec / 1e9 / peaks["hbm_gbs"], "traffic": None,
+            "peak_source": peaks_src, "algorithmic_bytes_per_launch": nbytes,
+            "fracs": {"hbm": nbytes / sec / 1e9 / peaks["hbm_gbs"],
+                      "tensor": flops / sec / 1e12 / peaks["bf16_tflops"]},
+            "kernel_ms": kernel_ms}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        t = oracle_decode_sample(w, 3)
+        cpu = {"value": w.B / t, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": f"3 decode steps of all {w.B}x{w.H} sequences (fp64 C oracle, "
+                         f"one thread), {t:.3f} s per step"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC_DECODE, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": K, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": w.dtype, "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "d": w.d, "M": w.M,
+                       "variant": w.variant, "causal": True,
+                       "l2": f"state {w.B * w.H * 2 * w.M * (w.d + 1) * 4 / 1e6:.0f} MB > L2 "
+                             f"{L2_BYTES / 1e6:.0f} MB, no flush",
+                       "parallelism": f"replicas x{world}"},
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+            "gpu_launches": launches,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def main():
     args = parse_args()
     w = workloads.WORKLOADS[args.workload]
     if args.impl == "reference":
         run_reference(args, w)
+    elif w.decode:
+        run_decode(args, w)
     else:
         run_ours(args, w)
 

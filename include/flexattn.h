@@ -120,6 +120,26 @@ int flex_linattn_bwd_noalloc(const flex_shape* shape, const void* q, const void*
                              const void* out, const float* den, const void* dout, void* dq,
                              void* dk, void* dv, float* dW1, float* dW2, void* stream);
 
+/* Workspace bytes needed by flex_linattn_decode for this shape (shape->N must be 1); 0 if
+ * the shape is invalid. */
+size_t flex_decode_workspace_bytes(const flex_shape* shape);
+
+/* One recurrent decode step of the causal form of Eq. (linear att) (the running sums of
+ * Sec. 2.2): for each (b, h) the new token's q, k, v ([B][H][d] in shape->dtype;
+ * shape->N must be 1) update S += phi(k) v^T and z += phi(k), then
+ * out = phi(q)^T S / den with den = phi(q)^T z -- the new token included (j <= i).
+ * S: [B][H][2M][d] fp32 and z: [B][H][2M] fp32, caller-owned, read and written in place
+ * (zero-filled before a sequence's first token); phi is scaled by M^{-1/2} as in Eq. phi_n
+ * / phi_non, so S and z are exactly the paper's running sums.  out: [B][H][d] in
+ * shape->dtype; den: NULL or [B][H] fp32.  Stepping through a sequence reproduces
+ * flex_linattn_fwd(causal = 1) row by row.  ws: workspace of at least
+ * flex_decode_workspace_bytes() bytes (it holds the step's phi(q), phi(k); a serving loop
+ * allocates it once).  Two kernels per call.  Errors: FLEX_EINVAL for NULL or misaligned
+ * pointers or N != 1, FLEX_EWORKSPACE, FLEX_EUNSUPPORTED as for the other entry points. */
+int flex_linattn_decode(const flex_shape* shape, const void* q, const void* k, const void* v,
+                        const float* W1, const float* W2, float* S, float* z, void* out,
+                        float* den, void* ws, size_t ws_bytes, void* stream);
+
 /* Cumulative number of kernels this library has enqueued in this process (all entry
  * points, all devices).  Lets a caller count the launches inside a timed region. */
 unsigned long long flex_kernel_launches(void);

@@ -151,6 +151,30 @@ int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, cons
                                           dW2, scratch, s));
 }
 
+size_t flex_decode_workspace_bytes(const flex_shape* shape)
+{
+    Problem p;
+    if (make_problem(shape, nullptr, 1, &p) != FLEX_OK || p.N != 1) return 0;
+    return header_bytes() + flex::align_up(flex::decode_ws_bytes(p), 256);
+}
+
+int flex_linattn_decode(const flex_shape* shape, const void* q, const void* k, const void* v,
+                        const float* W1, const float* W2, float* S, float* z, void* out,
+                        float* den, void* ws, size_t ws_bytes, void* stream)
+{
+    Problem p;
+    int rc = make_problem(shape, W2, 1, &p);
+    if (rc) return rc;
+    if (p.N != 1) return FLEX_EINVAL;
+    if (!q || !k || !v || !W1 || !S || !z || !out) return FLEX_EINVAL;
+    for (const void* t : {q, k, v, (const void*)W1, (const void*)S, (const void*)z, (const void*)out})
+        if (!aligned(t, 16)) return FLEX_EINVAL;
+    if ((W2 && !aligned(W2, 16)) || (den && !aligned(den, 16))) return FLEX_EINVAL;
+    if ((rc = check_ws(ws, ws_bytes, header_bytes() + flex::decode_ws_bytes(p)))) return rc;
+    return count(2, flex::launch_decode(p, q, k, v, W1, W2, S, z, out, den,
+                                        (char*)ws + header_bytes(), (cudaStream_t)stream));
+}
+
 unsigned long long flex_kernel_launches(void) { return g_launches.load(); }
 
 int flex_check_status(void* ws, void* stream)

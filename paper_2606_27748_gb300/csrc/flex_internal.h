@@ -46,6 +46,12 @@ cudaError_t launch_simt_bwd(const Problem& p, const void* q, const void* k, cons
                             const float* den, const void* dout, void* dq, void* dk, void* dv,
                             float* dW1, float* dW2, void* scratch, cudaStream_t s);
 
+// ---- recurrent decode step (one token per sequence; fp32 state) ----------------------
+size_t decode_ws_bytes(const Problem& p);  // phi(q), phi(k) of the step, fp32
+cudaError_t launch_decode(const Problem& p, const void* q, const void* k, const void* v,
+                          const float* W1, const float* W2, float* S, float* z, void* out,
+                          float* den, void* scratch, cudaStream_t s);
+
 // ---- tensor-core path (bf16 storage, d = 64, M in {64, 128}) ------------------------
 bool tc_fwd_supported(const Problem& p);
 int tc_fwd_splits(const Problem& p, int sms);  // segments per sequence (1-3)

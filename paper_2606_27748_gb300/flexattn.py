@@ -21,7 +21,9 @@ FLEX_OK, FLEX_EINVAL, FLEX_EUNSUPPORTED, FLEX_EWORKSPACE, FLEX_ECUDA, FLEX_ETIME
     0, -1, -2, -3, -4, -5)
 
 EXPORTS = ("flex_strerror", "flex_workspace_bytes", "flex_featmap", "flex_linattn_fwd",
-           "flex_linattn_bwd", "flex_kernel_launches", "flex_check_status")
+           "flex_linattn_bwd", "flex_decode_workspace_bytes", "flex_linattn_decode",
+           "flex_kernel_launches",
+           "flex_check_status")
 
 
 class FlexShape(ctypes.Structure):
@@ -59,11 +61,15 @@ def load(path: str = LIBRARY) -> ctypes.CDLL:
         lib.flex_linattn_fwd.argtypes = [shp, vp, vp, vp, vp, vp, ip, vp, vp, vp, sz, vp]
         lib.flex_linattn_bwd.argtypes = [shp, vp, vp, vp, vp, vp, ip, vp, vp, vp, vp, vp, vp,
                                          vp, vp, vp, sz, vp]
+        lib.flex_decode_workspace_bytes.argtypes = [shp]
+        lib.flex_decode_workspace_bytes.restype = sz
+        lib.flex_linattn_decode.argtypes = [shp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz,
+                                            vp]
         lib.flex_check_status.argtypes = [vp, vp]
         lib.flex_kernel_launches.argtypes = []
         lib.flex_kernel_launches.restype = ctypes.c_ulonglong
         for fn in (lib.flex_featmap, lib.flex_linattn_fwd, lib.flex_linattn_bwd,
-                   lib.flex_check_status):
+                   lib.flex_linattn_decode, lib.flex_check_status):
             fn.restype = ip
         _lib = lib
         return lib
@@ -165,6 +171,40 @@ def linattn_bwd(q, k, v, W1, W2, causal, out, den, dout, dq=None, dk=None, dv=No
                                    _ptr(dW2), _ptr(ws), ws.numel(), _stream(stream)),
            "flex_linattn_bwd")
     return dq, dk, dv, dW1, dW2
+
+
+def decode_state(B, H, M, d, device=None):
+    """A zero state (S [B, H, 2M, d], z [B, H, 2M], fp32) for flex_linattn_decode."""
+    dev = device or "cuda"
+    return (torch.zeros(B, H, 2 * M, d, dtype=torch.float32, device=dev),
+            torch.zeros(B, H, 2 * M, dtype=torch.float32, device=dev))
+
+
+def decode_workspace(B, H, M, d, device=None) -> torch.Tensor:
+    """A caller-owned workspace for flex_linattn_decode (allocate once per serving loop)."""
+    n = int(load().flex_decode_workspace_bytes(ctypes.byref(FlexShape(B, H, 1, d, M, 0))))
+    if n == 0:
+        raise FlexError(FLEX_EINVAL, "flex_decode_workspace_bytes")
+    return torch.zeros(n, dtype=torch.uint8, device=device or "cuda")
+
+
+def linattn_decode(q, k, v, W1, W2, S, z, out=None, den=None, want_den=True, ws=None,
+                   stream=None):
+    """One recurrent decode step: q, k, v [B, H, d] (one new token per sequence); the fp32
+    state (S, z) is updated in place.  Returns (out [B, H, d], den [B, H] or None)."""
+    B, H, d = q.shape
+    shape = FlexShape(B, H, 1, d, W1.shape[1], _dtype_code(q))
+    if out is None:
+        out = torch.empty_like(q)
+    if den is None and want_den:
+        den = torch.empty(B, H, dtype=torch.float32, device=q.device)
+    if ws is None:
+        ws = decode_workspace(B, H, W1.shape[1], d, q.device)
+    _check(load().flex_linattn_decode(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(v),
+                                      _ptr(W1), _ptr(W2), _ptr(S), _ptr(z), _ptr(out),
+                                      _ptr(den), _ptr(ws), ws.numel(), _stream(stream)),
+           "flex_linattn_decode")
+    return out, den
 
 
 def check_status(ws, stream=None):

@@ -38,6 +38,7 @@ class Workload:
     v_dist: str           # "normal": N(0, 1); "uniform": U(-1, 1)
     seed: int
     backward: bool = False
+    decode: bool = False  # recurrent decode steps: one new token per sequence per step
 
     @property
     def tokens(self) -> int:
@@ -65,8 +66,14 @@ WORKLOADS = {
                  128, 64 ** -0.25, "normal", 5, backward=True),
     ]
 }
-ORDERED = list(WORKLOADS.values())
+ORDERED = list(WORKLOADS.values())  # the five configurations
 HEADLINE = ORDERED[2]
+# Serving shape for the recurrent decode step: 256 sequences x 16 heads, the headline's
+# per-head sizes; the fp32 running state (268 MB) exceeds L2, so every step streams it.
+# N = tokens cycled through by the bench.
+DECODE = Workload("n_decode_bf16_B256H16_d64M128", "n", True, "bf16", 256, 16, 64, 64, 128,
+                  64 ** -0.25, "normal", 6, decode=True)
+WORKLOADS[DECODE.name] = DECODE
 
 
 def bf16_bits(x: np.ndarray) -> np.ndarray:

@@ -71,3 +71,24 @@ def test_host_validation_without_gpu(lib):
     args = [p] * 3 + [p, None, 1, p, p, p, p, p, p, p]
     assert lib.flex_linattn_bwd(ctypes.byref(ok), *args, p, p, 1 << 24, None) == FLEX_EINVAL
     assert lib.flex_strerror(FLEX_EINVAL)
+
+
+def test_decode_host_validation_without_gpu(lib):
+    from paper_2606_27748_gb300.flexattn import FlexShape, FLEX_EINVAL, FLEX_EWORKSPACE
+    p = ctypes.c_void_p(4096)  # never dereferenced: validation fails first
+    one = FlexShape(2, 3, 1, 64, 64, 1)
+    two = FlexShape(2, 3, 2, 64, 64, 1)  # more than one token per sequence
+    need = lib.flex_decode_workspace_bytes(ctypes.byref(one))
+    # header + phi(q), phi(k): B H x 2 x 2M fp32
+    assert need == 256 + 2 * 3 * 2 * 128 * 4
+    assert lib.flex_decode_workspace_bytes(ctypes.byref(two)) == 0
+    assert lib.flex_linattn_decode(ctypes.byref(two), p, p, p, p, None, p, p, p, None,
+                                   p, need, None) == FLEX_EINVAL
+    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, None, p, p, None,
+                                   p, need, None) == FLEX_EINVAL
+    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, p, p,
+                                   ctypes.c_void_p(4097), None, p, need, None) == FLEX_EINVAL
+    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, p, p, p, None,
+                                   p, need - 1, None) == FLEX_EWORKSPACE
+    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, p, p, p, None,
+                                   None, need, None) == FLEX_EINVAL
