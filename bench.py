@@ -16,6 +16,7 @@ collective on the data path), so the value is weak-scaled.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import glob
 import hashlib
 import json
@@ -51,6 +52,9 @@ def parse_args():
                     choices=list(workloads.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="run the workload with this batch B instead of its own (a smaller "
+                         "case for profiling; the line's config names the changed workload)")
     return ap.parse_args()
 
 
@@ -619,6 +623,8 @@ def run_decode(args, w):
 def main():
     args = parse_args()
     w = workloads.WORKLOADS[args.workload]
+    if args.batch is not None and args.batch != w.B:
+        w = dataclasses.replace(w, B=args.batch, name=f"{w.name}@B{args.batch}")
     if args.impl == "reference":
         run_reference(args, w)
     elif w.decode:

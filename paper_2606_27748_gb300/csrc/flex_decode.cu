@@ -7,12 +7,12 @@
 //
 // The step is a stream over the state (2 x 2M x (d + 1) x 4 bytes per (b, h), read and
 // written once); the feature map is a small batched product per head.  Two kernels:
-//   decode_features  one CTA per (head, kG sequences): the head's frequency rows are
-//                    staged in shared memory one tile of 32 rows at a time and serve all
-//                    kG sequences (q and k), so W is read 2 kG times less often than by a
-//                    per-token kernel; phi(q), phi(k) (Eq. phi_n, or the product form of
-//                    Eq. phi_non with u = (W1+W2)/2 x and w = (W1-W2)/2 x; scaled by
-//                    M^{-1/2}; fp32, accurate sincosf) go to the workspace;
+//   decode_features  one CTA per (head, kG sequences, tile of 32 frequency rows): the
+//                    tile is staged in shared memory and serves all kG sequences (q and
+//                    k), so W is read 2 kG times less often than by a per-token kernel;
+//                    phi(q), phi(k) (Eq. phi_n, or the product form of Eq. phi_non with
+//                    u = (W1+W2)/2 x and w = (W1-W2)/2 x; scaled by M^{-1/2}; fp32,
+//                    sin/cos after a reduction by 2 pi) go to the workspace;
 //   decode_state     one CTA of 256 threads per (b, h), three per SM: starts asynchronous
 //                    16-byte copies of S (up to 64 KB of rows) into shared memory and the
 //                    loads of z, THEN waits for the features (programmatic dependent
@@ -44,9 +44,31 @@ __device__ __forceinline__ void cp_async16(void* smem, const void* gmem)
     const unsigned s = (unsigned)__cvta_generic_to_shared(smem);
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(s), "l"(gmem) : "memory");
 }
+// A load that stays after griddepcontrol.wait: volatile asm keeps its order relative to
+// the wait (a plain load from a const __restrict__ pointer may be hoisted above it), and
+// .cg reads L2, where the previous grid's stores are.
+__device__ __forceinline__ float ld_after_wait(const float* p)
+{
+    float x;
+    asm volatile("ld.global.cg.f32 %0, [%1];\n" : "=f"(x) : "l"(p) : "memory");
+    return x;
+}
 __device__ __forceinline__ void cp_async_wait_all()
 {
     asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;\n" ::: "memory");
+}
+
+// sin and cos of x: Cody-Waite reduction by 2 pi (the fp32 value of 2 pi plus the fp32
+// value of the remainder, both computed from the mathematical constant) to |r| <= pi, then
+// the hardware approximations, whose absolute error on [-pi, pi] is a few 1e-7.
+__device__ __forceinline__ void sincos_reduced(float x, float* s, float* c)
+{
+    constexpr float kInv2Pi = 0.15915493667125702f;
+    constexpr float k2PiHi = 6.2831854820251465f;
+    constexpr float k2PiLo = -1.7484555314695172e-07f;
+    const float n = rintf(x * kInv2Pi);
+    const float r = fmaf(-n, k2PiLo, fmaf(-n, k2PiHi, x));
+    __sincosf(r, s, c);
 }
 
 __device__ __forceinline__ float to_f32(float x) { return x; }
@@ -54,87 +76,120 @@ __device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162flo
 __device__ __forceinline__ void from_f32(float* p, float x) { *p = x; }
 __device__ __forceinline__ void from_f32(__nv_bfloat16* p, float x) { *p = __float2bfloat16_rn(x); }
 
-// phi: [B*H][2][2M] fp32 (0 = phi(q), 1 = phi(k)).
-template <typename T, bool NS>
-__global__ void __launch_bounds__(kThreadsF)
+// phi: [B*H][2][2M] fp32 (0 = phi(q), 1 = phi(k)).  CTA = (head, kG sequences, tile of
+// kTF frequency rows); lane = row, warp = kTokW token vectors.
+// D4C: d / 4 as a compile-time constant (the inner loop unrolls fully), or 0 for any d.
+template <typename T, bool NS, int D4C>
+__global__ void __launch_bounds__(kThreadsF, 4)
     decode_features(int B, int H, int d, int M, const T* __restrict__ q,
                     const T* __restrict__ k, const float* __restrict__ W1,
                     const float* __restrict__ W2, float* __restrict__ phi)
 {
     // The state kernel may launch now; it waits for this grid before reading phi.
     asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
-    extern __shared__ float fsm[];
-    const int ld = d + 1, F = 2 * M;
-    float* wu = fsm;                              // [kTF][d + 1]: W1 rows, or U rows
-    float* wv = wu + kTF * ld;                    // [kTF][d + 1]: V rows (n only)
+    extern __shared__ float4 fsm4[];
+    // Row pitch d + 4 floats: the float4 reads of 32 rows (one per lane) take the minimum
+    // of 4 shared-memory wavefronts.
+    const int ld = d + 4, F = 2 * M;
+    float* wu = reinterpret_cast<float*>(fsm4);   // [kTF][d + 4]: W1 rows, or U rows
+    float* wv = wu + kTF * ld;                    // [kTF][d + 4]: V rows (n only)
     float* xs = wv + (NS ? kTF * ld : 0);         // [2 kG][d]: token vector t = 2 s + which
-    const int groups = (B + kG - 1) / kG;
-    const int h = blockIdx.x / groups, b0 = (blockIdx.x % groups) * kG;
-    const int ntok = 2 * min(kG, B - b0);
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int tiles = (M + kTF - 1) / kTF, groups = (B + kG - 1) / kG;
+    const int tile = blockIdx.x % tiles, grp = (blockIdx.x / tiles) % groups;
+    const int h = blockIdx.x / (tiles * groups);
+    const int b0 = grp * kG, f0 = tile * kTF, ntok = 2 * min(kG, B - b0);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, d4 = D4C ? D4C : d / 4;
     constexpr int kWarps = kThreadsF / 32;
     constexpr int kTokW = 2 * kG / kWarps;        // token vectors per warp
 
-    for (int i = tid; i < 2 * kG * d; i += kThreadsF) {
-        const int t = i / d, e = i % d;
-        float xv = 0.f;
-        if (t < ntok) {
-            const size_t io = ((size_t)(b0 + t / 2) * H + h) * d + e;
-            xv = to_f32((t & 1) ? k[io] : q[io]);
+    // Staging: every load of the thread is issued before the first shared-memory store
+    // (compile-time trip counts), so the CTA waits for one round trip, not one per row.
+    constexpr int kXE = kMaxD / 32;               // elements per lane and token vector
+    constexpr int kWR = kTF / kWarps;             // W rows per warp
+    float xr[kTokW][kXE];
+    float4 ar[kWR], cr[kWR];
+#pragma unroll
+    for (int j = 0; j < kTokW; ++j) {             // warp per token vector, lane per element
+        const int t = warp + j * kWarps;
+        const size_t io = ((size_t)(b0 + t / 2) * H + h) * d;
+#pragma unroll
+        for (int i = 0; i < kXE; ++i) {
+            const int e = lane + 32 * i;
+            xr[j][i] = (t < ntok && e < d) ? to_f32((t & 1) ? k[io + e] : q[io + e]) : 0.f;
         }
-        xs[i] = xv;
     }
-    const float scale = rsqrtf((float)M);
-    for (int f0 = 0; f0 < M; f0 += kTF) {
-        __syncthreads();  // the previous tile is consumed (and xs written, first time)
-        for (int i = tid; i < kTF * d; i += kThreadsF) {
-            const int r = i / d, e = i % d, f = f0 + r;
-            float a = 0.f, c = 0.f;
-            if (f < M) {
-                a = W1[((size_t)h * M + f) * d + e];
-                if (NS) c = W2[((size_t)h * M + f) * d + e];
-            }
+#pragma unroll
+    for (int i = 0; i < kWR; ++i) {               // warp per row, lane per float4 (d4 <= 32)
+        const int f = f0 + warp + kWarps * i;
+        ar[i] = cr[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (f < M && lane < d4) {
+            ar[i] = __ldg(reinterpret_cast<const float4*>(W1 + ((size_t)h * M + f) * d) + lane);
+            if (NS)
+                cr[i] = __ldg(reinterpret_cast<const float4*>(W2 + ((size_t)h * M + f) * d) + lane);
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < kTokW; ++j)
+#pragma unroll
+        for (int i = 0; i < kXE; ++i)
+            if (lane + 32 * i < d) xs[(warp + j * kWarps) * d + lane + 32 * i] = xr[j][i];
+#pragma unroll
+    for (int i = 0; i < kWR; ++i) {
+        if (lane < d4) {
+            const int r = warp + kWarps * i;
+            const float4 a = ar[i], c = cr[i];
+            float4* du = reinterpret_cast<float4*>(wu + r * ld) + lane;
             if (NS) {
-                wu[r * ld + e] = 0.5f * (a + c);
-                wv[r * ld + e] = 0.5f * (a - c);
+                *du = make_float4(0.5f * (a.x + c.x), 0.5f * (a.y + c.y), 0.5f * (a.z + c.z),
+                                  0.5f * (a.w + c.w));
+                *(reinterpret_cast<float4*>(wv + r * ld) + lane) =
+                    make_float4(0.5f * (a.x - c.x), 0.5f * (a.y - c.y), 0.5f * (a.z - c.z),
+                                0.5f * (a.w - c.w));
             } else {
-                wu[r * ld + e] = a;
+                *du = a;
             }
         }
-        __syncthreads();
-        float au[kTokW], av[kTokW];
+    }
+    __syncthreads();
+
+    float au[kTokW], av[kTokW];
 #pragma unroll
-        for (int j = 0; j < kTokW; ++j) au[j] = av[j] = 0.f;
-        const float* ru = wu + lane * ld;
-        const float* rv = wv + lane * ld;
-        for (int e = 0; e < d; ++e) {
-            const float pu = ru[e], pv = NS ? rv[e] : 0.f;
-#pragma unroll
-            for (int j = 0; j < kTokW; ++j) {
-                const float xv = xs[(warp + j * kWarps) * d + e];
-                au[j] = fmaf(pu, xv, au[j]);
-                if (NS) av[j] = fmaf(pv, xv, av[j]);
-            }
-        }
-        const int f = f0 + lane;
+    for (int j = 0; j < kTokW; ++j) au[j] = av[j] = 0.f;
+    const float4* ru = reinterpret_cast<const float4*>(wu + lane * ld);
+    const float4* rv = reinterpret_cast<const float4*>(wv + lane * ld);
+    const float4* x4 = reinterpret_cast<const float4*>(xs);
+#pragma unroll(D4C ? D4C : 2)
+    for (int e4 = 0; e4 < d4; ++e4) {
+        const float4 pu = ru[e4];
+        const float4 pv = NS ? rv[e4] : pu;
 #pragma unroll
         for (int j = 0; j < kTokW; ++j) {
-            const int t = warp + j * kWarps;
-            if (t < ntok && f < M) {
-                float su, cu;
-                sincosf(au[j], &su, &cu);
-                const float cw = NS ? scale * cosf(av[j]) : scale;
-                float* dst = phi + (((size_t)(b0 + t / 2) * H + h) * 2 + (t & 1)) * F;
-                dst[f] = cu * cw;
-                dst[M + f] = su * cw;
-            }
+            const float4 xv = x4[(warp + j * kWarps) * d4 + e4];  // broadcast
+            au[j] = fmaf(pu.x, xv.x, fmaf(pu.y, xv.y, fmaf(pu.z, xv.z, fmaf(pu.w, xv.w, au[j]))));
+            if (NS)
+                av[j] = fmaf(pv.x, xv.x, fmaf(pv.y, xv.y, fmaf(pv.z, xv.z, fmaf(pv.w, xv.w, av[j]))));
+        }
+    }
+    const float scale = rsqrtf((float)M);
+    const int f = f0 + lane;
+#pragma unroll
+    for (int j = 0; j < kTokW; ++j) {
+        const int t = warp + j * kWarps;
+        if (t < ntok && f < M) {
+            float su, cu, sw, cw = 1.f;
+            sincos_reduced(au[j], &su, &cu);
+            if (NS) sincos_reduced(av[j], &sw, &cw);
+            cw *= scale;
+            float* dst = phi + (((size_t)(b0 + t / 2) * H + h) * 2 + (t & 1)) * F;
+            dst[f] = cu * cw;
+            dst[M + f] = su * cw;
         }
     }
 }
 
 template <typename T>
 __global__ void __launch_bounds__(kThreadsD, 3)
-    decode_state(int d, int M, const T* __restrict__ v, const float* __restrict__ phi,
+    decode_state(int d, int M, const T* __restrict__ v, const float* phi,
                  float* __restrict__ S, float* __restrict__ z, T* __restrict__ out,
                  float* __restrict__ den)
 {
@@ -159,7 +214,15 @@ __global__ void __launch_bounds__(kThreadsD, 3)
     if (tid < d) vs[tid] = to_f32(v[u * d + tid]);
 
     asm volatile("griddepcontrol.wait;\n" ::: "memory");  // the features are written
-    for (int i = tid; i < 2 * F; i += kThreadsD) ph[i / F][i % F] = phi[u * 2 * F + i];
+    float pr[2 * kMaxF / kThreadsD];                        // all loads, then the stores
+#pragma unroll
+    for (int j = 0; j < 2 * kMaxF / kThreadsD; ++j)
+        if (tid + kThreadsD * j < 2 * F) pr[j] = ld_after_wait(phi + u * 2 * F + tid + kThreadsD * j);
+#pragma unroll
+    for (int j = 0; j < 2 * kMaxF / kThreadsD; ++j) {
+        const int i = tid + kThreadsD * j;
+        if (i < 2 * F) ph[i / F][i % F] = pr[j];
+    }
 
     // Thread (rg, c4) owns float4 column c4 of the rows rg + ngrp * i of each chunk.
     const int ngrp = kThreadsD / d4, rg = tid / d4, c4 = tid % d4;
@@ -223,12 +286,15 @@ cudaError_t launch_typed(const Problem& p, const void* q, const void* k, const v
                          const float* W1, const float* W2, float* S, float* z, void* out,
                          float* den, float* phi, cudaStream_t s)
 {
-    const long long fctas = (long long)p.H * ((p.B + kG - 1) / kG);
+    const long long fctas = (long long)p.H * ((p.B + kG - 1) / kG) * ((p.M + kTF - 1) / kTF);
     const long long sctas = (long long)p.B * p.H;
     if (fctas > 0x7fffffffLL || sctas > 0x7fffffffLL) return cudaErrorInvalidValue;
 
-    const size_t fsmem = ((size_t)kTF * (p.d + 1) * (NS ? 2 : 1) + 2 * kG * p.d) * sizeof(float);
-    auto fk = decode_features<T, NS>;
+    const size_t fsmem = ((size_t)kTF * (p.d + 4) * (NS ? 2 : 1) + 2 * kG * p.d) * sizeof(float);
+    auto fk = p.d == 32    ? decode_features<T, NS, 8>
+              : p.d == 64  ? decode_features<T, NS, 16>
+              : p.d == 128 ? decode_features<T, NS, 32>
+                           : decode_features<T, NS, 0>;
     cudaError_t e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fsmem);
     if (e != cudaSuccess) return e;
     fk<<<(unsigned)fctas, kThreadsF, fsmem, s>>>(p.B, p.H, p.d, p.M, (const T*)q, (const T*)k,

@@ -94,3 +94,31 @@ def test_decode_launch_count():
                             to_dev(ins["v"][:, :, 0], "bf16"), to_dev(ins["W1"], "f32"),
                             to_dev(ins["W2"], "f32"), S, z)
     assert flexattn.kernel_launches() - n0 == 2  # features, then the state stream
+
+
+def test_decode_reads_features_only_after_they_are_written():
+    """The state kernel starts before the features kernel ends (its state copies overlap
+    it) and must read phi only after the dependency wait.  Poison the workspace with NaN
+    before every step: any early read shows up as a NaN, and the results must equal, bit
+    for bit, those of a run whose workspace keeps the previous step's features."""
+    w = WL[2]
+    B, H, N, d, M = 64, 16, 24, 64, 128
+    _, ins = _inputs(w, B, H, N, d, M, "bf16")
+    W1, W2 = to_dev(ins["W1"], "f32"), to_dev(ins["W2"], "f32")
+    q, k, v = (to_dev(ins[n], "bf16") for n in "qkv")
+    toks = [tuple(t[:, :, i].contiguous() for t in (q, k, v)) for i in range(N)]
+    runs = []
+    for poison in (False, True):
+        S, z = flexattn.decode_state(B, H, M, d)
+        ws = flexattn.decode_workspace(B, H, M, d)
+        outs = []
+        for i in range(N):
+            if poison:
+                ws.view(torch.float32)[64:].fill_(float("nan"))  # past the 256-byte header
+            o, dn = flexattn.linattn_decode(*toks[i], W1, W2, S, z, ws=ws)
+            outs.append(torch.cat([o.float().flatten(), dn.flatten()]))
+        torch.cuda.synchronize()
+        runs.append((torch.stack(outs), S.clone(), z.clone()))
+    (oa, Sa, za), (ob, Sb, zb) = runs
+    assert torch.isfinite(ob).all() and torch.isfinite(Sb).all()
+    assert torch.equal(oa, ob) and torch.equal(Sa, Sb) and torch.equal(za, zb)
