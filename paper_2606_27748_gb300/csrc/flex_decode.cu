@@ -7,12 +7,13 @@
 //
 // The step is a stream over the state (2 x 2M x (d + 1) x 4 bytes per (b, h), read and
 // written once); the feature map is a small batched product per head.  Two kernels:
-//   decode_features  one CTA per (head, kG sequences, tile of 32 frequency rows): the
-//                    tile is staged in shared memory and serves all kG sequences (q and
-//                    k), so W is read 2 kG times less often than by a per-token kernel;
-//                    phi(q), phi(k) (Eq. phi_n, or the product form of Eq. phi_non with
-//                    u = (W1+W2)/2 x and w = (W1-W2)/2 x; scaled by M^{-1/2}; fp32,
-//                    sin/cos after a reduction by 2 pi) go to the workspace;
+//   decode_features  one CTA per (head, kG = 32 sequences, tile of 32 frequency rows):
+//                    the tile is copied into shared memory and serves all 2 kG token
+//                    vectors (q and k), so W is read 2 kG times less often than by a
+//                    per-token kernel; phi(q), phi(k) (Eq. phi_n, or the product form of
+//                    Eq. phi_non with u = (W1+W2)/2 x and w = (W1-W2)/2 x formed from the
+//                    two dot products; scaled by M^{-1/2}; fp32, sin/cos after a
+//                    reduction by 2 pi) go to the workspace;
 //   decode_state     one CTA of 256 threads per (b, h), three per SM: starts asynchronous
 //                    16-byte copies of S (up to 64 KB of rows) into shared memory and the
 //                    loads of z, THEN waits for the features (programmatic dependent
@@ -32,7 +33,7 @@ namespace flex {
 namespace {
 
 constexpr int kThreadsF = 256;
-constexpr int kG = 16;         // sequences of one head per features CTA
+constexpr int kG = 32;         // sequences of one head per features CTA
 constexpr int kTF = 32;        // frequency rows per shared-memory tile (one per lane)
 constexpr int kThreadsD = 256;
 constexpr int kSBuf = 16384;   // floats of S staged in shared memory per chunk (64 KB)
@@ -77,7 +78,8 @@ __device__ __forceinline__ void from_f32(float* p, float x) { *p = x; }
 __device__ __forceinline__ void from_f32(__nv_bfloat16* p, float x) { *p = __float2bfloat16_rn(x); }
 
 // phi: [B*H][2][2M] fp32 (0 = phi(q), 1 = phi(k)).  CTA = (head, kG sequences, tile of
-// kTF frequency rows); lane = row, warp = kTokW token vectors.
+// kTF frequency rows); lane = row, warp = kTokW token vectors, so each thread carries
+// 2 kTokW independent dot products (W1 x and W2 x of its rows).
 // D4C: d / 4 as a compile-time constant (the inner loop unrolls fully), or 0 for any d.
 template <typename T, bool NS, int D4C>
 __global__ void __launch_bounds__(kThreadsF, 4)
@@ -89,85 +91,70 @@ __global__ void __launch_bounds__(kThreadsF, 4)
     asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
     extern __shared__ float4 fsm4[];
     // Row pitch d + 4 floats: the float4 reads of 32 rows (one per lane) take the minimum
-    // of 4 shared-memory wavefronts.
-    const int ld = d + 4, F = 2 * M;
-    float* wu = reinterpret_cast<float*>(fsm4);   // [kTF][d + 4]: W1 rows, or U rows
-    float* wv = wu + kTF * ld;                    // [kTF][d + 4]: V rows (n only)
-    float* xs = wv + (NS ? kTF * ld : 0);         // [2 kG][d]: token vector t = 2 s + which
+    // of 4 shared-memory wavefronts, and every row starts on 16 bytes.
+    const int ld = D4C ? 4 * D4C + 4 : d + 4, F = 2 * M;
+    float* w1s = reinterpret_cast<float*>(fsm4);  // [kTF][ld]: W1 rows of the tile
+    float* w2s = w1s + kTF * ld;                  // [kTF][ld]: W2 rows (n only)
+    float* xs = w2s + (NS ? kTF * ld : 0);        // [2 kG][d]: token vector t = 2 s + which
     const int tiles = (M + kTF - 1) / kTF, groups = (B + kG - 1) / kG;
     const int tile = blockIdx.x % tiles, grp = (blockIdx.x / tiles) % groups;
     const int h = blockIdx.x / (tiles * groups);
     const int b0 = grp * kG, f0 = tile * kTF, ntok = 2 * min(kG, B - b0);
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, d4 = D4C ? D4C : d / 4;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int d4 = D4C ? D4C : d / 4, dd = 4 * d4;
     constexpr int kWarps = kThreadsF / 32;
     constexpr int kTokW = 2 * kG / kWarps;        // token vectors per warp
+    constexpr int kXE = D4C ? (4 * D4C + 31) / 32 : kMaxD / 32;  // elements per lane and vector
 
-    // Staging: every load of the thread is issued before the first shared-memory store
-    // (compile-time trip counts), so the CTA waits for one round trip, not one per row.
-    constexpr int kXE = kMaxD / 32;               // elements per lane and token vector
-    constexpr int kWR = kTF / kWarps;             // W rows per warp
+    // Staging: the W tile by asynchronous copies (no registers), rows past M zero; the
+    // token vectors through registers (bf16 -> fp32), all loads before the first store.
+    for (int i = tid; i < kTF * d4; i += kThreadsF) {
+        const int r = i / d4, e4 = i % d4, f = f0 + r;
+        float4* d1 = reinterpret_cast<float4*>(w1s + r * ld) + e4;
+        float4* d2 = reinterpret_cast<float4*>(w2s + r * ld) + e4;
+        if (f < M) {
+            cp_async16(d1, W1 + ((size_t)h * M + f) * dd + 4 * e4);
+            if (NS) cp_async16(d2, W2 + ((size_t)h * M + f) * dd + 4 * e4);
+        } else {
+            *d1 = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (NS) *d2 = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+    }
     float xr[kTokW][kXE];
-    float4 ar[kWR], cr[kWR];
 #pragma unroll
     for (int j = 0; j < kTokW; ++j) {             // warp per token vector, lane per element
         const int t = warp + j * kWarps;
-        const size_t io = ((size_t)(b0 + t / 2) * H + h) * d;
+        const size_t io = ((size_t)(b0 + t / 2) * H + h) * dd;
 #pragma unroll
         for (int i = 0; i < kXE; ++i) {
             const int e = lane + 32 * i;
-            xr[j][i] = (t < ntok && e < d) ? to_f32((t & 1) ? k[io + e] : q[io + e]) : 0.f;
-        }
-    }
-#pragma unroll
-    for (int i = 0; i < kWR; ++i) {               // warp per row, lane per float4 (d4 <= 32)
-        const int f = f0 + warp + kWarps * i;
-        ar[i] = cr[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (f < M && lane < d4) {
-            ar[i] = __ldg(reinterpret_cast<const float4*>(W1 + ((size_t)h * M + f) * d) + lane);
-            if (NS)
-                cr[i] = __ldg(reinterpret_cast<const float4*>(W2 + ((size_t)h * M + f) * d) + lane);
+            xr[j][i] = (t < ntok && e < dd) ? to_f32((t & 1) ? k[io + e] : q[io + e]) : 0.f;
         }
     }
 #pragma unroll
     for (int j = 0; j < kTokW; ++j)
 #pragma unroll
         for (int i = 0; i < kXE; ++i)
-            if (lane + 32 * i < d) xs[(warp + j * kWarps) * d + lane + 32 * i] = xr[j][i];
-#pragma unroll
-    for (int i = 0; i < kWR; ++i) {
-        if (lane < d4) {
-            const int r = warp + kWarps * i;
-            const float4 a = ar[i], c = cr[i];
-            float4* du = reinterpret_cast<float4*>(wu + r * ld) + lane;
-            if (NS) {
-                *du = make_float4(0.5f * (a.x + c.x), 0.5f * (a.y + c.y), 0.5f * (a.z + c.z),
-                                  0.5f * (a.w + c.w));
-                *(reinterpret_cast<float4*>(wv + r * ld) + lane) =
-                    make_float4(0.5f * (a.x - c.x), 0.5f * (a.y - c.y), 0.5f * (a.z - c.z),
-                                0.5f * (a.w - c.w));
-            } else {
-                *du = a;
-            }
-        }
-    }
+            if (lane + 32 * i < dd) xs[(warp + j * kWarps) * dd + lane + 32 * i] = xr[j][i];
+    cp_async_wait_all();
     __syncthreads();
 
-    float au[kTokW], av[kTokW];
+    float a[kTokW], c[kTokW];
 #pragma unroll
-    for (int j = 0; j < kTokW; ++j) au[j] = av[j] = 0.f;
-    const float4* ru = reinterpret_cast<const float4*>(wu + lane * ld);
-    const float4* rv = reinterpret_cast<const float4*>(wv + lane * ld);
+    for (int j = 0; j < kTokW; ++j) a[j] = c[j] = 0.f;
+    const float4* r1 = reinterpret_cast<const float4*>(w1s + lane * ld);
+    const float4* r2 = reinterpret_cast<const float4*>(w2s + lane * ld);
     const float4* x4 = reinterpret_cast<const float4*>(xs);
 #pragma unroll(D4C ? D4C : 2)
     for (int e4 = 0; e4 < d4; ++e4) {
-        const float4 pu = ru[e4];
-        const float4 pv = NS ? rv[e4] : pu;
+        const float4 p1 = r1[e4];
+        const float4 p2 = NS ? r2[e4] : p1;
 #pragma unroll
         for (int j = 0; j < kTokW; ++j) {
             const float4 xv = x4[(warp + j * kWarps) * d4 + e4];  // broadcast
-            au[j] = fmaf(pu.x, xv.x, fmaf(pu.y, xv.y, fmaf(pu.z, xv.z, fmaf(pu.w, xv.w, au[j]))));
+            a[j] = fmaf(p1.x, xv.x, fmaf(p1.y, xv.y, fmaf(p1.z, xv.z, fmaf(p1.w, xv.w, a[j]))));
             if (NS)
-                av[j] = fmaf(pv.x, xv.x, fmaf(pv.y, xv.y, fmaf(pv.z, xv.z, fmaf(pv.w, xv.w, av[j]))));
+                c[j] = fmaf(p2.x, xv.x, fmaf(p2.y, xv.y, fmaf(p2.z, xv.z, fmaf(p2.w, xv.w, c[j]))));
         }
     }
     const float scale = rsqrtf((float)M);
@@ -176,9 +163,10 @@ __global__ void __launch_bounds__(kThreadsF, 4)
     for (int j = 0; j < kTokW; ++j) {
         const int t = warp + j * kWarps;
         if (t < ntok && f < M) {
+            // n: u = (W1 + W2)/2 x, w = (W1 - W2)/2 x; s: u = W1 x
             float su, cu, sw, cw = 1.f;
-            sincos_reduced(au[j], &su, &cu);
-            if (NS) sincos_reduced(av[j], &sw, &cw);
+            sincos_reduced(NS ? 0.5f * (a[j] + c[j]) : a[j], &su, &cu);
+            if (NS) sincos_reduced(0.5f * (a[j] - c[j]), &sw, &cw);
             cw *= scale;
             float* dst = phi + (((size_t)(b0 + t / 2) * H + h) * 2 + (t & 1)) * F;
             dst[f] = cu * cw;
@@ -290,7 +278,7 @@ cudaError_t launch_typed(const Problem& p, const void* q, const void* k, const v
     const long long sctas = (long long)p.B * p.H;
     if (fctas > 0x7fffffffLL || sctas > 0x7fffffffLL) return cudaErrorInvalidValue;
 
-    const size_t fsmem = ((size_t)kTF * (p.d + 4) * (NS ? 2 : 1) + 2 * kG * p.d) * sizeof(float);
+    const size_t fsmem = ((size_t)kTF * (p.d + 4) * 2 + 2 * kG * p.d) * sizeof(float);
     auto fk = p.d == 32    ? decode_features<T, NS, 8>
               : p.d == 64  ? decode_features<T, NS, 16>
               : p.d == 128 ? decode_features<T, NS, 32>
