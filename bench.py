@@ -588,7 +588,8 @@ def run_decode(args, w):
     nbytes, flops, ops = decode_work(w)
     sec = kernel_ms * 1e-3
     roof = {"bound": "hbm", "achieved": nbytes / sec / 1e9, "peak": peaks["hbm_gbs"],
-            "unit": "GB/s", "frac": nbytes / sec / 1e9 / peaks["hbm_gbs"], "traffic": None,
+            "unit": "GB/s", "frac": nbytes / sec / 1e9 / peaks["hbm_gbs"],
+            "traffic": recorded_traffic(w),
             "peak_source": peaks_src, "algorithmic_bytes_per_launch": nbytes,
             "fracs": {"hbm": nbytes / sec / 1e9 / peaks["hbm_gbs"],
                       "tensor": flops / sec / 1e12 / peaks["bf16_tflops"]},
