@@ -52,6 +52,10 @@ def parse_args():
                     choices=list(workloads.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--sweep-n", default=None,
+                    help="comma-separated sequence lengths: time the workload's forward at "
+                         "each N (same B, H, d, M) and print one JSON line per N with the "
+                         "time and the device memory held (the linear-scaling curve)")
     ap.add_argument("--batch", type=int, default=None,
                     help="run the workload with this batch B instead of its own (a smaller "
                          "case for profiling; the line's config names the changed workload)")
@@ -621,12 +625,74 @@ def run_decode(args, w):
         dist.destroy_process_group()
 
 
+def run_sweep(args, w):
+    """Forward time and device memory against N for one workload family (the paper's
+    time-and-memory-versus-length comparison, our own curve only).  Per N: inputs from the
+    workload's generator at that N, warm-up, then `steps` forwards each timed with CUDA
+    events on the launching stream, L2 flushed (a 256 MB write) before each; memory is
+    the peak held by this program's device allocations (inputs, out, den, workspace)."""
+    import statistics as st
+
+    import torch
+
+    from paper_2606_27748_gb300 import build, flexattn
+    build.build()
+    flexattn.load()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    tdt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    for n in (int(x) for x in args.sweep_n.split(",")):
+        wn = w.replace(N=n, name=f"{w.name}@N{n}")
+        ins = workloads.make_inputs(wn)
+        torch.cuda.synchronize()
+        torch.cuda.reset_peak_memory_stats(dev)
+        base = torch.cuda.memory_allocated(dev)
+        q, k, v = (torch.from_numpy(ins[x]).to(tdt).to(dev) for x in "qkv")
+        W1 = torch.from_numpy(ins["W1"]).to(dev)
+        W2 = None if ins["W2"] is None else torch.from_numpy(ins["W2"]).to(dev)
+        del ins
+        out = torch.empty_like(q)
+        den = torch.empty(q.shape[:3], dtype=torch.float32, device=dev)
+        shape = flexattn.shape_of(q, W1)
+        ws = flexattn.workspace(shape, w.causal, False, dev)
+        for _ in range(max(3, args.warmup)):
+            flexattn.linattn_fwd(q, k, v, W1, W2, w.causal, out=out, den=den, ws=ws)
+        flexattn.check_status(ws)
+        times = []
+        for _ in range(args.steps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            flexattn.linattn_fwd(q, k, v, W1, W2, w.causal, out=out, den=den, ws=ws)
+            b.record(stream)
+            torch.cuda.synchronize()
+            times.append(a.elapsed_time(b))
+        flexattn.check_status(ws)
+        ms = st.median(times)
+        peak = torch.cuda.max_memory_allocated(dev) - base
+        print(json.dumps({
+            "sweep": "N", "workload": wn.name, "N": n, "B": w.B, "H": w.H, "d": w.d,
+            "M": w.M, "variant": w.variant, "causal": w.causal, "dtype": w.dtype,
+            "ms_per_forward": ms, "tokens_per_s": w.B * n / (ms * 1e-3),
+            "ns_per_token_head": ms * 1e6 / (w.B * w.H * n),
+            "device_bytes": peak, "workspace_bytes": ws.numel(),
+            "bytes_per_token_head": peak / (w.B * w.H * n), "steps": args.steps,
+            "l2": "flushed before each timed forward"}), flush=True)
+        del q, k, v, W1, W2, out, den, ws
+
+
 def main():
     args = parse_args()
     w = workloads.WORKLOADS[args.workload]
     if args.batch is not None and args.batch != w.B:
         w = dataclasses.replace(w, B=args.batch, name=f"{w.name}@B{args.batch}")
-    if args.impl == "reference":
+    if args.sweep_n:
+        if w.decode or w.backward:
+            raise SystemExit("--sweep-n times the forward of a forward workload")
+        run_sweep(args, w)
+    elif args.impl == "reference":
         run_reference(args, w)
     elif w.decode:
         run_decode(args, w)

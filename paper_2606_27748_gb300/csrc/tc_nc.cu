@@ -35,7 +35,9 @@ using namespace tc;
 constexpr int kC = 128;
 constexpr int kThreadsNC = 448;
 constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kWarpEW = 10;
-constexpr int kTargetUnits = 8 * 152;  // work units per launch (a multiple of the SMs)
+constexpr int kSMs = 152;
+constexpr int kTargetUnits = 8 * kSMs;  // most work units per launch
+constexpr int kSetupChunks = 5;         // fixed cost of a unit, in chunk times
 
 enum { kState = 0, kOut = 1 };
 
@@ -400,14 +402,26 @@ bool tc_nc_supported(const Problem& p)
     return p.bf16 && p.d == 64 && (p.M == 64 || p.M == 128) && !p.causal;
 }
 
+// Splits per sequence.  A unit costs a fixed set-up (frequencies, tensor memory, pipeline
+// fill, partial-state write: about kSetupChunks chunk times, fitted to measured times over
+// N = 1K..64K) plus its chunks, and one unit runs per SM at a time; the split count
+// minimises waves x (set-up + chunks per unit), at most kTargetUnits units (which bounds
+// the partial-state workspace), fewest splits on ties.
 int tc_nc_splits(const Problem& p)
 {
     const long long BH = (long long)p.B * p.H;
     const int nch = (p.N + kC - 1) / kC;
-    long long s = (kTargetUnits + BH - 1) / BH;
-    if (s > nch) s = nch;
-    if (s < 1) s = 1;
-    return (int)s;
+    const long long smax = std::max(1LL, std::min<long long>(nch, (kTargetUnits + BH - 1) / BH));
+    long long best = 1, best_cost = -1;
+    for (long long s = 1; s <= smax; ++s) {
+        const long long waves = (BH * s + kSMs - 1) / kSMs;
+        const long long cost = waves * (kSetupChunks + (nch + s - 1) / s);
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best = s;
+        }
+    }
+    return (int)best;
 }
 
 size_t tc_nc_ws_bytes(const Problem& p)
