@@ -65,10 +65,11 @@ class Oracle:
         i = ctypes.c_int
         lib.oracle_featmap.argtypes = [i, i, i, i, i, dp, dp, dp, dp]
         lib.oracle_featmap_sumform.argtypes = [i, i, i, i, i, dp, dp, dp, dp]
-        lib.oracle_linattn_fwd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, i, dp, dp, i]
-        lib.oracle_linattn_bwd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, i, dp, dp, dp,
-                                           dp, dp, dp, i]
-        lib.oracle_linattn_decode.argtypes = [i, i, i, i, dp, dp, dp, dp, dp, dp, dp, dp, dp]
+        lib.oracle_linattn_fwd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, dp, i, dp, dp, i]
+        lib.oracle_linattn_bwd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, dp, i, dp, dp, dp,
+                                           dp, dp, dp, dp, i]
+        lib.oracle_linattn_decode.argtypes = [i, i, i, i, dp, dp, dp, dp, dp, dp, dp, dp, dp,
+                                              dp]
         for fn in (lib.oracle_featmap, lib.oracle_featmap_sumform, lib.oracle_linattn_fwd,
                    lib.oracle_linattn_bwd, lib.oracle_linattn_decode):
             fn.restype = ctypes.c_int
@@ -109,43 +110,49 @@ class Oracle:
             raise ValueError("oracle_featmap_sumform: bad shape")
         return phi
 
-    def fwd(self, q, k, v, W1, W2=None, causal=True, nthreads=None):
-        """(out [B, H, N, d], den [B, H, N]) of Eq. (linear att)."""
-        q, k, v, W1, W2 = (self._f64(a) for a in (q, k, v, W1, W2))
+    def fwd(self, q, k, v, W1, W2=None, causal=True, nthreads=None, tau=None):
+        """(out [B, H, N, d], den [B, H, N]) of Eq. (linear att); tau [H]: the norm
+        prefactor of Sec. 3.2 (a key weight; den excludes the query's factor)."""
+        q, k, v, W1, W2, tau = (self._f64(a) for a in (q, k, v, W1, W2, tau))
         B, H, N, d = q.shape
         M = W1.shape[1]
         out = np.empty_like(q)
         den = np.empty((B, H, N))
         nt = nthreads or os.cpu_count() or 1
         rc = self._lib.oracle_linattn_fwd(B, H, N, d, M, self._p(q), self._p(k), self._p(v),
-                                          self._p(W1), self._p(W2), int(bool(causal)),
-                                          self._p(out), self._p(den), nt)
+                                          self._p(W1), self._p(W2), self._p(tau),
+                                          int(bool(causal)), self._p(out), self._p(den), nt)
         if rc != 0:
             raise ValueError("oracle_linattn_fwd: bad shape")
         return out, den
 
-    def bwd(self, q, k, v, W1, W2, causal, dout, nthreads=None):
-        """Gradients (dq, dk, dv, dW1, dW2) of L = sum(dout * out); dW2 is None if W2 is."""
-        q, k, v, W1, W2, dout = (self._f64(a) for a in (q, k, v, W1, W2, dout))
+    def bwd(self, q, k, v, W1, W2, causal, dout, nthreads=None, tau=None):
+        """Gradients (dq, dk, dv, dW1, dW2) of L = sum(dout * out); dW2 is None if W2 is.
+        With tau [H] (the norm prefactor) a sixth value, dtau [H], follows."""
+        q, k, v, W1, W2, dout, tau = (self._f64(a) for a in (q, k, v, W1, W2, dout, tau))
         B, H, N, d = q.shape
         M = W1.shape[1]
         dq, dk, dv = np.empty_like(q), np.empty_like(q), np.empty_like(q)
         dW1 = np.empty_like(W1)
         dW2 = None if W2 is None else np.empty_like(W2)
+        dtau = None if tau is None else np.empty(H)
         nt = nthreads or os.cpu_count() or 1
         rc = self._lib.oracle_linattn_bwd(B, H, N, d, M, self._p(q), self._p(k), self._p(v),
-                                          self._p(W1), self._p(W2), int(bool(causal)),
-                                          self._p(dout), self._p(dq), self._p(dk),
-                                          self._p(dv), self._p(dW1), self._p(dW2), nt)
+                                          self._p(W1), self._p(W2), self._p(tau),
+                                          int(bool(causal)), self._p(dout), self._p(dq),
+                                          self._p(dk), self._p(dv), self._p(dW1), self._p(dW2),
+                                          self._p(dtau), nt)
         if rc != 0:
             raise ValueError("oracle_linattn_bwd: bad shape")
-        return dq, dk, dv, dW1, dW2
+        if tau is None:
+            return dq, dk, dv, dW1, dW2
+        return dq, dk, dv, dW1, dW2, dtau
 
-    def decode(self, q, k, v, W1, W2, S, z):
+    def decode(self, q, k, v, W1, W2, S, z, tau=None):
         """One causal decode step (Eq. linear att as running sums, inclusive of the new
-        token): q, k, v [B, H, d]; state S [B, H, 2M, d], z [B, H, 2M] (not modified).
-        Returns (out [B, H, d], den [B, H], S', z')."""
-        q, k, v, W1, W2 = (self._f64(a) for a in (q, k, v, W1, W2))
+        token): q, k, v [B, H, d]; state S [B, H, 2M, d], z [B, H, 2M] (not modified);
+        tau [H] or None.  Returns (out [B, H, d], den [B, H], S', z')."""
+        q, k, v, W1, W2, tau = (self._f64(a) for a in (q, k, v, W1, W2, tau))
         S = np.array(S, dtype=np.float64, copy=True, order="C")
         z = np.array(z, dtype=np.float64, copy=True, order="C")
         B, H, d = q.shape
@@ -153,8 +160,8 @@ class Oracle:
         out = np.empty_like(q)
         den = np.empty((B, H))
         rc = self._lib.oracle_linattn_decode(B, H, d, M, self._p(q), self._p(k), self._p(v),
-                                             self._p(W1), self._p(W2), self._p(S), self._p(z),
-                                             self._p(out), self._p(den))
+                                             self._p(W1), self._p(W2), self._p(tau), self._p(S),
+                                             self._p(z), self._p(out), self._p(den))
         if rc != 0:
             raise ValueError("oracle_linattn_decode: bad shape")
         return out, den, S, z
@@ -175,13 +182,13 @@ def featmap(x, W1, W2=None):
     return load().featmap(x, W1, W2)
 
 
-def fwd(q, k, v, W1, W2=None, causal=True, nthreads=None):
-    return load().fwd(q, k, v, W1, W2, causal, nthreads)
+def fwd(q, k, v, W1, W2=None, causal=True, nthreads=None, tau=None):
+    return load().fwd(q, k, v, W1, W2, causal, nthreads, tau)
 
 
-def bwd(q, k, v, W1, W2, causal, dout, nthreads=None):
-    return load().bwd(q, k, v, W1, W2, causal, dout, nthreads)
+def bwd(q, k, v, W1, W2, causal, dout, nthreads=None, tau=None):
+    return load().bwd(q, k, v, W1, W2, causal, dout, nthreads, tau)
 
 
-def decode(q, k, v, W1, W2, S, z):
-    return load().decode(q, k, v, W1, W2, S, z)
+def decode(q, k, v, W1, W2, S, z, tau=None):
+    return load().decode(q, k, v, W1, W2, S, z, tau)

@@ -33,14 +33,26 @@ def features(x, W1, W2=None):
         2.0 * np.sqrt(M))
 
 
-def kernel_matrix(q, k, W1, W2=None):
-    """K[..., i, j] = phi(q_i) . phi(k_j)."""
-    return np.einsum("...if,...jf->...ij", features(q, W1, W2), features(k, W1, W2))
+def prefactored(x, W1, W2=None, tau=None):
+    """phi~(x) = exp(|x|^2 / exp(tau)) phi(x) (Sec. 3.2), tau [H]; phi(x) if tau is None."""
+    phi = features(x, W1, W2)
+    if tau is None:
+        return phi
+    x = np.asarray(x, dtype=np.float64)
+    t = np.asarray(tau, dtype=np.float64)[:, None]          # [H, 1] against [..., H, N]
+    return np.exp(np.sum(x * x, axis=-1) / np.exp(t))[..., None] * phi
 
 
-def attention(q, k, v, W1, W2=None, causal=True):
-    """(out, den): out_i = sum_j K_ij v_j / sum_j K_ij over j <= i (causal) or all j."""
-    K = kernel_matrix(q, k, W1, W2)
+def kernel_matrix(q, k, W1, W2=None, tau=None):
+    """K[..., i, j] = phi~(q_i) . phi~(k_j) (the prefactor on both sides, as printed)."""
+    return np.einsum("...if,...jf->...ij", prefactored(q, W1, W2, tau),
+                     prefactored(k, W1, W2, tau))
+
+
+def attention(q, k, v, W1, W2=None, causal=True, tau=None):
+    """(out, den): out_i = sum_j K_ij v_j / sum_j K_ij over j <= i (causal) or all j.
+    With tau, den includes the query's prefactor (it is the literal row sum)."""
+    K = kernel_matrix(q, k, W1, W2, tau)
     if causal:
         N = K.shape[-1]
         K = K * np.tril(np.ones((N, N)))

@@ -23,7 +23,12 @@
  *   - causal attention sums over j <= i (the diagonal is included).
  *   - the denominator is used as it is: no epsilon, no clamp.
  *   - the learned parameters of Flexformer_n are (W1, W2); dW1 and dW2 are returned.
- *   - the norm prefactor exp(|x|^2 / exp(tau)) is not part of this path.
+ *   - the norm prefactor of Sec. 3.2, phi~(x) = exp(|x|^2 / exp(tau)) phi(x), is optional
+ *     (tau per head; NULL = none).  The query's factor multiplies every term of row i of
+ *     both sums in Eq. (linear att) and cancels; what remains is a weight
+ *     w_j = exp(|k_j|^2 exp(-tau)) on key j, so S = sum_j w_j phi(k_j) v_j^T and
+ *     z = sum_j w_j phi(k_j).  den is phi(q_i)^T z (without the query factor), and dtau
+ *     is returned with the other gradients.
  *
  * The backward pass is the analytic gradient of L = sum_i dO_i . O_i, derived by hand
  * from Eq. (linear att) (the paper gives none; it only states that the frequencies are
@@ -32,7 +37,10 @@
  *   dphi(q_i) = S_i g_i + c_i z_i           (S_i, z_i: running sums over j <= i)
  *   dphi(k_j) = R_j v_j + r_j               (R_j = sum_{i>=j} phi(q_i) g_i^T, r_j = sum c_i phi(q_i))
  *   dv_j      = R_j^T phi(k_j)
- * and through the feature map by the chain rule.  For non-causal attention every
+ * and through the feature map by the chain rule.  With the key weight w_j the same
+ * formulas hold for phi~(k_j) = w_j phi(k_j); then dphi(k_j) = w_j dphi~(k_j) and, with
+ * dw_j = phi(k_j) . dphi~(k_j):  dk_j += dw_j w_j 2 exp(-tau) k_j,
+ * dtau += -dw_j w_j |k_j|^2 exp(-tau).  For non-causal attention every
  * running sum is replaced by the total.
  *
  * Layouts: q, k, v, out, dout, dq, dk, dv are [B][H][N][d]; W1, W2, dW1, dW2 are [H][M][d];
@@ -139,7 +147,15 @@ typedef struct {
     int N, d, M, causal;
     const double *q, *k, *v, *W1, *W2, *dout;
     double *out, *den, *dq, *dk, *dv, *dA, *dB;
+    double itau;   /* exp(-tau) of the head, 0 without the prefactor (then w_j = 1) */
+    double *dtau;  /* this sequence's dtau (backward with the prefactor), else NULL */
 } seq_job;
+
+/* Key weight of the norm prefactor (Sec. 3.2): w = exp(|k|^2 exp(-tau)). */
+static double key_weight(int d, const double* k, double itau)
+{
+    return exp(dot(d, k, k) * itau);
+}
 
 /* out[i] = phi(q_i)^T S / phi(q_i)^T z with S = sum phi(k_j) v_j^T, z = sum phi(k_j);
  * j runs over j <= i when causal, over all j otherwise. */
@@ -155,6 +171,8 @@ static void forward_seq(const seq_job* J)
     if (!J->causal) {
         for (int j = 0; j < N; ++j) {
             feature(d, M, J->k + (size_t)j * d, J->W1, J->W2, pk);
+            const double wj = key_weight(d, J->k + (size_t)j * d, J->itau);
+            for (int f = 0; f < D; ++f) pk[f] *= wj;
             for (int f = 0; f < D; ++f) {
                 z[f] += pk[f];
                 for (int e = 0; e < d; ++e) S[(size_t)f * d + e] += pk[f] * J->v[(size_t)j * d + e];
@@ -164,6 +182,8 @@ static void forward_seq(const seq_job* J)
     for (int i = 0; i < N; ++i) {
         if (J->causal) {
             feature(d, M, J->k + (size_t)i * d, J->W1, J->W2, pk);
+            const double wi = key_weight(d, J->k + (size_t)i * d, J->itau);
+            for (int f = 0; f < D; ++f) pk[f] *= wi;
             for (int f = 0; f < D; ++f) {
                 z[f] += pk[f];
                 for (int e = 0; e < d; ++e) S[(size_t)f * d + e] += pk[f] * J->v[(size_t)i * d + e];
@@ -194,12 +214,15 @@ static void backward_seq(const seq_job* J)
     forward_seq(&F);
 
     double* PQ = malloc(sizeof(double) * (size_t)N * D);   /* phi(q_i) */
-    double* PK = malloc(sizeof(double) * (size_t)N * D);   /* phi(k_j) */
+    double* PK = malloc(sizeof(double) * (size_t)N * D);   /* phi~(k_j) = w_j phi(k_j) */
+    double* wk = malloc(sizeof(double) * (size_t)N);       /* w_j */
     double* g = malloc(sizeof(double) * (size_t)N * d);    /* dout_i / den_i */
     double* cc = malloc(sizeof(double) * (size_t)N);       /* -(dout_i . out_i) / den_i */
     for (int i = 0; i < N; ++i) {
         feature(d, M, J->q + (size_t)i * d, J->W1, J->W2, PQ + (size_t)i * D);
         feature(d, M, J->k + (size_t)i * d, J->W1, J->W2, PK + (size_t)i * D);
+        wk[i] = key_weight(d, J->k + (size_t)i * d, J->itau);
+        for (int f = 0; f < D; ++f) PK[(size_t)i * D + f] *= wk[i];
         const double* dO = J->dout + (size_t)i * d;
         double s = 0.0;
         for (int e = 0; e < d; ++e) {
@@ -259,6 +282,7 @@ static void backward_seq(const seq_job* J)
                     R[(size_t)f * d + e] += PQ[(size_t)j * D + f] * g[(size_t)j * d + e];
             }
         const double* vj = J->v + (size_t)j * d;
+        const double* kj = J->k + (size_t)j * d;
         const double* pk = PK + (size_t)j * D;
         for (int f = 0; f < D; ++f) dphi[f] = r[f] + dot(d, R + (size_t)f * d, vj);
         for (int e = 0; e < d; ++e) {
@@ -266,10 +290,14 @@ static void backward_seq(const seq_job* J)
             for (int f = 0; f < D; ++f) s += R[(size_t)f * d + e] * pk[f];
             J->dv[(size_t)j * d + e] = s;
         }
-        feature_backward(d, M, J->k + (size_t)j * d, J->W1, J->W2, dphi, J->dk + (size_t)j * d,
-                         J->dA, J->dB);
+        /* dphi is the gradient with respect to phi~(k_j); dw_j = phi(k_j) . dphi. */
+        const double dw = dot(D, pk, dphi) / wk[j];
+        for (int f = 0; f < D; ++f) dphi[f] *= wk[j];
+        feature_backward(d, M, kj, J->W1, J->W2, dphi, J->dk + (size_t)j * d, J->dA, J->dB);
+        for (int e = 0; e < d; ++e) J->dk[(size_t)j * d + e] += dw * wk[j] * 2.0 * J->itau * kj[e];
+        if (J->dtau) *J->dtau += -dw * wk[j] * dot(d, kj, kj) * J->itau;
     }
-    free(out); free(den); free(PQ); free(PK); free(g); free(cc);
+    free(out); free(den); free(PQ); free(PK); free(wk); free(g); free(cc);
     free(S); free(z); free(dphi);
 }
 
@@ -347,8 +375,8 @@ int oracle_featmap_sumform(int B, int H, int N, int d, int M, const double* x,
 }
 
 int oracle_linattn_fwd(int B, int H, int N, int d, int M, const double* q, const double* k,
-                       const double* v, const double* W1, const double* W2, int causal,
-                       double* out, double* den, int nthreads)
+                       const double* v, const double* W1, const double* W2,
+                       const double* tau, int causal, double* out, double* den, int nthreads)
 {
     if (bad_shape(B, H, N, d, M)) return -1;
     seq_job* jobs = calloc((size_t)B * H, sizeof(seq_job));
@@ -358,24 +386,26 @@ int oracle_linattn_fwd(int B, int H, int N, int d, int M, const double* q, const
             jobs[u] = (seq_job){N, d, M, causal, q + off, k + off, v + off,
                                 W1 + (size_t)h * M * d, W2 ? W2 + (size_t)h * M * d : NULL,
                                 NULL, out + off, den ? den + u * N : NULL,
-                                NULL, NULL, NULL, NULL, NULL};
+                                NULL, NULL, NULL, NULL, NULL, tau ? exp(-tau[h]) : 0.0, NULL};
         }
     run_jobs(jobs, B * H, nthreads, 0);
     free(jobs);
     return 0;
 }
 
-/* dW1 (and dW2) are sums over the batch and the sequence; they are overwritten. */
+/* dW1 (and dW2, dtau) are sums over the batch and the sequence; they are overwritten. */
 int oracle_linattn_bwd(int B, int H, int N, int d, int M, const double* q, const double* k,
-                       const double* v, const double* W1, const double* W2, int causal,
-                       const double* dout, double* dq, double* dk, double* dv, double* dW1,
-                       double* dW2, int nthreads)
+                       const double* v, const double* W1, const double* W2,
+                       const double* tau, int causal, const double* dout, double* dq,
+                       double* dk, double* dv, double* dW1, double* dW2, double* dtau,
+                       int nthreads)
 {
     if (bad_shape(B, H, N, d, M)) return -1;
-    if ((W2 == NULL) != (dW2 == NULL)) return -1;
+    if ((W2 == NULL) != (dW2 == NULL) || (tau == NULL) != (dtau == NULL)) return -1;
     const size_t per = (size_t)M * d;
     double* dA = calloc((size_t)B * H * per, sizeof(double));
     double* dB = calloc((size_t)B * H * per, sizeof(double));
+    double* dt = calloc((size_t)B * H, sizeof(double));
     seq_job* jobs = calloc((size_t)B * H, sizeof(seq_job));
     for (int b = 0; b < B; ++b)
         for (int h = 0; h < H; ++h) {
@@ -385,7 +415,8 @@ int oracle_linattn_bwd(int B, int H, int N, int d, int M, const double* q, const
             jobs[u] = (seq_job){N, d, M, causal, q + off, k + off, v + off,
                                 W1 + (size_t)h * per, W2 ? W2 + (size_t)h * per : NULL,
                                 dout + off, NULL, NULL, dq + off, dk + off, dv + off,
-                                dA + u * per, dB + u * per};
+                                dA + u * per, dB + u * per, tau ? exp(-tau[h]) : 0.0,
+                                tau ? dt + u : NULL};
         }
     run_jobs(jobs, B * H, nthreads, 1);
     /* Sum the per-sequence parameter gradients over the batch in a fixed order. */
@@ -404,17 +435,24 @@ int oracle_linattn_bwd(int B, int H, int N, int d, int M, const double* q, const
                 dW2[h * per + t] = 0.5 * (a - bb);
             }
         }
-    free(dA); free(dB); free(jobs);
+    if (dtau)
+        for (int h = 0; h < H; ++h) {
+            double a = 0.0;
+            for (int b = 0; b < B; ++b) a += dt[(size_t)b * H + h];
+            dtau[h] = a;
+        }
+    free(dA); free(dB); free(dt); free(jobs);
     return 0;
 }
 
 /* One step of the causal recurrence behind Eq. (linear att) with j <= i: the running sums
  * S = sum_j phi(k_j) v_j^T and z = sum_j phi(k_j) absorb the new token (inclusive), then
  * out = phi(q)^T S / den with den = phi(q)^T z.  Per (b, h): q, k, v, out [d]; S [2M][d]
- * and z [2M] are updated in place; den [1]. */
+ * and z [2M] are updated in place; den [1].  With tau, the new key's phi carries its
+ * weight w = exp(|k|^2 exp(-tau)) as in the forward. */
 int oracle_linattn_decode(int B, int H, int d, int M, const double* q, const double* k,
-                          const double* v, const double* W1, const double* W2, double* S,
-                          double* z, double* out, double* den)
+                          const double* v, const double* W1, const double* W2,
+                          const double* tau, double* S, double* z, double* out, double* den)
 {
     if (bad_shape(B, H, 1, d, M)) return -1;
     const int F = 2 * M;
@@ -427,6 +465,8 @@ int oracle_linattn_decode(int B, int H, int d, int M, const double* q, const dou
             const double* w2 = W2 ? W2 + (size_t)h * M * d : NULL;
             feature(d, M, q + u * d, w1, w2, pq);
             feature(d, M, k + u * d, w1, w2, pk);
+            const double wk = key_weight(d, k + u * d, tau ? exp(-tau[h]) : 0.0);
+            for (int f = 0; f < F; ++f) pk[f] *= wk;
             double* Su = S + u * F * d;
             double* zu = z + u * F;
             for (int f = 0; f < F; ++f) {

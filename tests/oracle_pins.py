@@ -24,6 +24,11 @@ Facts used (none is the oracle's own formula retyped):
     sum_j dv_j = sum_i dO_i, translation invariance of the stationary kernel
     (sum dq + sum dk = 0) and Euler's identity for a = W x
     (<dW1, W1> + <dW2, W2> = sum <dq, q> + sum <dk, k>).
+  * the norm prefactor exp(|x|^2 / exp(tau)) (Sec. 3.2): the linear form with the key
+    weight equals the N x N form with the factor on queries and keys as printed; it
+    vanishes as tau grows; keys of equal norm make it a common factor (O unchanged);
+    finite differences (dq, dk, dv, dW, dtau); the scaling identity
+    <dW, W> = sum <dq, q> + <dk, k> + 2 dtau (x -> l x, W -> W / l, tau -> tau + 2 ln l).
 """
 from __future__ import annotations
 
@@ -215,10 +220,118 @@ def pin_gradient_invariants(orc):
                 assert np.all(np.abs(t) < 1e-11 * scale), "translation invariance"
 
 
+# -------------------------------------------------------------------------------------
+# The norm prefactor of Sec. 3.2: phi~(x) = exp(|x|^2 / exp(tau)) phi(x), tau per head.
+# The numpy N x N form applies it literally to queries and keys; the C linear form keeps
+# only the key weight (the query factor cancels row by row).
+# -------------------------------------------------------------------------------------
+_TAU = np.array([1.0, 2.5])
+
+
+def _qfactor(q, tau):
+    return np.exp(np.sum(q * q, axis=-1) / np.exp(tau)[:, None])
+
+
+def pin_prefactor_linear_equals_brute(orc):
+    for variant in ("s", "n"):
+        for causal in (True, False):
+            for N in (1, 3, 17, 64):
+                q, k, v, W1, W2 = _case(50 + N, 2, 2, N, 5, 7, variant)
+                out, den = orc.fwd(q, k, v, W1, W2, causal, tau=_TAU)
+                bo, bd = brute.attention(q, k, v, W1, W2, causal, tau=_TAU)
+                assert _rel(out, bo) < 1e-11, f"prefactor out {variant} causal={causal} N={N}"
+                assert _rel(den * _qfactor(q, _TAU), bd) < 1e-12, f"prefactor den {variant}"
+
+
+def pin_prefactor_vanishes_as_tau_grows(orc):
+    """exp(-tau) -> 0: the weights tend to 1 (tau = 80 makes them 1 in fp64)."""
+    for variant in ("s", "n"):
+        q, k, v, W1, W2 = _case(60, 2, 2, 11, 5, 7, variant)
+        o0, d0 = orc.fwd(q, k, v, W1, W2, True)
+        o1, d1 = orc.fwd(q, k, v, W1, W2, True, tau=np.array([80.0, 80.0]))
+        assert np.array_equal(o0, o1) and np.array_equal(d0, d1), "tau -> inf limit"
+
+
+def pin_prefactor_equal_key_norms(orc):
+    """Keys of one norm r: every weight is exp(r^2 exp(-tau)), a common factor, so O is
+    the output without the prefactor and den is that factor times its den."""
+    for variant in ("s", "n"):
+        for causal in (True, False):
+            q, k, v, W1, W2 = _case(61, 2, 2, 13, 5, 7, variant)
+            k = k / np.linalg.norm(k, axis=-1, keepdims=True) * 1.3
+            o0, d0 = orc.fwd(q, k, v, W1, W2, causal)
+            o1, d1 = orc.fwd(q, k, v, W1, W2, causal, tau=_TAU)
+            w = np.exp(1.3 ** 2 / np.exp(_TAU))[None, :, None]
+            assert _rel(o1, o0) < 1e-13, "equal key norms: O changed"
+            assert _rel(d1, w * d0) < 1e-13, "equal key norms: den not scaled"
+
+
+def _loss_tau(q, k, v, W1, W2, causal, dO, tau):
+    return float(np.sum(brute.attention(q, k, v, W1, W2, causal, tau=tau)[0] * dO))
+
+
+def pin_prefactor_finite_differences(orc):
+    h = 1e-6
+    for variant in ("s", "n"):
+        for causal in (True, False):
+            q, k, v, W1, W2 = _case(62, 2, 2, 5, 3, 4, variant)
+            tau = _TAU.copy()
+            dO = _rng(63).standard_normal(q.shape)
+            grads = orc.bwd(q, k, v, W1, W2, causal, dO, tau=tau)
+            params = [q, k, v, W1] + ([W2] if W2 is not None else [])
+            pg = list(zip(params, grads[:len(params)])) + [(tau, grads[5])]
+            for idx, (p, gp) in enumerate(pg):
+                fd = np.zeros_like(p)
+                it = np.nditer(p, flags=["multi_index"])
+                for _ in it:
+                    mi = it.multi_index
+                    old = p[mi]
+                    p[mi] = old + h
+                    lp = _loss_tau(q, k, v, W1, W2, causal, dO, tau)
+                    p[mi] = old - h
+                    lm = _loss_tau(q, k, v, W1, W2, causal, dO, tau)
+                    p[mi] = old
+                    fd[mi] = (lp - lm) / (2 * h)
+                err = np.linalg.norm(gp - fd) / np.linalg.norm(fd)
+                assert err < 1e-6, f"prefactor FD {variant} causal={causal} #{idx}: {err:.2e}"
+
+
+def pin_prefactor_scaling_identity(orc):
+    """x -> l x, W -> W / l, tau -> tau + 2 ln l leaves every output unchanged, so per head
+    <dW1, W1> + <dW2, W2> = sum <dq, q> + <dk, k> + 2 dtau; rows of weights still sum to 1."""
+    for variant in ("s", "n"):
+        for causal in (True, False):
+            q, k, v, W1, W2 = _case(64, 2, 2, 19, 5, 7, variant)
+            dO = _rng(65).standard_normal(q.shape)
+            dq, dk, dv, dW1, dW2, dtau = orc.bwd(q, k, v, W1, W2, causal, dO, tau=_TAU)
+            assert _rel(dv.sum(axis=2), dO.sum(axis=2)) < 1e-11, "prefactor: sum dv != sum dO"
+            lhs = np.sum(dW1 * W1, axis=(1, 2))
+            if W2 is not None:
+                lhs = lhs + np.sum(dW2 * W2, axis=(1, 2))
+            rhs = np.sum(dq * q, axis=(0, 2, 3)) + np.sum(dk * k, axis=(0, 2, 3)) + 2 * dtau
+            assert np.all(np.abs(lhs - rhs) < 1e-10 * np.maximum(np.abs(rhs), 1.0)), \
+                "prefactor scaling identity"
+
+
+def pin_prefactor_decode(orc):
+    for variant in ("s", "n"):
+        B, H, N, d, M = 2, 2, 9, 5, 7
+        q, k, v, W1, W2 = _case(66, B, H, N, d, M, variant)
+        bo, _ = brute.attention(q, k, v, W1, W2, True, tau=_TAU)
+        S = np.zeros((B, H, 2 * M, d))
+        z = np.zeros((B, H, 2 * M))
+        for i in range(N):
+            out, _, S, z = orc.decode(q[:, :, i], k[:, :, i], v[:, :, i], W1, W2, S, z,
+                                      tau=_TAU)
+            assert _rel(out, bo[:, :, i]) < 1e-11, f"prefactor decode {variant} i={i}"
+
+
 ALL_PINS = [
     pin_origin_features, pin_stationary_unit_norm, pin_sum_to_product, pin_w2_equals_w1,
     pin_bochner, pin_yaglom, pin_linear_equals_brute, pin_decode_equals_brute,
     pin_closed_form_d1,
     pin_causal_last_equals_noncausal, pin_first_and_constant, pin_finite_differences,
-    pin_gradient_invariants,
+    pin_gradient_invariants, pin_prefactor_linear_equals_brute,
+    pin_prefactor_vanishes_as_tau_grows, pin_prefactor_equal_key_norms,
+    pin_prefactor_finite_differences, pin_prefactor_scaling_identity, pin_prefactor_decode,
 ]

@@ -42,6 +42,17 @@ MUTATIONS = [
     ("decode_drops_new_value", "Su[(size_t)f * d + e] += pk[f] * v[u * d + e];",
      "Su[(size_t)f * d + e] += 0.0 * v[u * d + e];", 0),
     ("decode_forgets_z_update", "zu[f] += pk[f];", "zu[f] += 0.0;", 0),
+    ("prefactor_sign_of_exponent", "return exp(dot(d, k, k) * itau);",
+     "return exp(-dot(d, k, k) * itau);", 0),
+    ("prefactor_dk_without_2", "dw * wk[j] * 2.0 * J->itau * kj[e];",
+     "dw * wk[j] * J->itau * kj[e];", 0),
+    ("prefactor_dtau_sign", "*J->dtau += -dw * wk[j]", "*J->dtau += dw * wk[j]", 0),
+    ("prefactor_dphi_unweighted", "for (int f = 0; f < D; ++f) dphi[f] *= wk[j];",
+     "for (int f = 0; f < D; ++f) dphi[f] *= 1.0;", 0),
+    ("prefactor_decode_unweighted", "for (int f = 0; f < F; ++f) pk[f] *= wk;",
+     "for (int f = 0; f < F; ++f) pk[f] *= 1.0;", 0),
+    ("prefactor_noncausal_unweighted", "for (int f = 0; f < D; ++f) pk[f] *= wj;",
+     "for (int f = 0; f < D; ++f) pk[f] *= 1.0;", 0),
 ]
 
 
