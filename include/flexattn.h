@@ -80,11 +80,16 @@ int flex_featmap(const flex_shape* shape, const void* x, const float* W1, const 
                  void* phi, void* stream);
 
 /* Forward linear attention, Eq. (linear att) with the feature map above.
- * out: [B][H][N][d] in shape->dtype.  den: NULL, or [B][H][N] fp32 receiving den_i
- * (needed by flex_linattn_bwd).  ws: workspace of ws_bytes bytes. */
+ * tau: NULL, or [H] fp32: the norm prefactor of Sec. 3.2, phi~(x) = exp(|x|^2 / exp(tau_h))
+ * phi(x) on queries and keys.  The query's factor cancels in every row, so only the key
+ * weight w_j = exp(|k_j|^2 exp(-tau_h)) is applied (to k_j's share of both sums); the
+ * weight overflows fp32 when |k_j|^2 exp(-tau_h) > 88.
+ * out: [B][H][N][d] in shape->dtype.  den: NULL, or [B][H][N] fp32 receiving
+ * den_i = phi(q_i)^T sum_j w_j phi(k_j) (w_j = 1 without tau; the query's factor is not
+ * included), needed by flex_linattn_bwd.  ws: workspace of ws_bytes bytes. */
 int flex_linattn_fwd(const flex_shape* shape, const void* q, const void* k, const void* v,
-                     const float* W1, const float* W2, int causal, void* out, float* den,
-                     void* ws, size_t ws_bytes, void* stream);
+                     const float* W1, const float* W2, const float* tau, int causal,
+                     void* out, float* den, void* ws, size_t ws_bytes, void* stream);
 
 /* Backward of flex_linattn_fwd: gradients of L = sum(dout * out) with respect to q, k,
  * v and the frequencies.  out and den are the forward's outputs for the same inputs.
@@ -95,21 +100,27 @@ int flex_linattn_fwd(const flex_shape* shape, const void* q, const void* k, cons
  *   dphi(q_i) = S_i g_i + c_i z_i,  dphi(k_j) = R_j v_j + r_j,  dv_j = R_j^T phi(k_j),
  *   R_j = sum_{i >= j} phi(q_i) g_i^T,  r_j = sum_{i >= j} c_i phi(q_i)
  * (totals when non-causal), then through the feature map by the chain rule; for the
- * nonstationary variant dW1 = (dU + dV)/2 and dW2 = (dU - dV)/2. */
+ * nonstationary variant dW1 = (dU + dV)/2 and dW2 = (dU - dV)/2.  With tau (dtau [H]
+ * fp32, NULL exactly when tau is): the formulas hold for the weighted key features
+ * w_j phi(k_j); dv_j is multiplied by w_j, and with s_j = phi(k_j) . dphi(k_j) (the
+ * gradient with respect to the unweighted features) dk_j gains 2 exp(-tau) s_j k_j and
+ * dtau_h = -sum exp(-tau_h) |k_j|^2 s_j over the batch and the sequence (overwritten). */
 int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, const void* v,
-                     const float* W1, const float* W2, int causal, const void* out,
-                     const float* den, const void* dout, void* dq, void* dk, void* dv,
-                     float* dW1, float* dW2, void* ws, size_t ws_bytes, void* stream);
+                     const float* W1, const float* W2, const float* tau, int causal,
+                     const void* out, const float* den, const void* dout, void* dq,
+                     void* dk, void* dv, float* dW1, float* dW2, float* dtau, void* ws,
+                     size_t ws_bytes, void* stream);
 
 /* flex_linattn_bwd without a workspace, for callers that cannot allocate device memory:
  * for example a host framework whose memory pool owns all of the device's memory and
  * passes its operators only input and output pointers, or a latency-critical path that
  * must not call cudaMalloc/cudaFree, which can synchronise the device.  (The paper has
  * no counterpart; this is a convenience of this library.)
- * Same arguments, layouts and results as flex_linattn_bwd, minus ws and ws_bytes.  The
+ * Same arguments, layouts and results as flex_linattn_bwd without the norm prefactor,
+ * minus tau, dtau, ws and ws_bytes.  The
  * scratch is one array of 4 MiB (2^20 floats) in the library's own device memory, which
  * every GPU that loads the library keeps until the process exits; it must hold
- * B * H * Mc * d floats (Mc = M, or 2M when W2 is given), else FLEX_EWORKSPACE is
+ * B * H * (Mc * d + 1) floats (Mc = M, or 2M when W2 is given), else FLEX_EWORKSPACE is
  * returned and nothing runs.  Nothing is allocated or freed.  All calls on a device
  * share that array and it keeps the last call's contents, so two calls whose work may
  * overlap on the GPU (different streams, or different host threads) race and must be
@@ -132,13 +143,15 @@ size_t flex_decode_workspace_bytes(const flex_shape* shape);
  * (zero-filled before a sequence's first token); phi is scaled by M^{-1/2} as in Eq. phi_n
  * / phi_non, so S and z are exactly the paper's running sums.  out: [B][H][d] in
  * shape->dtype; den: NULL or [B][H] fp32.  Stepping through a sequence reproduces
- * flex_linattn_fwd(causal = 1) row by row.  ws: workspace of at least
+ * flex_linattn_fwd(causal = 1) row by row (with the same tau: the new key's features
+ * enter S and z with its weight w).  ws: workspace of at least
  * flex_decode_workspace_bytes() bytes (it holds the step's phi(q), phi(k); a serving loop
  * allocates it once).  Two kernels per call.  Errors: FLEX_EINVAL for NULL or misaligned
  * pointers or N != 1, FLEX_EWORKSPACE, FLEX_EUNSUPPORTED as for the other entry points. */
 int flex_linattn_decode(const flex_shape* shape, const void* q, const void* k, const void* v,
-                        const float* W1, const float* W2, float* S, float* z, void* out,
-                        float* den, void* ws, size_t ws_bytes, void* stream);
+                        const float* W1, const float* W2, const float* tau, float* S,
+                        float* z, void* out, float* den, void* ws, size_t ws_bytes,
+                        void* stream);
 
 /* Cumulative number of kernels this library has enqueued in this process (all entry
  * points, all devices).  Lets a caller count the launches inside a timed region. */

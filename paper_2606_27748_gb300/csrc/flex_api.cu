@@ -103,8 +103,8 @@ int flex_featmap(const flex_shape* shape, const void* x, const float* W1, const 
 }
 
 int flex_linattn_fwd(const flex_shape* shape, const void* q, const void* k, const void* v,
-                     const float* W1, const float* W2, int causal, void* out, float* den,
-                     void* ws, size_t ws_bytes, void* stream)
+                     const float* W1, const float* W2, const float* tau, int causal, void* out,
+                     float* den, void* ws, size_t ws_bytes, void* stream)
 {
     Problem p;
     int rc = make_problem(shape, W2, causal, &p);
@@ -112,30 +112,34 @@ int flex_linattn_fwd(const flex_shape* shape, const void* q, const void* k, cons
     if (!q || !k || !v || !W1 || !out) return FLEX_EINVAL;
     for (const void* t : {q, k, v, (const void*)W1, (const void*)out})
         if (!aligned(t, 16)) return FLEX_EINVAL;
-    if ((W2 && !aligned(W2, 16)) || (den && !aligned(den, 16))) return FLEX_EINVAL;
+    if ((W2 && !aligned(W2, 16)) || (den && !aligned(den, 16)) || (tau && !aligned(tau, 4)))
+        return FLEX_EINVAL;
     if ((rc = check_ws(ws, ws_bytes, fwd_ws_bytes(p)))) return rc;
     cudaStream_t s = (cudaStream_t)stream;
     int* status = &((flex::WsHeader*)ws)->status;
-    if (flex::tc_fwd_supported(p))
+    if (!tau && flex::tc_fwd_supported(p))
         return count(1, flex::launch_tc_fwd(p, q, k, v, W1, W2, out, den, status, s));
-    if (flex::tc_nc_supported(p))
+    if (!tau && flex::tc_nc_supported(p))
         return count(3, flex::launch_tc_nc(p, q, k, v, W1, W2, out, den,
                                            (char*)ws + header_bytes(), status, s));
     if (flex::simt_pick_chunk_fwd(p) == 0) return FLEX_EUNSUPPORTED;
-    return count(1, flex::launch_simt_fwd(p, q, k, v, W1, W2, out, den, s));
+    return count(1, flex::launch_simt_fwd(p, q, k, v, W1, W2, tau, out, den, s));
 }
 
 int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, const void* v,
-                     const float* W1, const float* W2, int causal, const void* out,
-                     const float* den, const void* dout, void* dq, void* dk, void* dv,
-                     float* dW1, float* dW2, void* ws, size_t ws_bytes, void* stream)
+                     const float* W1, const float* W2, const float* tau, int causal,
+                     const void* out, const float* den, const void* dout, void* dq, void* dk,
+                     void* dv, float* dW1, float* dW2, float* dtau, void* ws, size_t ws_bytes,
+                     void* stream)
 {
     Problem p;
     int rc = make_problem(shape, W2, causal, &p);
     if (rc) return rc;
     if (!q || !k || !v || !W1 || !out || !den || !dout || !dq || !dk || !dv || !dW1)
         return FLEX_EINVAL;
-    if ((W2 == nullptr) != (dW2 == nullptr)) return FLEX_EINVAL;
+    if ((W2 == nullptr) != (dW2 == nullptr) || (tau == nullptr) != (dtau == nullptr))
+        return FLEX_EINVAL;
+    if ((tau && !aligned(tau, 4)) || (dtau && !aligned(dtau, 4))) return FLEX_EINVAL;
     for (const void* t : {q, k, v, (const void*)W1, out, (const void*)den, dout, (const void*)dq,
                           (const void*)dk, (const void*)dv, (const void*)dW1})
         if (!aligned(t, 16)) return FLEX_EINVAL;
@@ -143,12 +147,12 @@ int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, cons
     if ((rc = check_ws(ws, ws_bytes, bwd_ws_bytes(p)))) return rc;
     cudaStream_t s = (cudaStream_t)stream;
     void* scratch = (char*)ws + header_bytes();
-    if (flex::tc_bwd_supported(p))
+    if (!tau && flex::tc_bwd_supported(p))
         return count(3, flex::launch_tc_bwd(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1,
                                             dW2, scratch, &((flex::WsHeader*)ws)->status, s));
     if (flex::simt_pick_chunk_bwd(p) == 0) return FLEX_EUNSUPPORTED;
-    return count(2, flex::launch_simt_bwd(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1,
-                                          dW2, scratch, s));
+    return count(2, flex::launch_simt_bwd(p, q, k, v, W1, W2, tau, out, den, dout, dq, dk, dv,
+                                          dW1, dW2, dtau, scratch, s));
 }
 
 size_t flex_decode_workspace_bytes(const flex_shape* shape)
@@ -159,8 +163,8 @@ size_t flex_decode_workspace_bytes(const flex_shape* shape)
 }
 
 int flex_linattn_decode(const flex_shape* shape, const void* q, const void* k, const void* v,
-                        const float* W1, const float* W2, float* S, float* z, void* out,
-                        float* den, void* ws, size_t ws_bytes, void* stream)
+                        const float* W1, const float* W2, const float* tau, float* S, float* z,
+                        void* out, float* den, void* ws, size_t ws_bytes, void* stream)
 {
     Problem p;
     int rc = make_problem(shape, W2, 1, &p);
@@ -169,9 +173,10 @@ int flex_linattn_decode(const flex_shape* shape, const void* q, const void* k, c
     if (!q || !k || !v || !W1 || !S || !z || !out) return FLEX_EINVAL;
     for (const void* t : {q, k, v, (const void*)W1, (const void*)S, (const void*)z, (const void*)out})
         if (!aligned(t, 16)) return FLEX_EINVAL;
-    if ((W2 && !aligned(W2, 16)) || (den && !aligned(den, 16))) return FLEX_EINVAL;
+    if ((W2 && !aligned(W2, 16)) || (den && !aligned(den, 16)) || (tau && !aligned(tau, 4)))
+        return FLEX_EINVAL;
     if ((rc = check_ws(ws, ws_bytes, header_bytes() + flex::decode_ws_bytes(p)))) return rc;
-    return count(2, flex::launch_decode(p, q, k, v, W1, W2, S, z, out, den,
+    return count(2, flex::launch_decode(p, q, k, v, W1, W2, tau, S, z, out, den,
                                         (char*)ws + header_bytes(), (cudaStream_t)stream));
 }
 

@@ -13,7 +13,8 @@
 //                    per-token kernel; phi(q), phi(k) (Eq. phi_n, or the product form of
 //                    Eq. phi_non with u = (W1+W2)/2 x and w = (W1-W2)/2 x formed from the
 //                    two dot products; scaled by M^{-1/2}; fp32, sin/cos after a
-//                    reduction by 2 pi) go to the workspace;
+//                    reduction by 2 pi; phi(k) times the key weight exp(|k|^2 exp(-tau))
+//                    of the norm prefactor when tau is given) go to the workspace;
 //   decode_state     one CTA of 256 threads per (b, h), three per SM: starts asynchronous
 //                    16-byte copies of S (up to 64 KB of rows) into shared memory and the
 //                    loads of z, THEN waits for the features (programmatic dependent
@@ -85,7 +86,8 @@ template <typename T, bool NS, int D4C>
 __global__ void __launch_bounds__(kThreadsF, 4)
     decode_features(int B, int H, int d, int M, const T* __restrict__ q,
                     const T* __restrict__ k, const float* __restrict__ W1,
-                    const float* __restrict__ W2, float* __restrict__ phi)
+                    const float* __restrict__ W2, const float* __restrict__ tau,
+                    float* __restrict__ phi)
 {
     // The state kernel may launch now; it waits for this grid before reading phi.
     asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
@@ -96,6 +98,7 @@ __global__ void __launch_bounds__(kThreadsF, 4)
     float* w1s = reinterpret_cast<float*>(fsm4);  // [kTF][ld]: W1 rows of the tile
     float* w2s = w1s + kTF * ld;                  // [kTF][ld]: W2 rows (n only)
     float* xs = w2s + (NS ? kTF * ld : 0);        // [2 kG][d]: token vector t = 2 s + which
+    float* kw = xs + 2 * kG * (D4C ? 4 * D4C : d); // [2 kG]: key weights (norm prefactor)
     const int tiles = (M + kTF - 1) / kTF, groups = (B + kG - 1) / kG;
     const int tile = blockIdx.x % tiles, grp = (blockIdx.x / tiles) % groups;
     const int h = blockIdx.x / (tiles * groups);
@@ -138,6 +141,14 @@ __global__ void __launch_bounds__(kThreadsF, 4)
             if (lane + 32 * i < dd) xs[(warp + j * kWarps) * dd + lane + 32 * i] = xr[j][i];
     cp_async_wait_all();
     __syncthreads();
+    if (tau) {  // key weight of the norm prefactor (Sec. 3.2): exp(|k|^2 exp(-tau))
+        if (tid < 2 * kG) {
+            float n2 = 0.f;
+            for (int e = 0; e < dd; ++e) n2 = fmaf(xs[tid * dd + e], xs[tid * dd + e], n2);
+            kw[tid] = expf(n2 * expf(-tau[h]));
+        }
+        __syncthreads();
+    }
 
     float a[kTokW], c[kTokW];
 #pragma unroll
@@ -168,6 +179,7 @@ __global__ void __launch_bounds__(kThreadsF, 4)
             sincos_reduced(NS ? 0.5f * (a[j] + c[j]) : a[j], &su, &cu);
             if (NS) sincos_reduced(0.5f * (a[j] - c[j]), &sw, &cw);
             cw *= scale;
+            if (tau && (t & 1)) cw *= kw[t];  // phi(k) carries its weight into S and z
             float* dst = phi + (((size_t)(b0 + t / 2) * H + h) * 2 + (t & 1)) * F;
             dst[f] = cu * cw;
             dst[M + f] = su * cw;
@@ -271,14 +283,14 @@ __global__ void __launch_bounds__(kThreadsD, 3)
 
 template <typename T, bool NS>
 cudaError_t launch_typed(const Problem& p, const void* q, const void* k, const void* v,
-                         const float* W1, const float* W2, float* S, float* z, void* out,
-                         float* den, float* phi, cudaStream_t s)
+                         const float* W1, const float* W2, const float* tau, float* S,
+                         float* z, void* out, float* den, float* phi, cudaStream_t s)
 {
     const long long fctas = (long long)p.H * ((p.B + kG - 1) / kG) * ((p.M + kTF - 1) / kTF);
     const long long sctas = (long long)p.B * p.H;
     if (fctas > 0x7fffffffLL || sctas > 0x7fffffffLL) return cudaErrorInvalidValue;
 
-    const size_t fsmem = ((size_t)kTF * (p.d + 4) * 2 + 2 * kG * p.d) * sizeof(float);
+    const size_t fsmem = ((size_t)kTF * (p.d + 4) * 2 + 2 * kG * p.d + 2 * kG) * sizeof(float);
     auto fk = p.d == 32    ? decode_features<T, NS, 8>
               : p.d == 64  ? decode_features<T, NS, 16>
               : p.d == 128 ? decode_features<T, NS, 32>
@@ -286,7 +298,7 @@ cudaError_t launch_typed(const Problem& p, const void* q, const void* k, const v
     cudaError_t e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fsmem);
     if (e != cudaSuccess) return e;
     fk<<<(unsigned)fctas, kThreadsF, fsmem, s>>>(p.B, p.H, p.d, p.M, (const T*)q, (const T*)k,
-                                                W1, W2, phi);
+                                                W1, W2, tau, phi);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
     const size_t ssmem = (size_t)std::min(2 * p.M, kSBuf / p.d) * p.d * sizeof(float);
@@ -313,16 +325,17 @@ cudaError_t launch_typed(const Problem& p, const void* q, const void* k, const v
 size_t decode_ws_bytes(const Problem& p) { return (size_t)p.B * p.H * 2 * 2 * p.M * sizeof(float); }
 
 cudaError_t launch_decode(const Problem& p, const void* q, const void* k, const void* v,
-                          const float* W1, const float* W2, float* S, float* z, void* out,
-                          float* den, void* scratch, cudaStream_t s)
+                          const float* W1, const float* W2, const float* tau, float* S,
+                          float* z, void* out, float* den, void* scratch, cudaStream_t s)
 {
     float* phi = (float*)scratch;
     if (p.bf16)
-        return p.nonstat
-                   ? launch_typed<__nv_bfloat16, true>(p, q, k, v, W1, W2, S, z, out, den, phi, s)
-                   : launch_typed<__nv_bfloat16, false>(p, q, k, v, W1, W2, S, z, out, den, phi, s);
-    return p.nonstat ? launch_typed<float, true>(p, q, k, v, W1, W2, S, z, out, den, phi, s)
-                     : launch_typed<float, false>(p, q, k, v, W1, W2, S, z, out, den, phi, s);
+        return p.nonstat ? launch_typed<__nv_bfloat16, true>(p, q, k, v, W1, W2, tau, S, z, out,
+                                                             den, phi, s)
+                         : launch_typed<__nv_bfloat16, false>(p, q, k, v, W1, W2, tau, S, z,
+                                                              out, den, phi, s);
+    return p.nonstat ? launch_typed<float, true>(p, q, k, v, W1, W2, tau, S, z, out, den, phi, s)
+                     : launch_typed<float, false>(p, q, k, v, W1, W2, tau, S, z, out, den, phi, s);
 }
 
 }  // namespace flex

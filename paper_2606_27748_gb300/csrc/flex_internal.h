@@ -38,19 +38,21 @@ size_t simt_bwd_ws_bytes(const Problem& p);
 
 cudaError_t launch_featmap(const Problem& p, const void* x, const float* W1, const float* W2,
                            void* phi, cudaStream_t s);
+// tau: per-head norm prefactor (Sec. 3.2) or NULL; dtau with it in the backward.
 cudaError_t launch_simt_fwd(const Problem& p, const void* q, const void* k, const void* v,
-                            const float* W1, const float* W2, void* out, float* den,
-                            cudaStream_t s);
+                            const float* W1, const float* W2, const float* tau, void* out,
+                            float* den, cudaStream_t s);
 cudaError_t launch_simt_bwd(const Problem& p, const void* q, const void* k, const void* v,
-                            const float* W1, const float* W2, const void* out,
-                            const float* den, const void* dout, void* dq, void* dk, void* dv,
-                            float* dW1, float* dW2, void* scratch, cudaStream_t s);
+                            const float* W1, const float* W2, const float* tau,
+                            const void* out, const float* den, const void* dout, void* dq,
+                            void* dk, void* dv, float* dW1, float* dW2, float* dtau,
+                            void* scratch, cudaStream_t s);
 
 // ---- recurrent decode step (one token per sequence; fp32 state) ----------------------
 size_t decode_ws_bytes(const Problem& p);  // phi(q), phi(k) of the step, fp32
 cudaError_t launch_decode(const Problem& p, const void* q, const void* k, const void* v,
-                          const float* W1, const float* W2, float* S, float* z, void* out,
-                          float* den, void* scratch, cudaStream_t s);
+                          const float* W1, const float* W2, const float* tau, float* S,
+                          float* z, void* out, float* den, void* scratch, cudaStream_t s);
 
 // ---- tensor-core path (bf16 storage, d = 64, M in {64, 128}) ------------------------
 bool tc_fwd_supported(const Problem& p);

@@ -75,7 +75,7 @@ extern "C" int flex_linattn_bwd_noalloc(const flex_shape* shape, const void* q, 
     if (rc != FLEX_OK) return rc;
     // Every partial slot the reduction reads is written first by this call, so the
     // array's previous contents need no clearing.
-    cudaError_t e = flex::launch_simt_bwd(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1,
-                                          dW2, scratch, (cudaStream_t)stream);
+    cudaError_t e = flex::launch_simt_bwd(p, q, k, v, W1, W2, nullptr, out, den, dout, dq, dk,
+                                          dv, dW1, dW2, nullptr, scratch, (cudaStream_t)stream);
     return e == cudaSuccess ? FLEX_OK : FLEX_ECUDA;
 }

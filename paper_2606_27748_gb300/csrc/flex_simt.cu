@@ -10,6 +10,12 @@
 // Inside the attention kernels the features are unscaled, phi' = [cos, sin] (times cos w
 // for the nonstationary map): the global factor M^{-1/2} of Eq. phi_n / phi_non cancels in
 // out and in every gradient, and only the stored denominator is rescaled, den = den'/M.
+//
+// Norm prefactor (Sec. 3.2, optional, tau per head): phi~(x) = exp(|x|^2 / exp(tau)) phi(x).
+// The query's factor cancels row by row; the key's is a weight w_j, carried by turning the
+// key rows [v_j | 1] into [w_j v_j | w_j].  The backward then multiplies dv_j by w_j and,
+// with s_j = phi(k_j) . dphi(k_j), adds 2 exp(-tau) s_j k_j to dk_j and
+// -exp(-tau) |k_j|^2 s_j to dtau.
 #include "flex_internal.h"
 
 #include <math.h>
@@ -125,6 +131,18 @@ __global__ void featmap_kernel(Problem p, const T* x, const float* W1, const flo
 // ------------------------------------------------------------------------------------
 // Forward.
 // ------------------------------------------------------------------------------------
+// [v_j | 1] -> [w_j v_j | w_j] for the key rows of a chunk, w_j = exp(|k_j|^2 itau).
+__device__ void weight_keys(const float* Xk, int rows, int d, float itau, float* Vx)
+{
+    for (int j = threadIdx.x; j < rows; j += blockDim.x) {
+        float n2 = 0.f;
+        for (int e = 0; e < d; ++e) n2 = fmaf(Xk[j * d + e], Xk[j * d + e], n2);
+        const float w = expf(n2 * itau);
+        for (int e = 0; e < d; ++e) Vx[j * (d + 1) + e] *= w;
+        Vx[j * (d + 1) + d] = w;
+    }
+}
+
 struct FwdLayout {
     size_t W, S, Xq, Xk, Vx, Pq, Pk, A, O, total;  // offsets in floats
 };
@@ -163,7 +181,8 @@ template <typename T>
 __global__ void __launch_bounds__(kThreads) simt_fwd_kernel(Problem p, int C, const T* q,
                                                             const T* k, const T* v,
                                                             const float* W1, const float* W2,
-                                                            T* out, float* den)
+                                                            const float* tau, T* out,
+                                                            float* den)
 {
     extern __shared__ float sm[];
     const int d = p.d, D = 2 * p.M, N = p.N;
@@ -173,6 +192,7 @@ __global__ void __launch_bounds__(kThreads) simt_fwd_kernel(Problem p, int C, co
     float *W = sm + L.W, *S = sm + L.S, *Xq = sm + L.Xq, *Xk = sm + L.Xk, *Vx = sm + L.Vx;
     float *Pq = sm + L.Pq, *Pk = sm + L.Pk, *A = sm + L.A, *O = sm + L.O;
     const float inv_m = 1.0f / (float)p.M;
+    const float itau = tau ? expf(-tau[h]) : 0.f;
 
     load_projection(p, W1, W2, h, W);
     for (int idx = threadIdx.x; idx < D * (d + 1); idx += blockDim.x) S[idx] = 0.f;
@@ -185,6 +205,7 @@ __global__ void __launch_bounds__(kThreads) simt_fwd_kernel(Problem p, int C, co
             load_rows(k, base + (size_t)t0 * d, CL, d, Xk, d);
             load_rows(v, base + (size_t)t0 * d, CL, d, Vx, d + 1);
             __syncthreads();
+            if (tau) weight_keys(Xk, CL, d, itau, Vx);
             features(p, Xk, CL, W, Pk, D + 1);
             __syncthreads();
             state_update(Pk, Vx, CL, D, d, S);
@@ -199,6 +220,7 @@ __global__ void __launch_bounds__(kThreads) simt_fwd_kernel(Problem p, int C, co
             load_rows(v, base + (size_t)t0 * d, CL, d, Vx, d + 1);
         }
         __syncthreads();
+        if (tau && p.causal) weight_keys(Xk, CL, d, itau, Vx);
         features(p, Xq, CL, W, Pq, D + 1);
         if (p.causal) features(p, Xk, CL, W, Pk, D + 1);
         __syncthreads();
@@ -238,7 +260,7 @@ __global__ void __launch_bounds__(kThreads) simt_fwd_kernel(Problem p, int C, co
 // Backward.
 // ------------------------------------------------------------------------------------
 struct BwdLayout {
-    size_t W, S, Xq, Xk, Vx, Gx, Pq, Pk, dP, A, dA, dAct, total;
+    size_t W, S, Xq, Xk, Vx, Gx, Pq, Pk, dP, A, dA, dAct, Kc, total;
 };
 
 __host__ __device__ inline BwdLayout bwd_layout(const Problem& p, int C)
@@ -258,6 +280,7 @@ __host__ __device__ inline BwdLayout bwd_layout(const Problem& p, int C)
     L.A = o;    o += (size_t)C * C;
     L.dA = o;   o += (size_t)C * C;
     L.dAct = o; o += (size_t)C * (Mc + 1);
+    L.Kc = o;   o += (size_t)C;
     L.total = o;
     return L;
 }
@@ -310,16 +333,19 @@ __device__ void feature_backward(const Problem& p, const float* X, const float* 
     }
 }
 
-// dx[t][i] = sum_m dAct[t][m] W[m][i]; dW[m][i] += sum_t dAct[t][m] X[t][i].
+// dx[t][i] = sum_m dAct[t][m] W[m][i] (+ xcoef[t] X[t][i], the key prefactor's term);
+// dW[m][i] += sum_t dAct[t][m] X[t][i].
 template <typename T>
 __device__ void project_back(const Problem& p, const float* X, const float* dAct, int rows,
-                             const float* W, T* dx, size_t base, float* dw_acc)
+                             const float* W, T* dx, size_t base, float* dw_acc,
+                             const float* xcoef)
 {
     const int d = p.d, Mc = p.nonstat ? 2 * p.M : p.M;
     for (int idx = threadIdx.x; idx < rows * d; idx += blockDim.x) {
         int t = idx / d, i = idx % d;
         float acc = 0.f;
         for (int m = 0; m < Mc; ++m) acc = fmaf(dAct[t * (Mc + 1) + m], W[m * (d + 1) + i], acc);
+        if (xcoef) acc = fmaf(xcoef[t], X[t * d + i], acc);
         store_act(dx, base + (size_t)t * d + i, acc);
     }
 #pragma unroll
@@ -337,7 +363,8 @@ __device__ void project_back(const Problem& p, const float* X, const float* dAct
 template <typename T>
 __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
     Problem p, int C, const T* q, const T* k, const T* v, const float* W1, const float* W2,
-    const T* out, const float* den, const T* dout, T* dq, T* dk, T* dv, float* dw_part)
+    const float* tau, const T* out, const float* den, const T* dout, T* dq, T* dk, T* dv,
+    float* dw_part, float* dtau_part)
 {
     extern __shared__ float sm[];
     const int d = p.d, D = 2 * p.M, N = p.N, Mc = p.nonstat ? 2 * p.M : p.M;
@@ -346,7 +373,9 @@ __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
     const BwdLayout L = bwd_layout(p, C);
     float *W = sm + L.W, *S = sm + L.S, *Xq = sm + L.Xq, *Xk = sm + L.Xk, *Vx = sm + L.Vx;
     float *Gx = sm + L.Gx, *Pq = sm + L.Pq, *Pk = sm + L.Pk, *dP = sm + L.dP;
-    float *A = sm + L.A, *dA = sm + L.dA, *dAct = sm + L.dAct;
+    float *A = sm + L.A, *dA = sm + L.dA, *dAct = sm + L.dAct, *Kc = sm + L.Kc;
+    const float itau = tau ? expf(-tau[h]) : 0.f;
+    float dtau_acc = 0.f;
 
     float dw_acc[kMaxDwPerThread];
 #pragma unroll
@@ -364,6 +393,7 @@ __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
             load_rows(k, base + (size_t)t0 * d, CL, d, Xk, d);
             load_rows(v, base + (size_t)t0 * d, CL, d, Vx, d + 1);
             __syncthreads();
+            if (tau) weight_keys(Xk, CL, d, itau, Vx);
             features(p, Xk, CL, W, Pk, D + 1);
             __syncthreads();
             state_update(Pk, Vx, CL, D, d, S);
@@ -380,6 +410,10 @@ __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
             load_rows(v, off, CL, d, Vx, d + 1);
         }
         __syncthreads();
+        if (tau && p.causal) {
+            weight_keys(Xk, CL, d, itau, Vx);
+            __syncthreads();
+        }
         features(p, Xq, CL, W, Pq, D + 1);
         if (p.causal) features(p, Xk, CL, W, Pk, D + 1);
         if (p.causal)
@@ -403,7 +437,7 @@ __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
         if (p.causal) state_update(Pk, Vx, CL, D, d, S);
         feature_backward(p, Xq, Pq, dP, CL, W, dAct);
         __syncthreads();
-        project_back(p, Xq, dAct, CL, W, dq, off, dw_acc);
+        project_back(p, Xq, dAct, CL, W, dq, off, dw_acc, nullptr);
         __syncthreads();
     }
 
@@ -435,6 +469,10 @@ __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
             load_upstream(p, dout, out, den, off, den_base + t0, CL, Gx);
         }
         __syncthreads();
+        if (tau) {
+            weight_keys(Xk, CL, d, itau, Vx);
+            __syncthreads();
+        }
         features(p, Xk, CL, W, Pk, D + 1);
         if (p.causal) features(p, Xq, CL, W, Pq, D + 1);
         __syncthreads();
@@ -464,13 +502,22 @@ __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
             if (p.causal)
                 for (int i = j; i < CL; ++i) acc = fmaf(A[i * C + j], Gx[i * (d + 1) + e], acc);
             for (int f = 0; f < D; ++f) acc = fmaf(R[f * (d + 1) + e], Pk[j * (D + 1) + f], acc);
+            if (tau) acc *= Vx[j * (d + 1) + d];  // dv_j = w_j R_j^T phi(k_j)
             store_act(dv, off + (size_t)j * d + e, acc);
         }
         __syncthreads();
+        if (tau)  // s_j = phi(k_j) . dphi(k_j): dk_j += 2 itau s_j k_j, dtau -= itau |k_j|^2 s_j
+            for (int j = threadIdx.x; j < CL; j += blockDim.x) {
+                float sj = 0.f, n2 = 0.f;
+                for (int f = 0; f < D; ++f) sj = fmaf(Pk[j * (D + 1) + f], dP[j * (D + 1) + f], sj);
+                for (int e = 0; e < d; ++e) n2 = fmaf(Xk[j * d + e], Xk[j * d + e], n2);
+                Kc[j] = 2.f * itau * sj;
+                dtau_acc = fmaf(-itau * n2, sj, dtau_acc);
+            }
         if (p.causal) state_update(Pq, Gx, CL, D, d, R);
         feature_backward(p, Xk, Pk, dP, CL, W, dAct);
         __syncthreads();
-        project_back(p, Xk, dAct, CL, W, dk, off, dw_acc);
+        project_back(p, Xk, dAct, CL, W, dk, off, dw_acc, tau ? Kc : nullptr);
         __syncthreads();
     }
 
@@ -480,14 +527,32 @@ __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
         int e = r * kThreads + threadIdx.x;
         if (e < Mc * d) part[e] = dw_acc[r];
     }
+    if (tau) {  // this sequence's dtau: warp sums, then the warps in order
+        for (int o = 16; o > 0; o >>= 1) dtau_acc += __shfl_xor_sync(0xffffffffu, dtau_acc, o);
+        __syncthreads();
+        if ((threadIdx.x & 31) == 0) Kc[threadIdx.x >> 5] = dtau_acc;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float t = 0.f;
+            for (int w = 0; w < kThreads / 32; ++w) t += Kc[w];
+            dtau_part[bh] = t;
+        }
+    }
 }
 
 // dW over the batch, in a fixed order (deterministic).  Nonstationary: the partials hold
 // dU (rows < M) and dV (rows >= M); dW1 = (dU + dV)/2, dW2 = (dU - dV)/2.
-__global__ void dw_reduce_kernel(Problem p, const float* part, float* dW1, float* dW2)
+__global__ void dw_reduce_kernel(Problem p, const float* part, float* dW1, float* dW2,
+                                 const float* dtau_part, float* dtau)
 {
     const int d = p.d, M = p.M, Mc = p.nonstat ? 2 * M : M;
     const size_t per = (size_t)M * d;
+    if (dtau && blockIdx.x == 0)  // dtau[h] = sum over the batch, in order
+        for (int h = threadIdx.x; h < p.H; h += blockDim.x) {
+            float t = 0.f;
+            for (int bb = 0; bb < p.B; ++bb) t += dtau_part[(size_t)bb * p.H + h];
+            dtau[h] = t;
+        }
     for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < (size_t)p.H * per;
          idx += (size_t)gridDim.x * blockDim.x) {
         int h = (int)(idx / per);
@@ -537,10 +602,11 @@ int simt_pick_chunk_bwd(const Problem& p)
     return 0;
 }
 
+// dW partials [B*H][Mc][d], then dtau partials [B*H].
 size_t simt_bwd_ws_bytes(const Problem& p)
 {
     const int Mc = p.nonstat ? 2 * p.M : p.M;
-    return (size_t)p.B * p.H * Mc * p.d * sizeof(float);
+    return (size_t)p.B * p.H * (Mc * p.d + 1) * sizeof(float);
 }
 
 cudaError_t launch_featmap(const Problem& p, const void* x, const float* W1, const float* W2,
@@ -559,8 +625,8 @@ cudaError_t launch_featmap(const Problem& p, const void* x, const float* W1, con
 }
 
 cudaError_t launch_simt_fwd(const Problem& p, const void* q, const void* k, const void* v,
-                            const float* W1, const float* W2, void* out, float* den,
-                            cudaStream_t s)
+                            const float* W1, const float* W2, const float* tau, void* out,
+                            float* den, cudaStream_t s)
 {
     const int C = simt_pick_chunk_fwd(p);
     const size_t smem = simt_fwd_smem_bytes(p, C);
@@ -570,45 +636,48 @@ cudaError_t launch_simt_fwd(const Problem& p, const void* q, const void* k, cons
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, kThreads, smem, s>>>(p, C, (const __nv_bfloat16*)q,
                                           (const __nv_bfloat16*)k, (const __nv_bfloat16*)v, W1,
-                                          W2, (__nv_bfloat16*)out, den);
+                                          W2, tau, (__nv_bfloat16*)out, den);
     } else {
         auto kern = simt_fwd_kernel<float>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, kThreads, smem, s>>>(p, C, (const float*)q, (const float*)k,
-                                          (const float*)v, W1, W2, (float*)out, den);
+                                          (const float*)v, W1, W2, tau, (float*)out, den);
     }
     return cudaGetLastError();
 }
 
 cudaError_t launch_simt_bwd(const Problem& p, const void* q, const void* k, const void* v,
-                            const float* W1, const float* W2, const void* out,
-                            const float* den, const void* dout, void* dq, void* dk, void* dv,
-                            float* dW1, float* dW2, void* scratch, cudaStream_t s)
+                            const float* W1, const float* W2, const float* tau,
+                            const void* out, const float* den, const void* dout, void* dq,
+                            void* dk, void* dv, float* dW1, float* dW2, float* dtau,
+                            void* scratch, cudaStream_t s)
 {
     const int C = simt_pick_chunk_bwd(p);
     const size_t smem = simt_bwd_smem_bytes(p, C);
     const int grid = p.B * p.H;
+    const int Mc = p.nonstat ? 2 * p.M : p.M;
     float* part = (float*)scratch;
+    float* tpart = part + (size_t)p.B * p.H * Mc * p.d;
     if (p.bf16) {
         typedef __nv_bfloat16 T;
         auto kern = simt_bwd_kernel<T>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, kThreads, smem, s>>>(p, C, (const T*)q, (const T*)k, (const T*)v, W1, W2,
-                                          (const T*)out, den, (const T*)dout, (T*)dq, (T*)dk,
-                                          (T*)dv, part);
+                                          tau, (const T*)out, den, (const T*)dout, (T*)dq,
+                                          (T*)dk, (T*)dv, part, tpart);
     } else {
         typedef float T;
         auto kern = simt_bwd_kernel<T>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         kern<<<grid, kThreads, smem, s>>>(p, C, (const T*)q, (const T*)k, (const T*)v, W1, W2,
-                                          (const T*)out, den, (const T*)dout, (T*)dq, (T*)dk,
-                                          (T*)dv, part);
+                                          tau, (const T*)out, den, (const T*)dout, (T*)dq,
+                                          (T*)dk, (T*)dv, part, tpart);
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const size_t work = (size_t)p.H * p.M * p.d;
     const int blocks = (int)std::min<size_t>((work + kThreads - 1) / kThreads, 152 * 8);
-    dw_reduce_kernel<<<blocks, kThreads, 0, s>>>(p, part, dW1, dW2);
+    dw_reduce_kernel<<<blocks, kThreads, 0, s>>>(p, part, dW1, dW2, tpart, tau ? dtau : nullptr);
     return cudaGetLastError();
 }
 

@@ -58,13 +58,13 @@ def load(path: str = LIBRARY) -> ctypes.CDLL:
         lib.flex_workspace_bytes.argtypes = [shp, ip, ip]
         lib.flex_workspace_bytes.restype = sz
         lib.flex_featmap.argtypes = [shp, vp, vp, vp, vp, vp]
-        lib.flex_linattn_fwd.argtypes = [shp, vp, vp, vp, vp, vp, ip, vp, vp, vp, sz, vp]
-        lib.flex_linattn_bwd.argtypes = [shp, vp, vp, vp, vp, vp, ip, vp, vp, vp, vp, vp, vp,
-                                         vp, vp, vp, sz, vp]
+        lib.flex_linattn_fwd.argtypes = [shp, vp, vp, vp, vp, vp, vp, ip, vp, vp, vp, sz, vp]
+        lib.flex_linattn_bwd.argtypes = [shp, vp, vp, vp, vp, vp, vp, ip, vp, vp, vp, vp, vp,
+                                         vp, vp, vp, vp, vp, sz, vp]
         lib.flex_decode_workspace_bytes.argtypes = [shp]
         lib.flex_decode_workspace_bytes.restype = sz
-        lib.flex_linattn_decode.argtypes = [shp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz,
-                                            vp]
+        lib.flex_linattn_decode.argtypes = [shp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp,
+                                            sz, vp]
         lib.flex_check_status.argtypes = [vp, vp]
         lib.flex_kernel_launches.argtypes = []
         lib.flex_kernel_launches.restype = ctypes.c_ulonglong
@@ -138,8 +138,9 @@ def featmap(x, W1, W2=None, phi=None, stream=None):
 
 
 def linattn_fwd(q, k, v, W1, W2=None, causal=True, out=None, den=None, ws=None,
-                want_den=True, stream=None):
-    """(out, den) of Eq. (linear att); den is None unless want_den or given."""
+                want_den=True, stream=None, tau=None):
+    """(out, den) of Eq. (linear att); den is None unless want_den or given.  tau [H] fp32:
+    the norm prefactor exp(|x|^2 / exp(tau)) (a key weight; den excludes the query's)."""
     shape = shape_of(q, W1)
     if out is None:
         out = torch.empty_like(q)
@@ -148,14 +149,15 @@ def linattn_fwd(q, k, v, W1, W2=None, causal=True, out=None, den=None, ws=None,
     if ws is None:
         ws = workspace(shape, causal, False, q.device)
     _check(load().flex_linattn_fwd(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(W1),
-                                   _ptr(W2), int(bool(causal)), _ptr(out), _ptr(den), _ptr(ws),
-                                   ws.numel(), _stream(stream)), "flex_linattn_fwd")
+                                   _ptr(W2), _ptr(tau), int(bool(causal)), _ptr(out), _ptr(den),
+                                   _ptr(ws), ws.numel(), _stream(stream)), "flex_linattn_fwd")
     return out, den
 
 
 def linattn_bwd(q, k, v, W1, W2, causal, out, den, dout, dq=None, dk=None, dv=None,
-                dW1=None, dW2=None, ws=None, stream=None):
-    """(dq, dk, dv, dW1, dW2) of L = sum(dout * out); dW2 is None when W2 is."""
+                dW1=None, dW2=None, ws=None, stream=None, tau=None, dtau=None):
+    """(dq, dk, dv, dW1, dW2) of L = sum(dout * out); dW2 is None when W2 is.  With tau
+    (the forward's norm prefactor) a sixth value, dtau [H], follows."""
     shape = shape_of(q, W1)
     dq = torch.empty_like(q) if dq is None else dq
     dk = torch.empty_like(k) if dk is None else dk
@@ -163,14 +165,18 @@ def linattn_bwd(q, k, v, W1, W2, causal, out, den, dout, dq=None, dk=None, dv=No
     dW1 = torch.empty_like(W1) if dW1 is None else dW1
     if W2 is not None and dW2 is None:
         dW2 = torch.empty_like(W2)
+    if tau is not None and dtau is None:
+        dtau = torch.empty_like(tau)
     if ws is None:
         ws = workspace(shape, causal, True, q.device)
     _check(load().flex_linattn_bwd(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(W1),
-                                   _ptr(W2), int(bool(causal)), _ptr(out), _ptr(den),
+                                   _ptr(W2), _ptr(tau), int(bool(causal)), _ptr(out), _ptr(den),
                                    _ptr(dout), _ptr(dq), _ptr(dk), _ptr(dv), _ptr(dW1),
-                                   _ptr(dW2), _ptr(ws), ws.numel(), _stream(stream)),
+                                   _ptr(dW2), _ptr(dtau), _ptr(ws), ws.numel(), _stream(stream)),
            "flex_linattn_bwd")
-    return dq, dk, dv, dW1, dW2
+    if tau is None:
+        return dq, dk, dv, dW1, dW2
+    return dq, dk, dv, dW1, dW2, dtau
 
 
 def decode_state(B, H, M, d, device=None):
@@ -189,7 +195,7 @@ def decode_workspace(B, H, M, d, device=None) -> torch.Tensor:
 
 
 def linattn_decode(q, k, v, W1, W2, S, z, out=None, den=None, want_den=True, ws=None,
-                   stream=None):
+                   stream=None, tau=None):
     """One recurrent decode step: q, k, v [B, H, d] (one new token per sequence); the fp32
     state (S, z) is updated in place.  Returns (out [B, H, d], den [B, H] or None)."""
     B, H, d = q.shape
@@ -201,7 +207,7 @@ def linattn_decode(q, k, v, W1, W2, S, z, out=None, den=None, want_den=True, ws=
     if ws is None:
         ws = decode_workspace(B, H, W1.shape[1], d, q.device)
     _check(load().flex_linattn_decode(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(v),
-                                      _ptr(W1), _ptr(W2), _ptr(S), _ptr(z), _ptr(out),
+                                      _ptr(W1), _ptr(W2), _ptr(tau), _ptr(S), _ptr(z), _ptr(out),
                                       _ptr(den), _ptr(ws), ws.numel(), _stream(stream)),
            "flex_linattn_decode")
     return out, den

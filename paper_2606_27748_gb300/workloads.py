@@ -123,6 +123,15 @@ def draw_frequencies(w: Workload, tensor: int, hs=None) -> np.ndarray:
     return out * np.float32(1.0 / np.sqrt(w.d))
 
 
+def draw_tau(w: Workload, hs=None) -> np.ndarray:
+    """Per-head tau of the norm prefactor exp(|x|^2 / exp(tau)): ln(2 sqrt d) (the fixed
+    softmax-kernel value the learnable exp(tau) replaces) plus -0.25, 0, +0.25 by head.
+    With q, k ~ N(0, 1) d^-1/4 the key weights spread over about 1.3-2.1."""
+    heads = range(w.H) if hs is None else hs
+    return np.array([np.log(2.0 * np.sqrt(w.d)) + 0.25 * ((h % 3) - 1) for h in heads],
+                    dtype=np.float32)
+
+
 def make_inputs(w: Workload, bs=None, hs=None, N=None) -> dict:
     """All inputs of one workload (or of a subset of its sequences) as float32 arrays.
 

@@ -53,23 +53,37 @@ def test_host_validation_without_gpu(lib):
     assert lib.flex_workspace_bytes(ctypes.byref(bad), 1, 0) == 0
     p = ctypes.c_void_p(4096)  # never dereferenced: validation fails first
     # null shape / N < 1 / null input
-    assert lib.flex_linattn_fwd(None, p, p, p, p, None, 1, p, None, p, 1 << 20, None) == FLEX_EINVAL
-    assert lib.flex_linattn_fwd(ctypes.byref(bad), p, p, p, p, None, 1, p, None, p, 1 << 20,
+    # (shape, q, k, v, W1, W2, tau, causal, out, den, ws, ws_bytes, stream)
+    assert lib.flex_linattn_fwd(None, p, p, p, p, None, None, 1, p, None, p, 1 << 20,
                                 None) == FLEX_EINVAL
-    assert lib.flex_linattn_fwd(ctypes.byref(ok), None, p, p, p, None, 1, p, None, p, 1 << 20,
-                                None) == FLEX_EINVAL
-    # misaligned pointer
+    assert lib.flex_linattn_fwd(ctypes.byref(bad), p, p, p, p, None, None, 1, p, None, p,
+                                1 << 20, None) == FLEX_EINVAL
+    assert lib.flex_linattn_fwd(ctypes.byref(ok), None, p, p, p, None, None, 1, p, None, p,
+                                1 << 20, None) == FLEX_EINVAL
+    # misaligned pointer (an input, or tau off 4 bytes)
     mis = ctypes.c_void_p(4096 + 2)
-    assert lib.flex_linattn_fwd(ctypes.byref(ok), mis, p, p, p, None, 1, p, None, p, 1 << 20,
-                                None) == FLEX_EINVAL
+    assert lib.flex_linattn_fwd(ctypes.byref(ok), mis, p, p, p, None, None, 1, p, None, p,
+                                1 << 20, None) == FLEX_EINVAL
+    assert lib.flex_linattn_fwd(ctypes.byref(ok), p, p, p, p, None, mis, 1, p, None, p,
+                                1 << 20, None) == FLEX_EINVAL
     # workspace too small
-    assert lib.flex_linattn_fwd(ctypes.byref(ok), p, p, p, p, None, 1, p, None, p, 16,
+    assert lib.flex_linattn_fwd(ctypes.byref(ok), p, p, p, p, None, None, 1, p, None, p, 16,
                                 None) == FLEX_EWORKSPACE
-    # W2 given without dW2 (and the reverse)
-    args = [p] * 3 + [p, p, 1, p, p, p, p, p, p, p]
-    assert lib.flex_linattn_bwd(ctypes.byref(ok), *args, None, p, 1 << 24, None) == FLEX_EINVAL
-    args = [p] * 3 + [p, None, 1, p, p, p, p, p, p, p]
-    assert lib.flex_linattn_bwd(ctypes.byref(ok), *args, p, p, 1 << 24, None) == FLEX_EINVAL
+    # (shape, q, k, v, W1, W2, tau, causal, out, den, dout, dq, dk, dv, dW1, dW2, dtau, ws,
+    #  ws_bytes, stream): W2 given without dW2 (and the reverse); tau without dtau (and the
+    # reverse)
+    args = [p] * 3 + [p, p, None, 1, p, p, p, p, p, p, p]
+    assert lib.flex_linattn_bwd(ctypes.byref(ok), *args, None, None, p, 1 << 24,
+                                None) == FLEX_EINVAL
+    args = [p] * 3 + [p, None, None, 1, p, p, p, p, p, p, p]
+    assert lib.flex_linattn_bwd(ctypes.byref(ok), *args, p, None, p, 1 << 24,
+                                None) == FLEX_EINVAL
+    args = [p] * 3 + [p, None, p, 1, p, p, p, p, p, p, p]
+    assert lib.flex_linattn_bwd(ctypes.byref(ok), *args, None, None, p, 1 << 24,
+                                None) == FLEX_EINVAL
+    args = [p] * 3 + [p, None, None, 1, p, p, p, p, p, p, p]
+    assert lib.flex_linattn_bwd(ctypes.byref(ok), *args, None, p, p, 1 << 24,
+                                None) == FLEX_EINVAL
     assert lib.flex_strerror(FLEX_EINVAL)
 
 
@@ -82,13 +96,17 @@ def test_decode_host_validation_without_gpu(lib):
     # header + phi(q), phi(k): B H x 2 x 2M fp32
     assert need == 256 + 2 * 3 * 2 * 128 * 4
     assert lib.flex_decode_workspace_bytes(ctypes.byref(two)) == 0
-    assert lib.flex_linattn_decode(ctypes.byref(two), p, p, p, p, None, p, p, p, None,
+    # (shape, q, k, v, W1, W2, tau, S, z, out, den, ws, ws_bytes, stream)
+    assert lib.flex_linattn_decode(ctypes.byref(two), p, p, p, p, None, None, p, p, p, None,
                                    p, need, None) == FLEX_EINVAL
-    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, None, p, p, None,
+    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, None, None, p, p, None,
                                    p, need, None) == FLEX_EINVAL
-    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, p, p,
+    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, None, p, p,
                                    ctypes.c_void_p(4097), None, p, need, None) == FLEX_EINVAL
-    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, p, p, p, None,
+    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, None, p, p, p, None,
                                    p, need - 1, None) == FLEX_EWORKSPACE
-    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, p, p, p, None,
+    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None, None, p, p, p, None,
                                    None, need, None) == FLEX_EINVAL
+    assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None,
+                                   ctypes.c_void_p(4097 + 2), p, p, p, None, p, need,
+                                   None) == FLEX_EINVAL
