@@ -40,12 +40,18 @@ int check_ws(void* ws, size_t ws_bytes, size_t need)
     return FLEX_OK;
 }
 
-size_t fwd_ws_bytes(const Problem& p)
+// Header, the non-causal partial states (tensor-core path), then the key weights of the
+// norm prefactor [B*H*N] fp32 (tensor-core paths, used only when tau is given).
+size_t nc_scratch_bytes(const Problem& p)
 {
-    size_t n = header_bytes();
-    if (flex::tc_nc_supported(p)) n += flex::align_up(flex::tc_nc_ws_bytes(p), 256);
-    return n;
+    return flex::tc_nc_supported(p) ? flex::align_up(flex::tc_nc_ws_bytes(p), 256) : 0;
 }
+size_t kw_bytes(const Problem& p)
+{
+    const bool tc = flex::tc_fwd_supported(p) || flex::tc_nc_supported(p);
+    return tc ? flex::align_up((size_t)p.B * p.H * p.N * sizeof(float), 256) : 0;
+}
+size_t fwd_ws_bytes(const Problem& p) { return header_bytes() + nc_scratch_bytes(p) + kw_bytes(p); }
 
 size_t bwd_ws_bytes(const Problem& p)
 {
@@ -117,11 +123,17 @@ int flex_linattn_fwd(const flex_shape* shape, const void* q, const void* k, cons
     if ((rc = check_ws(ws, ws_bytes, fwd_ws_bytes(p)))) return rc;
     cudaStream_t s = (cudaStream_t)stream;
     int* status = &((flex::WsHeader*)ws)->status;
-    if (!tau && flex::tc_fwd_supported(p))
-        return count(1, flex::launch_tc_fwd(p, q, k, v, W1, W2, out, den, status, s));
-    if (!tau && flex::tc_nc_supported(p))
-        return count(3, flex::launch_tc_nc(p, q, k, v, W1, W2, out, den,
+    const bool tcf = flex::tc_fwd_supported(p), tcn = !tcf && flex::tc_nc_supported(p);
+    if (tcf || tcn) {
+        float* kw = nullptr;  // key weights of the norm prefactor, one pass over k
+        if (tau) {
+            kw = (float*)((char*)ws + header_bytes() + nc_scratch_bytes(p));
+            if (int e = count(1, flex::launch_key_weights(p, k, tau, kw, s))) return e;
+        }
+        if (tcf) return count(1, flex::launch_tc_fwd(p, q, k, v, W1, W2, kw, out, den, status, s));
+        return count(3, flex::launch_tc_nc(p, q, k, v, W1, W2, kw, out, den,
                                            (char*)ws + header_bytes(), status, s));
+    }
     if (flex::simt_pick_chunk_fwd(p) == 0) return FLEX_EUNSUPPORTED;
     return count(1, flex::launch_simt_fwd(p, q, k, v, W1, W2, tau, out, den, s));
 }

@@ -48,6 +48,11 @@ cudaError_t launch_simt_bwd(const Problem& p, const void* q, const void* k, cons
                             void* dk, void* dv, float* dW1, float* dW2, float* dtau,
                             void* scratch, cudaStream_t s);
 
+// Key weights of the norm prefactor (Sec. 3.2), kw [B*H*N] fp32, for the tensor-core
+// forwards: exp(|k|^2 exp(-tau_h)).
+cudaError_t launch_key_weights(const Problem& p, const void* k, const float* tau, float* kw,
+                               cudaStream_t s);
+
 // ---- recurrent decode step (one token per sequence; fp32 state) ----------------------
 size_t decode_ws_bytes(const Problem& p);  // phi(q), phi(k) of the step, fp32
 cudaError_t launch_decode(const Problem& p, const void* q, const void* k, const void* v,
@@ -57,16 +62,17 @@ cudaError_t launch_decode(const Problem& p, const void* q, const void* k, const 
 // ---- tensor-core path (bf16 storage, d = 64, M in {64, 128}) ------------------------
 bool tc_fwd_supported(const Problem& p);
 int tc_fwd_splits(const Problem& p, int sms);  // segments per sequence (1-3)
+// kw: key weights of the norm prefactor or NULL.
 cudaError_t launch_tc_fwd(const Problem& p, const void* q, const void* k, const void* v,
-                          const float* W1, const float* W2, void* out, float* den, int* status,
-                          cudaStream_t s);
+                          const float* W1, const float* W2, const float* kw, void* out,
+                          float* den, int* status, cudaStream_t s);
 
 bool tc_nc_supported(const Problem& p);
 int tc_nc_splits(const Problem& p);
 size_t tc_nc_ws_bytes(const Problem& p);
 cudaError_t launch_tc_nc(const Problem& p, const void* q, const void* k, const void* v,
-                         const float* W1, const float* W2, void* out, float* den, void* scratch,
-                         int* status, cudaStream_t s);
+                         const float* W1, const float* W2, const float* kw, void* out,
+                         float* den, void* scratch, int* status, cudaStream_t s);
 
 bool tc_bwd_supported(const Problem& p);
 size_t tc_bwd_ws_bytes(const Problem& p);

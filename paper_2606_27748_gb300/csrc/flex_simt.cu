@@ -540,6 +540,36 @@ __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
     }
 }
 
+// Key weights of the norm prefactor for the tensor-core forwards: kw[row] =
+// exp(|k_row|^2 exp(-tau_h)) for every row of k [B*H*N][d]; one thread per row, vector
+// loads of 4 elements (d % 4 == 0).
+template <typename T>
+__global__ void __launch_bounds__(kThreads) key_weights_kernel(Problem p, const T* k,
+                                                               const float* tau, float* kw)
+{
+    const size_t rows = (size_t)p.B * p.H * p.N;
+    for (size_t r = (size_t)blockIdx.x * blockDim.x + threadIdx.x; r < rows;
+         r += (size_t)gridDim.x * blockDim.x) {
+        const T* x = k + r * p.d;
+        float n2 = 0.f;
+        for (int e = 0; e < p.d; e += 4) {
+            float v[4];
+            if constexpr (sizeof(T) == 4) {
+                const float4 f = *reinterpret_cast<const float4*>(x + e);
+                v[0] = f.x; v[1] = f.y; v[2] = f.z; v[3] = f.w;
+            } else {
+                const uint2 u = *reinterpret_cast<const uint2*>(x + e);
+                v[0] = __uint_as_float(u.x << 16); v[1] = __uint_as_float(u.x & 0xffff0000u);
+                v[2] = __uint_as_float(u.y << 16); v[3] = __uint_as_float(u.y & 0xffff0000u);
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) n2 = fmaf(v[i], v[i], n2);
+        }
+        const int h = (int)((r / p.N) % p.H);
+        kw[r] = expf(n2 * expf(-tau[h]));
+    }
+}
+
 // dW over the batch, in a fixed order (deterministic).  Nonstationary: the partials hold
 // dU (rows < M) and dV (rows >= M); dW1 = (dU + dV)/2, dW2 = (dU - dV)/2.
 __global__ void dw_reduce_kernel(Problem p, const float* part, float* dW1, float* dW2,
@@ -607,6 +637,18 @@ size_t simt_bwd_ws_bytes(const Problem& p)
 {
     const int Mc = p.nonstat ? 2 * p.M : p.M;
     return (size_t)p.B * p.H * (Mc * p.d + 1) * sizeof(float);
+}
+
+cudaError_t launch_key_weights(const Problem& p, const void* k, const float* tau, float* kw,
+                               cudaStream_t s)
+{
+    const size_t rows = (size_t)p.B * p.H * p.N;
+    const int blocks = (int)std::min<size_t>((rows + kThreads - 1) / kThreads, 152 * 16);
+    if (p.bf16)
+        key_weights_kernel<<<blocks, kThreads, 0, s>>>(p, (const __nv_bfloat16*)k, tau, kw);
+    else
+        key_weights_kernel<<<blocks, kThreads, 0, s>>>(p, (const float*)k, tau, kw);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_featmap(const Problem& p, const void* x, const float* W1, const float* W2,

@@ -124,8 +124,8 @@ __global__ void __maxnreg__(96)
                          const __grid_constant__ CUtensorMap tmap_k,
                          const __grid_constant__ CUtensorMap tmap_v, int H, int N, int M,
                          int splits, const float* __restrict__ W1,
-                         const float* __restrict__ W2, __nv_bfloat16* __restrict__ out,
-                         float* __restrict__ den, int* status)
+                         const float* __restrict__ W2, const float* __restrict__ kw,
+                         __nv_bfloat16* __restrict__ out, float* __restrict__ den, int* status)
 {
     using L = Cfg<NS>;
     extern __shared__ uint8_t smem_raw[];
@@ -376,6 +376,8 @@ __global__ void __maxnreg__(96)
         for (int c = 0; c < ce; ++c) {
             const bool main = c >= cb;
             const bool valid = t < min(kC, N - c * kC);
+            // key weight of the norm prefactor (phi(k) scaled by it), loaded early
+            const float wk = (kw && valid) ? kw[(size_t)bh * N + (size_t)c * kC + t] : 1.f;
             for (int which = main ? 0 : 1; which < 2; ++which) {  // 0: q, 1: k
                 uint32_t pc[16], ps[16];  // [8 r + i]: frequencies 32r + 16 half + 2i, +1
 #pragma unroll
@@ -403,6 +405,7 @@ __global__ void __maxnreg__(96)
                             const float cw0 = __cosf(w[2 * i]), cw1 = __cosf(w[2 * i + 1]);
                             c0 *= cw0; s0 *= cw0; c1 *= cw1; s1 *= cw1;
                         }
+                        if (kw && which == 1) { c0 *= wk; s0 *= wk; c1 *= wk; s1 *= wk; }
                         if (!valid) { c0 = s0 = c1 = s1 = 0.f; }
                         pc[8 * r + i] = pack_bf16(c0, c1);
                         ps[8 * r + i] = pack_bf16(s0, s1);
@@ -626,8 +629,8 @@ __global__ void __maxnreg__(96)
 
 template <bool NS, int CS>
 cudaError_t launch_one(const Problem& p, const void* q, const void* k, const void* v,
-                       const float* W1, const float* W2, void* out, float* den, int* status,
-                       cudaStream_t s)
+                       const float* W1, const float* W2, const float* kw, void* out,
+                       float* den, int* status, cudaStream_t s)
 {
     CUtensorMap mq, mk, mv;
     const int BH = p.B * p.H;
@@ -651,7 +654,7 @@ cudaError_t launch_one(const Problem& p, const void* q, const void* k, const voi
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, mq, mk, mv, p.H, p.N, p.M, splits, W1, W2,
+    return cudaLaunchKernelEx(&cfg, kern, mq, mk, mv, p.H, p.N, p.M, splits, W1, W2, kw,
                               (__nv_bfloat16*)out, den, status);
 }
 
@@ -672,15 +675,15 @@ bool tc_fwd_supported(const Problem& p)
 }
 
 cudaError_t launch_tc_fwd(const Problem& p, const void* q, const void* k, const void* v,
-                          const float* W1, const float* W2, void* out, float* den, int* status,
-                          cudaStream_t s)
+                          const float* W1, const float* W2, const float* kw, void* out,
+                          float* den, int* status, cudaStream_t s)
 {
     const bool pair = p.M == 128;
     if (p.nonstat)
-        return pair ? launch_one<true, 2>(p, q, k, v, W1, W2, out, den, status, s)
-                    : launch_one<true, 1>(p, q, k, v, W1, W2, out, den, status, s);
-    return pair ? launch_one<false, 2>(p, q, k, v, W1, W2, out, den, status, s)
-                : launch_one<false, 1>(p, q, k, v, W1, W2, out, den, status, s);
+        return pair ? launch_one<true, 2>(p, q, k, v, W1, W2, kw, out, den, status, s)
+                    : launch_one<true, 1>(p, q, k, v, W1, W2, kw, out, den, status, s);
+    return pair ? launch_one<false, 2>(p, q, k, v, W1, W2, kw, out, den, status, s)
+                : launch_one<false, 1>(p, q, k, v, W1, W2, kw, out, den, status, s);
 }
 
 }  // namespace flex

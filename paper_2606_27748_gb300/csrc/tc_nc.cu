@@ -69,8 +69,9 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
     tc_nc_kernel(const __grid_constant__ CUtensorMap tmap_x,
                  const __grid_constant__ CUtensorMap tmap_v, int H, int N, int M, int splits,
                  const float* __restrict__ W1, const float* __restrict__ W2,
-                 float* __restrict__ part, const float* __restrict__ total,
-                 __nv_bfloat16* __restrict__ out, float* __restrict__ den, int* status)
+                 const float* __restrict__ kw, float* __restrict__ part,
+                 const float* __restrict__ total, __nv_bfloat16* __restrict__ out,
+                 float* __restrict__ den, int* status)
 {
     using L = NcCfg<NS, G>;
     extern __shared__ uint8_t smem_raw[];
@@ -249,6 +250,9 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
         for (int j = 0; j < njobs; ++j) {
             const int i = j / G, pb = j & 1;
             const bool valid = t < min(kC, N - (c0 + i) * kC);
+            // state mode: key weight of the norm prefactor (phi(k) scaled by it)
+            const float wk = (MODE == kState && kw && valid)
+                                 ? kw[(size_t)bh * N + (size_t)(c0 + i) * kC + t] : 1.f;
             if (!bar_wait(&bars.p_full[pb], (j >> 1) & 1, &abort_flag, status)) break;
             fence_after_sync();
             const uint32_t tp = tm_row + (pb ? L::T_P1 : L::T_P0);
@@ -273,6 +277,7 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
                     const float cw0 = __cosf(w[2 * e]), cw1 = __cosf(w[2 * e + 1]);
                     cc0 *= cw0; s0 *= cw0; cc1 *= cw1; s1 *= cw1;
                 }
+                if (MODE == kState && kw) { cc0 *= wk; s0 *= wk; cc1 *= wk; s1 *= wk; }
                 if (!valid) { cc0 = s0 = cc1 = s1 = 0.f; }
                 pc[e] = pack_bf16(cc0, cc1);
                 ps[e] = pack_bf16(s0, s1);
@@ -366,8 +371,8 @@ __global__ void nc_reduce_kernel(int BH, int splits, int G, const float* __restr
 
 template <bool NS, int G>
 cudaError_t launch_nc(const Problem& p, const void* q, const void* k, const void* v,
-                      const float* W1, const float* W2, void* out, float* den, void* scratch,
-                      int* status, cudaStream_t s)
+                      const float* W1, const float* W2, const float* kw, void* out, float* den,
+                      void* scratch, int* status, cudaStream_t s)
 {
     const int BH = p.B * p.H, splits = tc_nc_splits(p);
     CUtensorMap mq, mk, mv;
@@ -383,15 +388,15 @@ cudaError_t launch_nc(const Problem& p, const void* q, const void* k, const void
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(k_out, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    k_state<<<BH * splits, kThreadsNC, smem, s>>>(mk, mv, p.H, p.N, p.M, splits, W1, W2, part,
-                                                 nullptr, nullptr, nullptr, status);
+    k_state<<<BH * splits, kThreadsNC, smem, s>>>(mk, mv, p.H, p.N, p.M, splits, W1, W2, kw,
+                                                 part, nullptr, nullptr, nullptr, status);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const size_t n = (size_t)BH * G * 128 * kRow;
     nc_reduce_kernel<<<(int)std::min<size_t>((n + 255) / 256, 152 * 8), 256, 0, s>>>(BH, splits, G,
                                                                                     part, total);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     k_out<<<BH * splits, kThreadsNC, smem, s>>>(mq, mv, p.H, p.N, p.M, splits, W1, W2, nullptr,
-                                               total, (__nv_bfloat16*)out, den, status);
+                                               nullptr, total, (__nv_bfloat16*)out, den, status);
     return cudaGetLastError();
 }
 
@@ -431,15 +436,15 @@ size_t tc_nc_ws_bytes(const Problem& p)
 }
 
 cudaError_t launch_tc_nc(const Problem& p, const void* q, const void* k, const void* v,
-                         const float* W1, const float* W2, void* out, float* den, void* scratch,
-                         int* status, cudaStream_t s)
+                         const float* W1, const float* W2, const float* kw, void* out,
+                         float* den, void* scratch, int* status, cudaStream_t s)
 {
     const int G = p.M / 64;
     if (p.nonstat)
-        return G == 1 ? launch_nc<true, 1>(p, q, k, v, W1, W2, out, den, scratch, status, s)
-                      : launch_nc<true, 2>(p, q, k, v, W1, W2, out, den, scratch, status, s);
-    return G == 1 ? launch_nc<false, 1>(p, q, k, v, W1, W2, out, den, scratch, status, s)
-                  : launch_nc<false, 2>(p, q, k, v, W1, W2, out, den, scratch, status, s);
+        return G == 1 ? launch_nc<true, 1>(p, q, k, v, W1, W2, kw, out, den, scratch, status, s)
+                      : launch_nc<true, 2>(p, q, k, v, W1, W2, kw, out, den, scratch, status, s);
+    return G == 1 ? launch_nc<false, 1>(p, q, k, v, W1, W2, kw, out, den, scratch, status, s)
+                  : launch_nc<false, 2>(p, q, k, v, W1, W2, kw, out, den, scratch, status, s);
 }
 
 }  // namespace flex

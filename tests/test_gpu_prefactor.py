@@ -108,3 +108,21 @@ def test_decode_with_prefactor(w, causal, d, M, dtype):
         _, _, So, zo = oracle.decode(ins["q"][:, :, i], ins["k"][:, :, i], ins["v"][:, :, i],
                                      ins["W1"], ins["W2"], So, zo, tau=ins["tau"])
     assert rel_l2(to_host(S), So) <= F32_REL_L2 and rel_l2(to_host(z), zo) <= F32_REL_L2
+
+
+@pytest.mark.parametrize("causal,launches", [(True, 2), (False, 4)])
+def test_tensor_core_forward_takes_the_prefactor(causal, launches):
+    """bf16 d = 64 shapes keep the tensor-core forward with tau: one pass over k for the
+    key weights, then the usual kernels (causal 1, non-causal 3)."""
+    w = WL[2] if causal else WL[3]
+    _, ins = _setup(w, causal, 64, 64, "bf16", N=700)
+    q, k, v, _, W1, W2, tau = _dev(ins, "bf16")
+    shape = flexattn.shape_of(q, W1)
+    ws = flexattn.workspace(shape, causal, False)
+    n0 = flexattn.kernel_launches()
+    out, den = flexattn.linattn_fwd(q, k, v, W1, W2, causal, ws=ws, tau=tau)
+    flexattn.check_status(ws)
+    assert flexattn.kernel_launches() - n0 == launches
+    ro, _ = oracle.fwd(ins["q"], ins["k"], ins["v"], ins["W1"], ins["W2"], causal,
+                       tau=ins["tau"])
+    assert_close(to_host(out), ro, "bf16", "out")
