@@ -159,9 +159,11 @@ int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, cons
     if ((rc = check_ws(ws, ws_bytes, bwd_ws_bytes(p)))) return rc;
     cudaStream_t s = (cudaStream_t)stream;
     void* scratch = (char*)ws + header_bytes();
-    if (!tau && flex::tc_bwd_supported(p))
-        return count(3, flex::launch_tc_bwd(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1,
-                                            dW2, scratch, &((flex::WsHeader*)ws)->status, s));
+    if (flex::tc_bwd_supported(p))  // with tau: one more launch, the key weights
+        return count(tau ? 4 : 3,
+                     flex::launch_tc_bwd(p, q, k, v, W1, W2, tau, out, den, dout, dq, dk, dv,
+                                         dW1, dW2, dtau, scratch, &((flex::WsHeader*)ws)->status,
+                                         s));
     if (flex::simt_pick_chunk_bwd(p) == 0) return FLEX_EUNSUPPORTED;
     return count(2, flex::launch_simt_bwd(p, q, k, v, W1, W2, tau, out, den, dout, dq, dk, dv,
                                           dW1, dW2, dtau, scratch, s));

@@ -77,8 +77,9 @@ cudaError_t launch_tc_nc(const Problem& p, const void* q, const void* k, const v
 bool tc_bwd_supported(const Problem& p);
 size_t tc_bwd_ws_bytes(const Problem& p);
 cudaError_t launch_tc_bwd(const Problem& p, const void* q, const void* k, const void* v,
-                          const float* W1, const float* W2, const void* out, const float* den,
-                          const void* dout, void* dq, void* dk, void* dv, float* dW1, float* dW2,
-                          void* scratch, int* status, cudaStream_t s);
+                          const float* W1, const float* W2, const float* tau, const void* out,
+                          const float* den, const void* dout, void* dq, void* dk, void* dv,
+                          float* dW1, float* dW2, float* dtau, void* scratch, int* status,
+                          cudaStream_t s);
 
 }  // namespace flex

@@ -18,6 +18,14 @@
 // S, z), pass R runs them backward (dk, dv and the k part of dW, state R, r); the two are
 // independent and run as the two halves of one grid.
 //
+// Norm prefactor (Sec. 3.2, optional): with key weights w_j = exp(|k_j|^2 exp(-tau)) (kw,
+// one pass over k before this kernel), phi(k) is stored weighted, so S, z, A and dv come
+// out weighted and T_D holds the gradient with respect to the weighted features.  In pass
+// R the chain rule then needs dphi(k) = w dphi~(k) (the stationary feature tile already
+// carries w; the nonstationary recomputation multiplies by it), s_j = phi~(k_j).dphi~(k_j)
+// adds 2 exp(-tau) s_j k_j to dk_j (folded into the same row adds) and -ln(w_j) s_j to
+// dtau (per-CTA slots, reduced with dW in a fixed order).
+//
 // Phases are serialised: all 256 threads load, compute features and run the CUDA-core
 // epilogues; thread 0 issues the MMAs; one mbarrier tracks their completion (bounded waits).
 //
@@ -49,7 +57,8 @@ struct BwCfg {
     static constexpr uint32_t SN = 200704;    // state snapshot [feature][64 dcol], bf16
     static constexpr uint32_t ZR = 217088;    // z or r [128] fp32
     static constexpr uint32_t CROW = 217600;  // c_t [128] fp32
-    static constexpr uint32_t BYTES = 218112;
+    static constexpr uint32_t SPART = 218112; // prefactor: s_t partials [2 warpgroups][128]
+    static constexpr uint32_t BYTES = 219136;
     static constexpr uint32_t T_P = 0, T_A = 128, T_D = 256, T_S = 384;
     static_assert(BYTES + 1024 <= 232448, "shared memory budget");
 };
@@ -78,7 +87,8 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                   const __nv_bfloat16* __restrict__ outp, const float* __restrict__ den,
                   const __nv_bfloat16* __restrict__ dout, float* __restrict__ acc_q,
                   float* __restrict__ acc_k, float* __restrict__ acc_v, float* __restrict__ dw_part,
-                  int units, int* status)
+                  const float* __restrict__ kw, const float* __restrict__ tau,
+                  float* __restrict__ dtau_part, int units, int* status)
 {
     using L = BwCfg<NS>;
     // blocks [0, units): pass F, [units, 2 units): pass R; unit = (sequence, group)
@@ -98,6 +108,9 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     const size_t base = (size_t)bh * N * 64;
     float* zr = reinterpret_cast<float*>(sm + L::ZR);
     float* crow = reinterpret_cast<float*>(sm + L::CROW);
+    float* spart = reinterpret_cast<float*>(sm + L::SPART);
+    const float itau = kw ? expf(-tau[h]) : 0.f;
+    float dtau_acc = 0.f;
 
     // ---- set-up: this group's projection rows, zero state, C16 ----
     for (int idx = tid; idx < L::P * 8; idx += kThreadsB) {
@@ -195,7 +208,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         }
         return commit_wait();
     };
-    auto features = [&](uint32_t dst, uint32_t tcol, bool valid) {
+    auto features = [&](uint32_t dst, uint32_t tcol, bool valid, float wsc) {
         float a[32], w[32];
         tmem_ld16(tm_row + tcol + 32 * wg, *reinterpret_cast<float(*)[16]>(&a[0]));
         tmem_ld16(tm_row + tcol + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
@@ -214,6 +227,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 const float cw0 = __cosf(w[2 * i]), cw1 = __cosf(w[2 * i + 1]);
                 c0 *= cw0; s0 *= cw0; c1 *= cw1; s1 *= cw1;
             }
+            if (kw) { c0 *= wsc; s0 *= wsc; c1 *= wsc; s1 *= wsc; }
             if (!valid) { c0 = s0 = c1 = s1 = 0.f; }
             pc[i] = pack_bf16(c0, c1);
             ps[i] = pack_bf16(s0, s1);
@@ -228,7 +242,9 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     // Chain rule through the features of this thread's 32 frequencies: dphi from T_D plus
     // the per-feature term zr * scale, then da written over the feature tile in place
     // (s: da in the cos columns, zeros in the sin columns; n: du | dw).
-    auto feature_backward = [&](uint32_t tile, float scale, bool valid) {
+    // wkey: the key weight (pass R with the prefactor, else 1); returns this thread's part
+    // of s_t = phi~(k_t) . dphi~(k_t) (pass R with the prefactor, else 0).
+    auto feature_backward = [&](uint32_t tile, float scale, bool valid, float wkey) -> float {
         float dc[32], ds[32];
         tmem_ld16(tm_row + L::T_D + 32 * wg, *reinterpret_cast<float(*)[16]>(&dc[0]));
         tmem_ld16(tm_row + L::T_D + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&dc[16]));
@@ -261,6 +277,8 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             zc[4 * j] = a4.x; zc[4 * j + 1] = a4.y; zc[4 * j + 2] = a4.z; zc[4 * j + 3] = a4.w;
             zs[4 * j] = b4.x; zs[4 * j + 1] = b4.y; zs[4 * j + 2] = b4.z; zs[4 * j + 3] = b4.w;
         }
+        const bool wt = kw && PASS == kPassR;
+        float sdot = 0.f;
         uint32_t o1[16], o2[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
@@ -269,17 +287,23 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             for (int e = 0; e < 2; ++e) {
                 const int fi = 2 * i + e;
                 const float dphic = dc[fi] + scale * zc[fi], dphis = ds[fi] + scale * zs[fi];
-                if (!NS) {
+                if (!NS) {  // the tile's features carry the key weight (pass R, prefactor)
                     const float pc = __uint_as_float(e ? cpair[i] & 0xFFFF0000u : cpair[i] << 16);
                     const float psn = __uint_as_float(e ? spair[i] & 0xFFFF0000u : spair[i] << 16);
                     r1[e] = -psn * dphic + pc * dphis;
                     r2[e] = 0.f;
+                    if (wt) sdot = fmaf(pc, dphic, fmaf(psn, dphis, sdot));
                 } else {
                     float su, cu, sw, cw;
                     __sincosf(a[fi], &su, &cu);
                     __sincosf(w[fi], &sw, &cw);
                     r1[e] = cw * (-su * dphic + cu * dphis);
                     r2[e] = -sw * (cu * dphic + su * dphis);
+                    if (wt) {
+                        sdot = fmaf(cu * cw, dphic, fmaf(su * cw, dphis, sdot));
+                        r1[e] *= wkey;
+                        r2[e] *= wkey;
+                    }
                 }
                 if (!valid) r1[e] = r2[e] = 0.f;
             }
@@ -292,6 +316,8 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             st_shared_v4(tile + off, o1[4 * j], o1[4 * j + 1], o1[4 * j + 2], o1[4 * j + 3]);
             st_shared_v4(tile + 16384 + off, o2[4 * j], o2[4 * j + 1], o2[4 * j + 2], o2[4 * j + 3]);
         }
+        if (!valid) sdot = 0.f;
+        return NS ? sdot * wkey : sdot;  // n: phi~ = w cos u cos w, w sin u cos w
     };
     // dx = da W (T_A[0,64)) and dW = da^T x: n: this chunk's in T_A[64,128); s: summed
     // over the chunks in the projection's unused half, T_P[64,128)
@@ -343,11 +369,25 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         if (wg == 0) zr[t] = zz[0];
     };
     // rows of a [128 x 64] TMEM block (T_A[0,64)) added into an fp32 [token][64] accumulator
-    auto add_rows = [&](float* acc, int t0, bool valid) {
+    // kcoef != 0: + kcoef * k_t (the prefactor's dk term; k row from the K tile)
+    auto add_rows = [&](float* acc, int t0, bool valid, float kcoef) {
         float v_[32];
         tmem_ld16(tm_row + L::T_A + 32 * wg, *reinterpret_cast<float(*)[16]>(&v_[0]));
         tmem_ld16(tm_row + L::T_A + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&v_[16]));
         tmem_wait_ld();
+        if (kcoef != 0.f) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint4 k4 = *reinterpret_cast<const uint4*>(sm + L::K + swz128(t, 32 * wg + 8 * j));
+                const uint32_t kw4[4] = {k4.x, k4.y, k4.z, k4.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    v_[8 * j + 2 * e] = fmaf(kcoef, __uint_as_float(kw4[e] << 16), v_[8 * j + 2 * e]);
+                    v_[8 * j + 2 * e + 1] =
+                        fmaf(kcoef, __uint_as_float(kw4[e] & 0xFFFF0000u), v_[8 * j + 2 * e + 1]);
+                }
+            }
+        }
         if (valid) {
             float* dst = acc + base + (size_t)(t0 + t) * 64 + 32 * wg;
 #pragma unroll
@@ -362,6 +402,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         const int c = PASS == kPassF ? it : nch - 1 - it;
         const int t0 = c * kC, CL = min(kC, N - t0);
         const bool valid = t < CL;
+        const float wk = (kw && valid) ? kw[(size_t)bh * N + t0 + t] : 1.f;
         if (tid == 0) {  // the next chunk's tiles into L2 while this one is worked on
             const int cn = PASS == kPassF ? c + 1 : c - 1;
             if (cn >= 0 && cn < nch) {
@@ -425,8 +466,8 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         handoff();
         // ---- features of q and k for this group ----
         if (!project_qk()) goto done;
-        features(sb + L::PQ, L::T_P, valid);
-        features(sb + L::PK, L::T_A, valid);
+        features(sb + L::PQ, L::T_P, valid, 1.f);
+        features(sb + L::PK, L::T_A, valid, wk);
         handoff();
 
         if (PASS == kPassF) {
@@ -480,10 +521,10 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             }
             if (!commit_wait()) goto done;
             // n: u, w of q for the chain rule are still in T_P
-            feature_backward(sb + L::PQ, crow[t], valid);
+            feature_backward(sb + L::PQ, crow[t], valid, 1.f);
             handoff();
             if (!project_back(dPQ, dPQmn, dQmn, it == 0)) goto done;
-            add_rows(acc_x, t0, valid);
+            add_rows(acc_x, t0, valid, 0.f);
             if (NS) dw_accumulate(it == 0);
             snapshot();
             handoff();
@@ -560,20 +601,37 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 }
             }
             if (!commit_wait()) goto done;
-            add_rows(acc_v, t0, valid);  // dv of this group
+            add_rows(acc_v, t0, valid, 0.f);  // dv of this group
             fence_before_sync();
             __syncthreads();
             if (NS && !project(dK)) goto done;  // u, w of k for the chain rule
-            feature_backward(sb + L::PK, 1.0f, valid);
+            {
+                const float sp = feature_backward(sb + L::PK, 1.0f, valid, wk);
+                if (kw) {
+                    spart[128 * wg + t] = sp;
+                    dtau_acc = fmaf(-logf(wk), sp, dtau_acc);  // ln w = |k|^2 exp(-tau)
+                }
+            }
             handoff();
             if (!project_back(dPK, dPKmn, dKmn, it == 0)) goto done;
-            add_rows(acc_x, t0, valid);
+            add_rows(acc_x, t0, valid, kw ? 2.f * itau * (spart[t] + spart[128 + t]) : 0.f);
             if (NS) dw_accumulate(it == 0);
             snapshot();
             handoff();
         }
     }
     if (!NS) dw_accumulate(true);  // s: the sum over all chunks, from T_P[64,128)
+    if (kw) {  // this CTA's dtau (pass R; 0 in pass F): warps, then in order
+        for (int o = 16; o > 0; o >>= 1) dtau_acc += __shfl_xor_sync(0xffffffffu, dtau_acc, o);
+        __syncthreads();
+        if (lane == 0) spart[warp] = dtau_acc;
+        __syncthreads();
+        if (tid == 0) {
+            float sum = 0.f;
+            for (int w8 = 0; w8 < kThreadsB / 32; ++w8) sum += spart[w8];
+            dtau_part[blockIdx.x] = sum;
+        }
+    }
 done:
     fence_before_sync();
     __syncthreads();
@@ -586,8 +644,16 @@ done:
 // 64g + row%64.
 __global__ void tc_dw_reduce_kernel(int B, int H, int M, int G, int nonstat,
                                     const float* __restrict__ part, float* __restrict__ dW1,
-                                    float* __restrict__ dW2)
+                                    float* __restrict__ dW2, const float* __restrict__ dtau_part,
+                                    float* __restrict__ dtau)
 {
+    if (dtau && blockIdx.x == 0)  // dtau[h]: the pass R slots of head h, in order
+        for (int h = threadIdx.x; h < H; h += blockDim.x) {
+            float a = 0.f;
+            for (int b = 0; b < B; ++b)
+                for (int g = 0; g < G; ++g) a += dtau_part[(size_t)B * H * G + (b * H + h) * G + g];
+            dtau[h] = a;
+        }
     const size_t total = (size_t)H * M * 64;
     for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
          idx += (size_t)gridDim.x * blockDim.x) {
@@ -624,9 +690,10 @@ __global__ void tc_to_bf16_kernel(size_t n, const float* __restrict__ a, const f
 
 template <bool NS>
 cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const void* v,
-                       const float* W1, const float* W2, const void* out, const float* den,
-                       const void* dout, void* dq, void* dk, void* dv, float* dW1, float* dW2,
-                       void* scratch, int* status, cudaStream_t s)
+                       const float* W1, const float* W2, const float* tau, const void* out,
+                       const float* den, const void* dout, void* dq, void* dk, void* dv,
+                       float* dW1, float* dW2, float* dtau, void* scratch, int* status,
+                       cudaStream_t s)
 {
     const int BH = p.B * p.H, G = p.M / 64;
     const size_t n = (size_t)BH * p.N * 64;
@@ -634,8 +701,11 @@ cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const voi
     float* acc_k = acc_q + n;
     float* acc_v = acc_k + n;
     float* part = acc_v + n;
+    float* kw = part + (size_t)2 * BH * G * 128 * 64;  // key weights [B*H*N] (prefactor)
+    float* dtau_part = kw + (size_t)BH * p.N;           // [2 units]
     cudaError_t e = cudaMemsetAsync(acc_q, 0, 3 * n * sizeof(float), s);
     if (e != cudaSuccess) return e;
+    if (tau && (e = launch_key_weights(p, k, tau, kw, s)) != cudaSuccess) return e;
     const int smem = (int)BwCfg<NS>::BYTES + 1024;
     CUtensorMap mq, mk, mv;
     if (!make_act_map(&mq, q, BH, p.N) || !make_act_map(&mk, k, BH, p.N) ||
@@ -648,11 +718,11 @@ cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const voi
     kb<<<2 * units, kThreadsB, smem, s>>>(mq, mk, mv, p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k,
                                           (CB)v, W1,
                                           W2, (CB)out, den, (CB)dout, acc_q, acc_k, acc_v, part,
-                                          units, status);
+                                          tau ? kw : nullptr, tau, dtau_part, units, status);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     const size_t work = (size_t)p.H * p.M * 64;
     tc_dw_reduce_kernel<<<(int)std::min<size_t>((work + 255) / 256, 152 * 8), 256, 0, s>>>(
-        p.B, p.H, p.M, G, p.nonstat, part, dW1, dW2);
+        p.B, p.H, p.M, G, p.nonstat, part, dW1, dW2, dtau_part, tau ? dtau : nullptr);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     tc_to_bf16_kernel<<<152 * 8, 256, 0, s>>>(n, acc_q, acc_k, acc_v, (__nv_bfloat16*)dq,
                                                (__nv_bfloat16*)dk, (__nv_bfloat16*)dv);
@@ -668,22 +738,25 @@ bool tc_bwd_supported(const Problem& p)
     return p.bf16 && p.causal && p.d == 64 && (p.M == 64 || p.M == 128);
 }
 
+// fp32 dq/dk/dv accumulators, dW partials [2 passes][B*H*G][128][64], key weights
+// [B*H*N] and dtau partials [2 B*H*G] (norm prefactor).
 size_t tc_bwd_ws_bytes(const Problem& p)
 {
     const size_t BH = (size_t)p.B * p.H, G = (size_t)p.M / 64;
-    return (3 * BH * p.N * 64 + 2 * BH * G * 128 * 64) * sizeof(float);
+    return (3 * BH * p.N * 64 + 2 * BH * G * 128 * 64 + BH * p.N + 2 * BH * G) * sizeof(float);
 }
 
 cudaError_t launch_tc_bwd(const Problem& p, const void* q, const void* k, const void* v,
-                          const float* W1, const float* W2, const void* out, const float* den,
-                          const void* dout, void* dq, void* dk, void* dv, float* dW1, float* dW2,
-                          void* scratch, int* status, cudaStream_t s)
+                          const float* W1, const float* W2, const float* tau, const void* out,
+                          const float* den, const void* dout, void* dq, void* dk, void* dv,
+                          float* dW1, float* dW2, float* dtau, void* scratch, int* status,
+                          cudaStream_t s)
 {
     if (p.nonstat)
-        return launch_bwd<true>(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1, dW2, scratch,
-                                status, s);
-    return launch_bwd<false>(p, q, k, v, W1, W2, out, den, dout, dq, dk, dv, dW1, dW2, scratch,
-                             status, s);
+        return launch_bwd<true>(p, q, k, v, W1, W2, tau, out, den, dout, dq, dk, dv, dW1, dW2,
+                                dtau, scratch, status, s);
+    return launch_bwd<false>(p, q, k, v, W1, W2, tau, out, den, dout, dq, dk, dv, dW1, dW2,
+                             dtau, scratch, status, s);
 }
 
 }  // namespace flex

@@ -126,3 +126,34 @@ def test_tensor_core_forward_takes_the_prefactor(causal, launches):
     ro, _ = oracle.fwd(ins["q"], ins["k"], ins["v"], ins["W1"], ins["W2"], causal,
                        tau=ins["tau"])
     assert_close(to_host(out), ro, "bf16", "out")
+
+
+@pytest.mark.parametrize("w,M", [(WL[2], 128), (WL[1], 64)], ids=["n-M128", "s-M64"])
+def test_tensor_core_backward_takes_the_prefactor(w, M):
+    """Causal bf16 d = 64 keeps the tensor-core backward with tau: the key-weight pass, the
+    two-pass kernel, the dW/dtau reduction and the bf16 conversion (4 launches); the result
+    matches the oracle and repeats bit for bit."""
+    _, ins = _setup(w, True, 64, M, "bf16", N=520)
+    q, k, v, dO, W1, W2, tau = _dev(ins, "bf16")
+    out, den = flexattn.linattn_fwd(q, k, v, W1, W2, True, tau=tau)
+    shape = flexattn.shape_of(q, W1)
+    ws = flexattn.workspace(shape, True, True)
+    runs = []
+    for _ in range(2):
+        n0 = flexattn.kernel_launches()
+        g = flexattn.linattn_bwd(q, k, v, W1, W2, True, out, den, dO, ws=ws, tau=tau)
+        flexattn.check_status(ws)
+        assert flexattn.kernel_launches() - n0 == 4
+        runs.append([None if x is None else x.clone() for x in g])
+    for a, b in zip(*runs):
+        assert (a is None and b is None) or torch.equal(a, b), "not bit-exact repeatable"
+    r = oracle.bwd(ins["q"], ins["k"], ins["v"], ins["W1"], ins["W2"], True, ins["dO"],
+                   tau=ins["tau"])
+    g = runs[0]
+    for name, x, ref in zip(("dq", "dk", "dv", "dW1", "dW2"), g, r):
+        if ref is None:
+            continue
+        scale = 1.0 if name in ("dq", "dk", "dv") else float(np.sqrt(np.mean(ref * ref)))
+        assert_close(to_host(x), ref, "bf16", name, max_abs_scale=scale)
+    err = rel_l2(to_host(g[5]), r[5])
+    assert err <= 5e-2, f"dtau: rel L2 {err:.3e}"
