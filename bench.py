@@ -39,6 +39,7 @@ METRIC_DECODE = ("RFF linear-attn recurrent decode tokens/s (one new token per s
 L2_BYTES = 129e6
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+PREFACTOR = "exp(|x|^2 / exp(tau)), tau per head (workloads.draw_tau)"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -56,6 +57,9 @@ def parse_args():
                     help="comma-separated sequence lengths: time the workload's forward at "
                          "each N (same B, H, d, M) and print one JSON line per N with the "
                          "time and the device memory held (the linear-scaling curve)")
+    ap.add_argument("--prefactor", action="store_true",
+                    help="with the norm prefactor exp(|x|^2 / exp(tau)) of the paper's "
+                         "Flexformer_n, tau per head from the workload generator (both arms)")
     ap.add_argument("--batch", type=int, default=None,
                     help="run the workload with this batch B instead of its own (a smaller "
                          "case for profiling; the line's config names the changed workload)")
@@ -218,7 +222,7 @@ def cpu_cores():
         return os.cpu_count() or 1
 
 
-def oracle_sample(w, nseq, cores):
+def oracle_sample(w, nseq, cores, prefactor=False):
     """Time the oracle forward over the first `nseq` whole sequences of `w`."""
     import oracle
     nb = -(-nseq // w.H)
@@ -229,20 +233,21 @@ def oracle_sample(w, nseq, cores):
     heads = [s % w.H for s in range(nseq)]
     W1 = ins["W1"][heads]
     W2 = None if ins["W2"] is None else ins["W2"][heads]
+    tau = workloads.draw_tau(w)[heads] if prefactor else None
     t0 = time.perf_counter()
-    oracle.fwd(q, k, v, W1, W2, w.causal, nthreads=cores)
+    oracle.fwd(q, k, v, W1, W2, w.causal, nthreads=cores, tau=tau)
     return time.perf_counter() - t0
 
 
-def cpu_baseline(w, cores, target_s=12.0):
+def cpu_baseline(w, cores, target_s=12.0, prefactor=False):
     bh = w.B * w.H
     n1 = min(bh, cores)
-    t1 = oracle_sample(w, n1, cores)
+    t1 = oracle_sample(w, n1, cores, prefactor)
     nseq, t = n1, t1
     if t1 < target_s / 2 and n1 < bh:
         nseq = min(bh, n1 * max(1, int(target_s / max(t1, 1e-3))))
         if nseq > n1:
-            t = oracle_sample(w, nseq, cores)
+            t = oracle_sample(w, nseq, cores, prefactor)
     tokens = nseq * w.N / w.H
     return {"value": tokens / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
             "sample": f"{nseq} of {bh} whole (b,h) sequences of N={w.N} (fp64 C oracle, "
@@ -255,8 +260,9 @@ def run_reference(args, w):
         return
     if w.decode:
         for _ in range(args.warmup):
-            oracle_decode_sample(w, 1)
-        step = sum(oracle_decode_sample(w, 1) for _ in range(args.steps)) / args.steps
+            oracle_decode_sample(w, 1, args.prefactor)
+        step = sum(oracle_decode_sample(w, 1, args.prefactor)
+                   for _ in range(args.steps)) / args.steps
         value = w.B / step
         print(json.dumps({
             "metric": METRIC_DECODE, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
@@ -273,8 +279,8 @@ def run_reference(args, w):
     cores = cpu_cores()
     nseq = min(w.B * w.H, cores)
     for _ in range(args.warmup):
-        oracle_sample(w, nseq, cores)
-    times = [oracle_sample(w, nseq, cores) for _ in range(args.steps)]
+        oracle_sample(w, nseq, cores, args.prefactor)
+    times = [oracle_sample(w, nseq, cores, args.prefactor) for _ in range(args.steps)]
     step = sum(times) / len(times)
     value = nseq * w.N / w.H / step
     line = {
@@ -351,6 +357,8 @@ def run_ours(args, w):
     shape = flexattn.shape_of(q, W1)
     ws = flexattn.workspace(shape, w.causal, False, dev)
     stream = torch.cuda.current_stream()
+    tau = torch.from_numpy(workloads.draw_tau(w)).to(dev) if args.prefactor else None
+    dtau = torch.empty_like(tau) if args.prefactor else None
 
     if w.backward:  # a training step: forward, then backward of sum(dO * out)
         host["dO"] = torch.from_numpy(workloads.draw_activation(w, workloads.DO)).to(tdt).pin_memory()
@@ -360,9 +368,10 @@ def run_ours(args, w):
         ws_b = flexattn.workspace(shape, w.causal, True, dev)
 
     def step():
-        flexattn.linattn_fwd(q, k, v, W1, W2, w.causal, out=out, den=den, ws=ws)
+        flexattn.linattn_fwd(q, k, v, W1, W2, w.causal, out=out, den=den, ws=ws, tau=tau)
         if w.backward:
-            flexattn.linattn_bwd(q, k, v, W1, W2, w.causal, out, den, dO, *grads, ws=ws_b)
+            flexattn.linattn_bwd(q, k, v, W1, W2, w.causal, out, den, dO, *grads, ws=ws_b,
+                                 tau=tau, dtau=dtau)
 
     for _ in range(max(3, args.warmup)):
         step()
@@ -432,12 +441,13 @@ def run_ours(args, w):
 
     peaks, peaks_src = load_peaks()
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    roof = roofline(w, kernel_ms, peaks, sms, recorded_traffic(w))
+    # the recorded DRAM traffic is that of the kernel without the prefactor
+    roof = roofline(w, kernel_ms, peaks, sms, None if args.prefactor else recorded_traffic(w))
     roof["peak_source"] = peaks_src
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(w, cpu_cores())
+        cpu = cpu_baseline(w, cpu_cores(), prefactor=args.prefactor)
 
     if rank == 0:
         line = {
@@ -450,7 +460,8 @@ def run_ours(args, w):
                        "variant": w.variant, "causal": w.causal,
                        "l2": f"inputs {3 * w.token_heads * w.d * elem_bytes(w) / 1e6:.0f} MB "
                              f"> L2 {L2_BYTES / 1e6:.0f} MB, no flush",
-                       "parallelism": f"replicas x{world}"},
+                       "parallelism": f"replicas x{world}",
+                       "prefactor": PREFACTOR if args.prefactor else None},
             "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
             "gpu_launches": launches,
         }
@@ -475,7 +486,7 @@ def decode_work(w):
     return nbytes, flops, ops
 
 
-def oracle_decode_sample(w, steps):
+def oracle_decode_sample(w, steps, prefactor=False):
     """Seconds per oracle decode step of all B x H sequences (the first token)."""
     import numpy as np
     import oracle
@@ -484,9 +495,10 @@ def oracle_decode_sample(w, steps):
     W1, W2 = ins["W1"], ins["W2"]
     S = np.zeros((w.B, w.H, 2 * w.M, w.d))
     z = np.zeros((w.B, w.H, 2 * w.M))
+    tau = workloads.draw_tau(w) if prefactor else None
     t0 = time.perf_counter()
     for _ in range(steps):
-        _, _, S, z = oracle.decode(q, k, v, W1, W2, S, z)
+        _, _, S, z = oracle.decode(q, k, v, W1, W2, S, z, tau=tau)
     return (time.perf_counter() - t0) / steps
 
 
@@ -519,6 +531,7 @@ def run_decode(args, w):
     del ins
     S, z = flexattn.decode_state(w.B, w.H, w.M, w.d, dev)
     ws = flexattn.decode_workspace(w.B, w.H, w.M, w.d, dev)
+    tau = torch.from_numpy(workloads.draw_tau(w)).to(dev) if args.prefactor else None
     out = torch.empty_like(toks[0][0])
     den = torch.empty(w.B, w.H, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
@@ -527,7 +540,7 @@ def run_decode(args, w):
     def step(tk=None):
         q, k, v = tk if tk is not None else toks[it[0] % w.N]
         it[0] += 1
-        flexattn.linattn_decode(q, k, v, W1, W2, S, z, out=out, den=den, ws=ws)
+        flexattn.linattn_decode(q, k, v, W1, W2, S, z, out=out, den=den, ws=ws, tau=tau)
 
     def barrier():
         if world > 1:
@@ -593,7 +606,7 @@ def run_decode(args, w):
     sec = kernel_ms * 1e-3
     roof = {"bound": "hbm", "achieved": nbytes / sec / 1e9, "peak": peaks["hbm_gbs"],
             "unit": "GB/s", "frac": nbytes / sec / 1e9 / peaks["hbm_gbs"],
-            "traffic": recorded_traffic(w),
+            "traffic": None if args.prefactor else recorded_traffic(w),
             "peak_source": peaks_src, "algorithmic_bytes_per_launch": nbytes,
             "fracs": {"hbm": nbytes / sec / 1e9 / peaks["hbm_gbs"],
                       "tensor": flops / sec / 1e12 / peaks["bf16_tflops"]},
@@ -601,7 +614,7 @@ def run_decode(args, w):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        t = oracle_decode_sample(w, 3)
+        t = oracle_decode_sample(w, 3, args.prefactor)
         cpu = {"value": w.B / t, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                "sample": f"3 decode steps of all {w.B}x{w.H} sequences (fp64 C oracle, "
                          f"one thread), {t:.3f} s per step"}
@@ -616,7 +629,8 @@ def run_decode(args, w):
                        "variant": w.variant, "causal": True,
                        "l2": f"state {w.B * w.H * 2 * w.M * (w.d + 1) * 4 / 1e6:.0f} MB > L2 "
                              f"{L2_BYTES / 1e6:.0f} MB, no flush",
-                       "parallelism": f"replicas x{world}"},
+                       "parallelism": f"replicas x{world}",
+                       "prefactor": PREFACTOR if args.prefactor else None},
             "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
             "gpu_launches": launches,
         }

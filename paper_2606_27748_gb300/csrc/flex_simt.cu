@@ -570,6 +570,45 @@ __global__ void __launch_bounds__(kThreads) key_weights_kernel(Problem p, const 
     }
 }
 
+// The same for bf16 rows of d = 64 (the tensor-core shapes): 8 lanes per row, one 16-byte
+// load each (fully coalesced), 4 rows in flight per lane, the 8 partial sums combined by
+// xor shuffles.
+__global__ void __launch_bounds__(kThreads) key_weights_bf16_d64_kernel(Problem p,
+                                                                         const __nv_bfloat16* k,
+                                                                         const float* tau,
+                                                                         float* kw)
+{
+    constexpr int kUnroll = 4;
+    const size_t rows = (size_t)p.B * p.H * p.N;
+    const int lane = threadIdx.x & 31, sub = lane & 7;
+    const size_t warps = (size_t)gridDim.x * (blockDim.x / 32);
+    const size_t gw = (size_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+    for (size_t r0 = gw * 4 * kUnroll; r0 < rows; r0 += warps * 4 * kUnroll) {
+        uint4 x[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const size_t r = r0 + 4 * u + (lane >> 3);
+            x[u] = r < rows ? *reinterpret_cast<const uint4*>(k + r * 64 + 8 * sub)
+                            : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const uint32_t wv[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
+            float n2 = 0.f;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float a = __uint_as_float(wv[e] << 16), b = __uint_as_float(wv[e] & 0xffff0000u);
+                n2 = fmaf(a, a, fmaf(b, b, n2));
+            }
+            n2 += __shfl_xor_sync(0xffffffffu, n2, 1);
+            n2 += __shfl_xor_sync(0xffffffffu, n2, 2);
+            n2 += __shfl_xor_sync(0xffffffffu, n2, 4);
+            const size_t r = r0 + 4 * u + (lane >> 3);
+            if (sub == 0 && r < rows) kw[r] = expf(n2 * expf(-tau[(r / p.N) % p.H]));
+        }
+    }
+}
+
 // dW over the batch, in a fixed order (deterministic).  Nonstationary: the partials hold
 // dU (rows < M) and dV (rows >= M); dW1 = (dU + dV)/2, dW2 = (dU - dV)/2.
 __global__ void dw_reduce_kernel(Problem p, const float* part, float* dW1, float* dW2,
@@ -643,6 +682,12 @@ cudaError_t launch_key_weights(const Problem& p, const void* k, const float* tau
                                cudaStream_t s)
 {
     const size_t rows = (size_t)p.B * p.H * p.N;
+    if (p.bf16 && p.d == 64) {  // 16 rows per warp and iteration, 8 warps per block
+        const int blocks = (int)std::min<size_t>((rows + 127) / 128, 152 * 16);
+        key_weights_bf16_d64_kernel<<<blocks, kThreads, 0, s>>>(p, (const __nv_bfloat16*)k, tau,
+                                                                 kw);
+        return cudaGetLastError();
+    }
     const int blocks = (int)std::min<size_t>((rows + kThreads - 1) / kThreads, 152 * 16);
     if (p.bf16)
         key_weights_kernel<<<blocks, kThreads, 0, s>>>(p, (const __nv_bfloat16*)k, tau, kw);
