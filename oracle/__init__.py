@@ -10,7 +10,8 @@ Contents
     (Eq. phi_n, Flexformer_s) and nonstationary (Eq. phi_non, Flexformer_n) feature maps,
     forward and analytic backward, in plain fp64 C loops.  Loaded here through ctypes.
   * ``brute.py`` -- the explicit N x N kernel-matrix form of Eq. (attention) with
-    sim(q, k) = phi(q) . phi(k) (Eq. kernel), written independently in numpy.
+    sim(q, k) = phi(q) . phi(k) (Eq. kernel), written independently in numpy, and the
+    distillation loss written with explicit matrices.
 
 Every function takes and returns float64 numpy arrays in the layouts
 q, k, v, out: [B, H, N, d];  W1, W2: [H, M, d];  den: [B, H, N];  phi: [B, H, N, 2M].
@@ -70,8 +71,9 @@ class Oracle:
                                            dp, dp, dp, dp, i]
         lib.oracle_linattn_decode.argtypes = [i, i, i, i, dp, dp, dp, dp, dp, dp, dp, dp, dp,
                                               dp]
+        lib.oracle_awd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, i, dp]
         for fn in (lib.oracle_featmap, lib.oracle_featmap_sumform, lib.oracle_linattn_fwd,
-                   lib.oracle_linattn_bwd, lib.oracle_linattn_decode):
+                   lib.oracle_linattn_bwd, lib.oracle_linattn_decode, lib.oracle_awd):
             fn.restype = ctypes.c_int
         self._lib = lib
         self.path = path
@@ -167,6 +169,21 @@ class Oracle:
         return out, den, S, z
 
 
+    def awd(self, q, k, W1, W2=None, causal=False, tau=None):
+        """Attention-weight distillation loss of every sequence, [B, H]: the cross-entropy
+        of the kernel's normalised weights against softmax(q k^T / sqrt(d)), averaged over
+        the queries (entries with a non-positive kernel estimate count log 1e-6)."""
+        q, k, W1, W2, tau = (self._f64(a) for a in (q, k, W1, W2, tau))
+        B, H, N, d = q.shape
+        M = W1.shape[1]
+        loss = np.empty((B, H))
+        rc = self._lib.oracle_awd(B, H, N, d, M, self._p(q), self._p(k), self._p(W1),
+                                  self._p(W2), self._p(tau), int(bool(causal)), self._p(loss))
+        if rc != 0:
+            raise ValueError("oracle_awd: bad shape")
+        return loss
+
+
 def load() -> Oracle:
     """The oracle built from ``flex_oracle.c`` (compiled on first use if needed)."""
     global _lib
@@ -192,3 +209,7 @@ def bwd(q, k, v, W1, W2, causal, dout, nthreads=None, tau=None):
 
 def decode(q, k, v, W1, W2, S, z, tau=None):
     return load().decode(q, k, v, W1, W2, S, z, tau)
+
+
+def awd(q, k, W1, W2=None, causal=False, tau=None):
+    return load().awd(q, k, W1, W2, causal, tau)

@@ -59,3 +59,25 @@ def attention(q, k, v, W1, W2=None, causal=True, tau=None):
     den = K.sum(axis=-1)
     out = np.einsum("...ij,...je->...ie", K, np.asarray(v, dtype=np.float64)) / den[..., None]
     return out, den
+
+
+def awd_loss(q, k, W1, W2=None, causal=False, tau=None, eps=1e-6):
+    """Attention-weight distillation loss per sequence [..., H] with explicit N x N
+    matrices: P = softmax(q k^T / sqrt(d)) (masked when causal), R = K~ / rowsum(K~) with
+    the prefactored kernel K~ as printed (query and key factors), and
+    L = -mean_i sum_j P_ij log R_ij; entries with R_ij <= 0 count log(eps)."""
+    q = np.asarray(q, dtype=np.float64)
+    k = np.asarray(k, dtype=np.float64)
+    d = q.shape[-1]
+    s = np.einsum("...id,...jd->...ij", q, k) / np.sqrt(d)
+    K = kernel_matrix(q, k, W1, W2, tau)
+    N = K.shape[-1]
+    mask = np.tril(np.ones((N, N), dtype=bool)) if causal else np.ones((N, N), dtype=bool)
+    s = np.where(mask, s, -np.inf)
+    P = np.exp(s - s.max(axis=-1, keepdims=True))
+    P = P / P.sum(axis=-1, keepdims=True)
+    K = np.where(mask, K, 0.0)
+    R = K / K.sum(axis=-1, keepdims=True)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        logR = np.where(R > 0, np.log(np.where(R > 0, R, 1.0)), np.log(eps))
+    return -np.sum(np.where(mask, P * logR, 0.0), axis=(-1, -2)) / N

@@ -445,6 +445,72 @@ int oracle_linattn_bwd(int B, int H, int N, int d, int M, const double* q, const
     return 0;
 }
 
+/* ------------------------------------------------------------------------------------ */
+/* Attention-weight distillation loss (the loss of the softmax-recovery experiments, the   */
+/* appendix's distillation setting): per query i, the teacher distribution                 */
+/* P_ij = softmax_j(q_i . k_j / sqrt(d)) and the kernel's normalised weights               */
+/* R_ij = A~_ij / D_i with A~_ij = phi~(q_i) . phi~(k_j), D_i = sum_l A~_il; the loss of   */
+/* a sequence is L = -(1/N) sum_i sum_j P_ij log R_ij (j over all keys, or j <= i when     */
+/* causal).  The query's prefactor and the global scale cancel in R, so A~_ij =            */
+/* w_j phi(q_i) . phi(k_j) with the key weight of the norm prefactor (w = 1 without tau).  */
+/* Reading: RFF estimates can be negative, and so can a row sum D_i; an entry whose        */
+/* normalised weight R_ij = A~_ij / D_i is not positive has no logarithm and contributes    */
+/* log(AWD_EPS) and no gradient.                                                            */
+/* ------------------------------------------------------------------------------------ */
+#define AWD_EPS 1e-6
+
+static double awd_seq(int N, int d, int M, int causal, const double* q, const double* k,
+                      const double* W1, const double* W2, double itau)
+{
+    const int D = 2 * M;
+    double* PQ = malloc(sizeof(double) * (size_t)N * D);
+    double* PK = malloc(sizeof(double) * (size_t)N * D);
+    double* sc = malloc(sizeof(double) * (size_t)N);
+    double* at = malloc(sizeof(double) * (size_t)N);
+    for (int i = 0; i < N; ++i) {
+        feature(d, M, q + (size_t)i * d, W1, W2, PQ + (size_t)i * D);
+        feature(d, M, k + (size_t)i * d, W1, W2, PK + (size_t)i * D);
+        const double wk = key_weight(d, k + (size_t)i * d, itau);
+        for (int f = 0; f < D; ++f) PK[(size_t)i * D + f] *= wk;
+    }
+    double loss = 0.0;
+    for (int i = 0; i < N; ++i) {
+        const int J = causal ? i + 1 : N;
+        double smax = -INFINITY, Dn = 0.0;
+        for (int j = 0; j < J; ++j) {
+            sc[j] = dot(d, q + (size_t)i * d, k + (size_t)j * d) / sqrt((double)d);
+            at[j] = dot(D, PQ + (size_t)i * D, PK + (size_t)j * D);
+            if (sc[j] > smax) smax = sc[j];
+            Dn += at[j];
+        }
+        double Z = 0.0, ce = 0.0;
+        for (int j = 0; j < J; ++j) Z += exp(sc[j] - smax);
+        for (int j = 0; j < J; ++j) {
+            const double Pij = exp(sc[j] - smax) / Z;
+            const double r = at[j] / Dn;
+            ce -= Pij * (r > 0.0 ? log(r) : log(AWD_EPS));
+        }
+        loss += ce;
+    }
+    free(PQ); free(PK); free(sc); free(at);
+    return loss / N;
+}
+
+/* loss [B][H]: the distillation loss of every (b, h) sequence; tau [H] or NULL. */
+int oracle_awd(int B, int H, int N, int d, int M, const double* q, const double* k,
+               const double* W1, const double* W2, const double* tau, int causal,
+               double* loss)
+{
+    if (bad_shape(B, H, N, d, M)) return -1;
+    for (int b = 0; b < B; ++b)
+        for (int h = 0; h < H; ++h) {
+            const size_t u = (size_t)b * H + h, off = u * N * d;
+            loss[u] = awd_seq(N, d, M, causal, q + off, k + off, W1 + (size_t)h * M * d,
+                              W2 ? W2 + (size_t)h * M * d : NULL, tau ? exp(-tau[h]) : 0.0);
+        }
+    return 0;
+}
+
 /* One step of the causal recurrence behind Eq. (linear att) with j <= i: the running sums
  * S = sum_j phi(k_j) v_j^T and z = sum_j phi(k_j) absorb the new token (inclusive), then
  * out = phi(q)^T S / den with den = phi(q)^T z.  Per (b, h): q, k, v, out [d]; S [2M][d]

@@ -29,6 +29,10 @@ Facts used (none is the oracle's own formula retyped):
     vanishes as tau grows; keys of equal norm make it a common factor (O unchanged);
     finite differences (dq, dk, dv, dW, dtau); the scaling identity
     <dW, W> = sum <dq, q> + <dk, k> + 2 dtau (x -> l x, W -> W / l, tau -> tau + 2 ln l).
+  * the distillation loss: the C loss equals the explicit-matrix numpy form; one key gives
+    0; d = 1, M = 1 in closed form (cos kernel, softmax teacher); Gibbs' inequality
+    (loss >= the teacher's entropy); keys of equal norm make tau irrelevant; entries with
+    a non-positive normalised weight count log 1e-6 in both forms.
 """
 from __future__ import annotations
 
@@ -326,6 +330,75 @@ def pin_prefactor_decode(orc):
             assert _rel(out, bo[:, :, i]) < 1e-11, f"prefactor decode {variant} i={i}"
 
 
+# -------------------------------------------------------------------------------------
+# Attention-weight distillation loss (the appendix's distillation setting).
+# -------------------------------------------------------------------------------------
+def pin_awd_equals_brute(orc):
+    """The C loss equals the numpy form with explicit P and R, the prefactor on queries
+    and keys as printed (so the query factor's cancellation is checked too)."""
+    for variant in ("s", "n"):
+        for causal in (False, True):
+            for N in (1, 3, 17, 64):
+                for tau in (None, _TAU):
+                    q, k, _, W1, W2 = _case(70 + N, 2, 2, N, 5, 7, variant)
+                    a = orc.awd(q, k, W1, W2, causal, tau=tau)
+                    b = brute.awd_loss(q, k, W1, W2, causal, tau=tau)
+                    assert _rel(a, b) < 1e-12, f"awd {variant} causal={causal} N={N}"
+
+
+def pin_awd_single_key(orc):
+    """One key: P = R = 1, so the loss is 0 exactly; causally the first query adds 0."""
+    q, k, _, W1, W2 = _case(71, 2, 2, 1, 5, 7, "n")
+    assert np.all(orc.awd(q, k, W1, W2) == 0.0), "awd N=1"
+
+
+def pin_awd_closed_form_d1(orc):
+    """d = 1, M = 1, stationary: A_ij is proportional to cos(w (q_i - k_j)) and the teacher
+    is softmax_j(q_i k_j)."""
+    q = np.array([0.3, -0.4, 0.2, 0.5]).reshape(1, 1, 4, 1)
+    k = np.array([0.1, 0.25, -0.3, 0.0]).reshape(1, 1, 4, 1)
+    w = 0.7
+    L = orc.awd(q, k, np.array([[[w]]]), None, causal=False)[0, 0]
+    qq, kk = q.reshape(4, 1), k.reshape(1, 4)
+    P = np.exp(qq * kk) / np.exp(qq * kk).sum(axis=1, keepdims=True)
+    A = np.cos(w * (qq - kk))
+    R = A / A.sum(axis=1, keepdims=True)
+    assert abs(L - (-np.sum(P * np.log(R)) / 4)) < 1e-14, "awd closed form"
+
+
+def pin_awd_gibbs(orc):
+    """Cross-entropy >= entropy: L >= mean_i H(P_i) (all kernel entries positive here)."""
+    for variant in ("s", "n"):
+        for causal in (False, True):
+            q, k, _, W1, W2 = _case(72, 2, 3, 29, 6, 9, variant)
+            L = orc.awd(q, k, W1, W2, causal)
+            s = np.einsum("bhid,bhjd->bhij", q, k) / np.sqrt(6)
+            if causal:
+                s = np.where(np.tril(np.ones((29, 29), bool)), s, -np.inf)
+            P = np.exp(s - s.max(-1, keepdims=True))
+            P /= P.sum(-1, keepdims=True)
+            Hp = -np.sum(np.where(P > 0, P * np.log(np.where(P > 0, P, 1.0)), 0.0), axis=(-1, -2)) / 29
+            assert np.all(L >= Hp - 1e-12), "awd below the teacher's entropy"
+
+
+def pin_awd_equal_key_norms(orc):
+    """Keys of one norm make the prefactor a common factor of R: the loss is unchanged."""
+    q, k, _, W1, W2 = _case(73, 2, 2, 21, 5, 7, "n")
+    k = k / np.linalg.norm(k, axis=-1, keepdims=True) * 1.1
+    assert _rel(orc.awd(q, k, W1, W2, tau=_TAU), orc.awd(q, k, W1, W2)) < 1e-13, "awd tau"
+
+
+def pin_awd_nonpositive_entries(orc):
+    """Large frequencies and few of them make some kernel estimates and some row sums
+    negative; entries with a non-positive normalised weight count log 1e-6, as in the
+    numpy form."""
+    q, k, _, W1, W2 = _case(74, 1, 2, 23, 5, 3, "s", qk_scale=2.0)
+    W1 = W1 * 4.0
+    K = brute.kernel_matrix(q, k, W1)
+    assert np.any(K <= 0) and np.any(K.sum(-1) < 0), "the case needs both kinds"
+    assert _rel(orc.awd(q, k, W1), brute.awd_loss(q, k, W1)) < 1e-12, "awd clamp"
+
+
 ALL_PINS = [
     pin_origin_features, pin_stationary_unit_norm, pin_sum_to_product, pin_w2_equals_w1,
     pin_bochner, pin_yaglom, pin_linear_equals_brute, pin_decode_equals_brute,
@@ -334,4 +407,6 @@ ALL_PINS = [
     pin_gradient_invariants, pin_prefactor_linear_equals_brute,
     pin_prefactor_vanishes_as_tau_grows, pin_prefactor_equal_key_norms,
     pin_prefactor_finite_differences, pin_prefactor_scaling_identity, pin_prefactor_decode,
+    pin_awd_equals_brute, pin_awd_single_key, pin_awd_closed_form_d1, pin_awd_gibbs,
+    pin_awd_equal_key_norms, pin_awd_nonpositive_entries,
 ]

@@ -53,6 +53,13 @@ MUTATIONS = [
      "for (int f = 0; f < F; ++f) pk[f] *= 1.0;", 0),
     ("prefactor_noncausal_unweighted", "for (int f = 0; f < D; ++f) pk[f] *= wj;",
      "for (int f = 0; f < D; ++f) pk[f] *= 1.0;", 0),
+    ("awd_teacher_without_sqrt_d", "/ sqrt((double)d);", "/ 1.0;", 0),
+    ("awd_unnormalised_kernel", "const double r = at[j] / Dn;", "const double r = at[j];", 0),
+    ("awd_causal_mask_exclusive", "const int J = causal ? i + 1 : N;",
+     "const int J = causal ? (i > 0 ? i : 1) : N;", 0),
+    ("awd_unweighted_keys", "for (int f = 0; f < D; ++f) PK[(size_t)i * D + f] *= wk;\n    }\n    double loss",
+     "for (int f = 0; f < D; ++f) PK[(size_t)i * D + f] *= 1.0;\n    }\n    double loss", 0),
+    ("awd_clamp_value", "log(AWD_EPS)", "log(1e-3)", 0),
 ]
 
 
