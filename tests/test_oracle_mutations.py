@@ -59,7 +59,7 @@ MUTATIONS = [
      "const int J = causal ? (i > 0 ? i : 1) : N;", 0),
     ("awd_unweighted_keys", "for (int f = 0; f < D; ++f) PK[(size_t)i * D + f] *= wk;\n    }\n    double loss",
      "for (int f = 0; f < D; ++f) PK[(size_t)i * D + f] *= 1.0;\n    }\n    double loss", 0),
-    ("awd_clamp_value", "log(AWD_EPS)", "log(1e-3)", 0),
+    ("awd_clamp_value", "(r > 0.0 ? log(r) : log(AWD_EPS))", "(r > 0.0 ? log(r) : log(1e-3))", 0),
 ]
 
 
