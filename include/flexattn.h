@@ -153,6 +153,27 @@ int flex_linattn_decode(const flex_shape* shape, const void* q, const void* k, c
                         float* z, void* out, float* den, void* ws, size_t ws_bytes,
                         void* stream);
 
+/* Workspace bytes needed by flex_awd_loss for this shape; 0 if the shape is invalid or
+ * unsupported. */
+size_t flex_awd_workspace_bytes(const flex_shape* shape);
+
+/* Attention-weight distillation loss (the loss of the paper's softmax-recovery
+ * experiments, appendix "Attention Distillation Setting"): for every (b, h) sequence
+ *   loss[b][h] = -(1/N) sum_i sum_j P_ij log R_ij,
+ *   P_ij = softmax_j(q_i . k_j / sqrt(d))               (the teacher: softmax attention),
+ *   R_ij = A~_ij / sum_l A~_il,  A~_ij = phi~(q_i) . phi~(k_j)   (this kernel's weights),
+ * j over all keys, or j <= i when causal; phi~ is the feature map above with the optional
+ * norm prefactor tau ([H] fp32 or NULL).  An entry whose R_ij is not positive (random
+ * Fourier estimates and row sums can be negative) counts log(1e-6).  Computed blockwise
+ * (128 x 128 tiles of scores and kernel values on the tensor cores, online softmax), never
+ * materialising the N x N matrices.  q, k: [B][H][N][d] bf16 (d = 64, M in {64, 128});
+ * loss: [B][H] fp32, overwritten.  ws: workspace of flex_awd_workspace_bytes() bytes.
+ * Launches 4 kernels (5 with tau).  Errors: FLEX_EINVAL for NULL or misaligned pointers,
+ * FLEX_EUNSUPPORTED for other shapes or fp32 storage, FLEX_EWORKSPACE. */
+int flex_awd_loss(const flex_shape* shape, const void* q, const void* k, const float* W1,
+                  const float* W2, const float* tau, int causal, float* loss, void* ws,
+                  size_t ws_bytes, void* stream);
+
 /* Cumulative number of kernels this library has enqueued in this process (all entry
  * points, all devices).  Lets a caller count the launches inside a timed region. */
 unsigned long long flex_kernel_launches(void);

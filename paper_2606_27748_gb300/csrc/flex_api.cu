@@ -194,6 +194,55 @@ int flex_linattn_decode(const flex_shape* shape, const void* q, const void* k, c
                                         (char*)ws + header_bytes(), (cudaStream_t)stream));
 }
 
+// Distillation-loss workspace: header, phi(q), phi~(k) [B*H*N][2M] bf16, key weights
+// [B*H*N] fp32, partial sums [B*H][query blocks] fp32.
+struct AwdWs {
+    size_t pq, pk, kw, part, total;
+};
+AwdWs awd_ws(const Problem& p)
+{
+    const size_t rows = (size_t)p.B * p.H * p.N, feat = flex::align_up(rows * 2 * p.M * 2, 256);
+    AwdWs w;
+    w.pq = header_bytes();
+    w.pk = w.pq + feat;
+    w.kw = w.pk + feat;
+    w.part = w.kw + flex::align_up(rows * sizeof(float), 256);
+    w.total = w.part + flex::align_up(flex::tc_awd_part_floats(p) * sizeof(float), 256);
+    return w;
+}
+
+size_t flex_awd_workspace_bytes(const flex_shape* shape)
+{
+    Problem p;
+    if (make_problem(shape, nullptr, 0, &p) != FLEX_OK || !flex::tc_awd_supported(p)) return 0;
+    return awd_ws(p).total;
+}
+
+int flex_awd_loss(const flex_shape* shape, const void* q, const void* k, const float* W1,
+                  const float* W2, const float* tau, int causal, float* loss, void* ws,
+                  size_t ws_bytes, void* stream)
+{
+    Problem p;
+    int rc = make_problem(shape, W2, causal, &p);
+    if (rc) return rc;
+    if (!q || !k || !W1 || !loss) return FLEX_EINVAL;
+    for (const void* t : {q, k, (const void*)W1, (const void*)loss})
+        if (!aligned(t, 16)) return FLEX_EINVAL;
+    if ((W2 && !aligned(W2, 16)) || (tau && !aligned(tau, 4))) return FLEX_EINVAL;
+    if (!flex::tc_awd_supported(p)) return FLEX_EUNSUPPORTED;
+    const AwdWs w = awd_ws(p);
+    if ((rc = check_ws(ws, ws_bytes, w.total))) return rc;
+    cudaStream_t s = (cudaStream_t)stream;
+    char* base = (char*)ws;
+    float* kw = tau ? (float*)(base + w.kw) : nullptr;
+    if (tau && (rc = count(1, flex::launch_key_weights(p, k, tau, kw, s)))) return rc;
+    if ((rc = count(1, flex::launch_featmap_scaled(p, q, W1, W2, nullptr, base + w.pq, s))))
+        return rc;
+    if ((rc = count(1, flex::launch_featmap_scaled(p, k, W1, W2, kw, base + w.pk, s)))) return rc;
+    return count(2, flex::launch_tc_awd(p, q, k, base + w.pq, base + w.pk, (float*)(base + w.part),
+                                        loss, &((flex::WsHeader*)ws)->status, s));
+}
+
 unsigned long long flex_kernel_launches(void) { return g_launches.load(); }
 
 int flex_check_status(void* ws, void* stream)

@@ -38,6 +38,10 @@ size_t simt_bwd_ws_bytes(const Problem& p);
 
 cudaError_t launch_featmap(const Problem& p, const void* x, const float* W1, const float* W2,
                            void* phi, cudaStream_t s);
+// phi times rowscale[row] (rowscale [B*H*N] or NULL)
+cudaError_t launch_featmap_scaled(const Problem& p, const void* x, const float* W1,
+                                  const float* W2, const float* rowscale, void* phi,
+                                  cudaStream_t s);
 // tau: per-head norm prefactor (Sec. 3.2) or NULL; dtau with it in the backward.
 cudaError_t launch_simt_fwd(const Problem& p, const void* q, const void* k, const void* v,
                             const float* W1, const float* W2, const float* tau, void* out,
@@ -81,5 +85,12 @@ cudaError_t launch_tc_bwd(const Problem& p, const void* q, const void* k, const 
                           const float* den, const void* dout, void* dq, void* dk, void* dv,
                           float* dW1, float* dW2, float* dtau, void* scratch, int* status,
                           cudaStream_t s);
+
+// ---- attention-weight distillation loss (tensor cores: bf16, d = 64, M in {64, 128}) ---
+bool tc_awd_supported(const Problem& p);
+size_t tc_awd_part_floats(const Problem& p);  // partial slots [B*H][query blocks]
+// pq, pk: phi(q) and the key-weighted phi(k), [B*H][N][2M] bf16; loss [B*H] fp32
+cudaError_t launch_tc_awd(const Problem& p, const void* q, const void* k, const void* pq,
+                          const void* pk, float* part, float* loss, int* status, cudaStream_t s);
 
 }  // namespace flex

@@ -99,7 +99,7 @@ __device__ void features(const Problem& p, const float* X, int rows, const float
 // ------------------------------------------------------------------------------------
 template <typename T>
 __global__ void featmap_kernel(Problem p, const T* x, const float* W1, const float* W2, T* phi,
-                               float scale)
+                               float scale, const float* rowscale)
 {
     const int d = p.d, M = p.M;
     const size_t rows = (size_t)p.B * p.H * p.N;
@@ -122,9 +122,9 @@ __global__ void featmap_kernel(Problem p, const T* x, const float* W1, const flo
         }
         float sa, ca;
         sincosf(a, &sa, &ca);
-        float cw = p.nonstat ? cosf(w) : 1.f;
-        store_act(phi, row * 2 * M + m, scale * ca * cw);
-        store_act(phi, row * 2 * M + M + m, scale * sa * cw);
+        float cw = (p.nonstat ? cosf(w) : 1.f) * scale * (rowscale ? rowscale[row] : 1.f);
+        store_act(phi, row * 2 * M + m, ca * cw);
+        store_act(phi, row * 2 * M + M + m, sa * cw);
     }
 }
 
@@ -699,15 +699,22 @@ cudaError_t launch_key_weights(const Problem& p, const void* k, const float* tau
 cudaError_t launch_featmap(const Problem& p, const void* x, const float* W1, const float* W2,
                            void* phi, cudaStream_t s)
 {
+    return launch_featmap_scaled(p, x, W1, W2, nullptr, phi, s);
+}
+
+cudaError_t launch_featmap_scaled(const Problem& p, const void* x, const float* W1,
+                                  const float* W2, const float* rowscale, void* phi,
+                                  cudaStream_t s)
+{
     const size_t work = (size_t)p.B * p.H * p.N * p.M;
     const int blocks = (int)std::min<size_t>((work + kThreads - 1) / kThreads, 152 * 16);
     const float scale = 1.0f / sqrtf((float)p.M);
     if (p.bf16)
         featmap_kernel<<<blocks, kThreads, 0, s>>>(p, (const __nv_bfloat16*)x, W1, W2,
-                                                   (__nv_bfloat16*)phi, scale);
+                                                   (__nv_bfloat16*)phi, scale, rowscale);
     else
         featmap_kernel<<<blocks, kThreads, 0, s>>>(p, (const float*)x, W1, W2, (float*)phi,
-                                                   scale);
+                                                   scale, rowscale);
     return cudaGetLastError();
 }
 

@@ -99,6 +99,22 @@ inline bool make_act_map(CUtensorMap* m, const void* base, int BH, int N)
            CUDA_SUCCESS;
 }
 
+// [BH][N][F] bf16 rows of F features (F a multiple of 64), box 64 x 128, 128B swizzle:
+// a load at x = 64 g brings feature block g of 128 rows.
+inline bool make_feat_map(CUtensorMap* m, const void* base, int BH, int N, int F)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)F, (cuuint64_t)N, (cuuint64_t)BH};
+    cuuint64_t strides[2] = {(cuuint64_t)F * 2, (cuuint64_t)N * F * 2};
+    cuuint32_t box[3] = {64, 128, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+               box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
+}
+
 inline int sm_count()
 {
     int dev = 0, n = 0;

@@ -22,7 +22,7 @@ FLEX_OK, FLEX_EINVAL, FLEX_EUNSUPPORTED, FLEX_EWORKSPACE, FLEX_ECUDA, FLEX_ETIME
 
 EXPORTS = ("flex_strerror", "flex_workspace_bytes", "flex_featmap", "flex_linattn_fwd",
            "flex_linattn_bwd", "flex_decode_workspace_bytes", "flex_linattn_decode",
-           "flex_kernel_launches",
+           "flex_awd_workspace_bytes", "flex_awd_loss", "flex_kernel_launches",
            "flex_check_status")
 
 
@@ -65,11 +65,14 @@ def load(path: str = LIBRARY) -> ctypes.CDLL:
         lib.flex_decode_workspace_bytes.restype = sz
         lib.flex_linattn_decode.argtypes = [shp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp,
                                             sz, vp]
+        lib.flex_awd_workspace_bytes.argtypes = [shp]
+        lib.flex_awd_workspace_bytes.restype = sz
+        lib.flex_awd_loss.argtypes = [shp, vp, vp, vp, vp, vp, ip, vp, vp, sz, vp]
         lib.flex_check_status.argtypes = [vp, vp]
         lib.flex_kernel_launches.argtypes = []
         lib.flex_kernel_launches.restype = ctypes.c_ulonglong
         for fn in (lib.flex_featmap, lib.flex_linattn_fwd, lib.flex_linattn_bwd,
-                   lib.flex_linattn_decode, lib.flex_check_status):
+                   lib.flex_linattn_decode, lib.flex_awd_loss, lib.flex_check_status):
             fn.restype = ip
         _lib = lib
         return lib
@@ -211,6 +214,28 @@ def linattn_decode(q, k, v, W1, W2, S, z, out=None, den=None, want_den=True, ws=
                                       _ptr(den), _ptr(ws), ws.numel(), _stream(stream)),
            "flex_linattn_decode")
     return out, den
+
+
+def awd_workspace(shape: FlexShape, device=None) -> torch.Tensor:
+    """A caller-owned workspace for flex_awd_loss."""
+    n = int(load().flex_awd_workspace_bytes(ctypes.byref(shape)))
+    if n == 0:
+        raise FlexError(FLEX_EUNSUPPORTED, "flex_awd_workspace_bytes")
+    return torch.zeros(n, dtype=torch.uint8, device=device or "cuda")
+
+
+def awd_loss(q, k, W1, W2=None, causal=False, tau=None, loss=None, ws=None, stream=None):
+    """Attention-weight distillation loss of every sequence, [B, H] fp32: the cross-entropy
+    of this kernel's normalised attention weights against softmax(q k^T / sqrt(d))."""
+    shape = shape_of(q, W1)
+    if loss is None:
+        loss = torch.empty(q.shape[:2], dtype=torch.float32, device=q.device)
+    if ws is None:
+        ws = awd_workspace(shape, q.device)
+    _check(load().flex_awd_loss(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(W1), _ptr(W2),
+                                _ptr(tau), int(bool(causal)), _ptr(loss), _ptr(ws),
+                                ws.numel(), _stream(stream)), "flex_awd_loss")
+    return loss
 
 
 def check_status(ws, stream=None):

@@ -110,3 +110,22 @@ def test_decode_host_validation_without_gpu(lib):
     assert lib.flex_linattn_decode(ctypes.byref(one), p, p, p, p, None,
                                    ctypes.c_void_p(4097 + 2), p, p, p, None, p, need,
                                    None) == FLEX_EINVAL
+
+
+def test_awd_host_validation_without_gpu(lib):
+    from paper_2606_27748_gb300.flexattn import (FlexShape, FLEX_EINVAL, FLEX_EUNSUPPORTED,
+                                                 FLEX_EWORKSPACE)
+    p = ctypes.c_void_p(4096)  # never dereferenced: validation fails first
+    ok = FlexShape(2, 3, 300, 64, 64, 1)
+    f32 = FlexShape(2, 3, 300, 64, 64, 0)
+    need = lib.flex_awd_workspace_bytes(ctypes.byref(ok))
+    assert need > 256 and lib.flex_awd_workspace_bytes(ctypes.byref(f32)) == 0
+    # (shape, q, k, W1, W2, tau, causal, loss, ws, ws_bytes, stream)
+    assert lib.flex_awd_loss(ctypes.byref(ok), None, p, p, None, None, 0, p, p, need,
+                             None) == FLEX_EINVAL
+    assert lib.flex_awd_loss(ctypes.byref(f32), p, p, p, None, None, 0, p, p, need,
+                             None) == FLEX_EUNSUPPORTED
+    assert lib.flex_awd_loss(ctypes.byref(ok), p, p, p, None, None, 0, p, p, need - 1,
+                             None) == FLEX_EWORKSPACE
+    assert lib.flex_awd_loss(ctypes.byref(ok), p, p, p, None, ctypes.c_void_p(4098), 0, p, p,
+                             need, None) == FLEX_EINVAL
