@@ -36,6 +36,8 @@ METRIC = "RFF linear-attn fwd tokens/s (N=16K causal) & % of bf16 tensor/HBM roo
 METRIC_TRAIN = "RFF linear-attn fwd+bwd training-step tokens/s & % of roofline"
 METRIC_DECODE = ("RFF linear-attn recurrent decode tokens/s (one new token per sequence, fp32 "
                  "running state) & % of HBM roofline")
+METRIC_AWD = ("RFF attention-weight distillation loss tokens/s (softmax teacher vs kernel "
+              "weights, blockwise N x N) & % of roofline")
 L2_BYTES = 129e6
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
@@ -273,6 +275,25 @@ def run_reference(args, w):
                        "variant": w.variant, "causal": True},
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                              "sample": f"one decode step of all {w.B}x{w.H} sequences per step"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}), flush=True)
+        return
+    if w.awd:
+        nseq = 8
+        for _ in range(args.warmup):
+            oracle_awd_sample(w, nseq, args.prefactor)
+        step = sum(oracle_awd_sample(w, nseq, args.prefactor)
+                   for _ in range(args.steps)) / args.steps
+        value = nseq * w.N / w.H / step
+        print(json.dumps({
+            "metric": METRIC_AWD, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d, "M": w.M,
+                       "variant": w.variant, "causal": w.causal},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                             "sample": f"{nseq} sequences of N={w.N} per step"},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}), flush=True)
         return
@@ -639,6 +660,178 @@ def run_decode(args, w):
         dist.destroy_process_group()
 
 
+# ---------------------------------------------------------------------------------------
+# Attention-weight distillation loss: a step is the loss of every sequence of the batch.
+# ---------------------------------------------------------------------------------------
+def awd_work(w):
+    """(bytes, flops, sin/cos+exp/log) per step: q, k read, the loss written; the score and
+    kernel contractions over the (masked) pairs plus the feature projections; per pair one
+    exp and one log, per token and frequency 2 (s) or 3 (n) sin/cos for q and for k."""
+    bh, N = w.B * w.H, w.N
+    pairs = bh * (N * (N + 1) // 2 if w.causal else N * N)
+    c = 2 if w.variant == "n" else 1
+    nbytes = bh * N * w.d * elem_bytes(w) * 2 + bh * 4
+    flops = 2 * pairs * (w.d + 2 * w.M) + 2 * bh * N * 2 * w.d * w.M * c
+    ops = 2 * pairs + bh * N * 2 * w.M * (3 if w.variant == "n" else 2)
+    return nbytes, flops, ops
+
+
+def oracle_awd_sample(w, nseq, prefactor=False):
+    """Seconds of the oracle loss over the first `nseq` sequences (one thread)."""
+    import oracle
+    nb = -(-nseq // w.H)
+    ins = workloads.make_inputs(w, bs=range(nb))
+    q, k = (ins[n].reshape(nb * w.H, w.N, w.d)[None, :nseq] for n in "qk")
+    heads = [s_ % w.H for s_ in range(nseq)]
+    W1 = ins["W1"][heads]
+    W2 = None if ins["W2"] is None else ins["W2"][heads]
+    tau = workloads.draw_tau(w)[heads] if prefactor else None
+    t0 = time.perf_counter()
+    oracle.awd(q, k, W1, W2, w.causal, tau=tau)
+    return time.perf_counter() - t0
+
+
+def run_awd(args, w):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2606_27748_gb300 import build, flexattn
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if rank == 0 or not os.path.exists(flexattn.LIBRARY):
+        build.build()
+    if world > 1:
+        dist.barrier()
+    flexattn.load()
+    tdt = torch.bfloat16
+    ins = workloads.make_inputs(w)
+    host = {n: torch.from_numpy(ins[n]).to(tdt).pin_memory() for n in "qk"}
+    q, k = host["q"].to(dev), host["k"].to(dev)
+    W1 = torch.from_numpy(ins["W1"]).to(dev)
+    W2 = None if ins["W2"] is None else torch.from_numpy(ins["W2"]).to(dev)
+    del ins
+    tau = torch.from_numpy(workloads.draw_tau(w)).to(dev) if args.prefactor else None
+    shape = flexattn.shape_of(q, W1)
+    ws = flexattn.awd_workspace(shape, dev)
+    loss = torch.empty(w.B, w.H, dtype=torch.float32, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > L2: a cold step
+    stream = torch.cuda.current_stream()
+
+    def step():
+        flexattn.awd_loss(q, k, W1, W2, w.causal, tau=tau, loss=loss, ws=ws)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    flexattn.check_status(ws)
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(K)]
+    clocks = Clocks(torch.cuda.current_device()) if rank == 0 else None
+    if clocks:
+        clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    launches0 = flexattn.kernel_launches()
+    for i in range(K):
+        flush.zero_()  # outside the step's events
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = flexattn.kernel_launches() - launches0
+    clk = clocks.stop() if clocks else None
+    flexattn.check_status(ws)
+    kernel_ms = sum(a.elapsed_time(b) for a, b in ev) / K
+    kernel_ms = max_over_ranks([kernel_ms], world, dev)[0]
+    value = job_value(world, w.tokens, kernel_ms)
+
+    e2e = None
+    if not args.no_e2e:  # q, k from pinned host memory, the losses back
+        host_out = torch.empty(loss.shape, dtype=loss.dtype).pin_memory()
+
+        def e2e_step():
+            q.copy_(host["q"], non_blocking=True)
+            k.copy_(host["k"], non_blocking=True)
+            step()
+            host_out.copy_(loss, non_blocking=True)
+
+        for _ in range(max(3, args.warmup)):
+            e2e_step()
+        barrier()
+        torch.cuda.synchronize()
+        tot = 0.0
+        for _ in range(K):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            e2e_step()
+            b.record(stream)
+            torch.cuda.synchronize()
+            tot += a.elapsed_time(b)
+        barrier()
+        e2e_ms = max_over_ranks([tot / K], world, dev)[0]
+        e2e = {"value": job_value(world, w.tokens, e2e_ms), "unit": "tokens/s",
+               "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in host.values()),
+               "d2h_bytes_per_step": host_out.numel() * host_out.element_size()}
+
+    peaks, peaks_src = load_peaks()
+    nbytes, flops, ops = awd_work(w)
+    sec = kernel_ms * 1e-3
+    sms = 152
+    sfu_peak = SFU_PER_CLK_PER_SM * sms * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e9
+    roofs = {"hbm": (nbytes / sec / 1e9, peaks["hbm_gbs"], "GB/s", nbytes / (peaks["hbm_gbs"] * 1e9)),
+             "tensor": (flops / sec / 1e12, peaks["bf16_tflops"], "TFLOP/s",
+                        flops / (peaks["bf16_tflops"] * 1e12)),
+             "alu": (ops / sec / 1e9, sfu_peak, "Gops/s", ops / (sfu_peak * 1e9))}
+    bound = max(roofs, key=lambda r: roofs[r][3])
+    ach, pk, unit, _ = roofs[bound]
+    roof = {"bound": bound, "achieved": ach, "peak": pk, "unit": unit, "frac": ach / pk,
+            "traffic": None, "peak_source": peaks_src, "algorithmic_bytes_per_launch": nbytes,
+            "algorithmic_flops_per_launch": flops, "sfu_ops_per_launch": ops,
+            "time_at_peak_us": {r: v[3] * 1e6 for r, v in roofs.items()},
+            "fracs": {r: v[0] / v[1] for r, v in roofs.items()},
+            "alu_peak_note": f"{SFU_PER_CLK_PER_SM} MUFU results (ex2, lg2, sin, cos) per clock "
+                             f"per SM x {sms} SMs x {peaks.get('sm_max_mhz', 2070.0):.0f} MHz",
+            "kernel_ms": kernel_ms}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        nseq = w.B * w.H  # the whole batch: ~10 s of one core
+        t = oracle_awd_sample(w, nseq, args.prefactor)
+        cpu = {"value": nseq * w.N / w.H / t, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": f"{nseq} of {w.B * w.H} sequences of N={w.N} (fp64 C oracle, one "
+                         f"thread), {t:.2f} s; tokens = sequences*N/H"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC_AWD, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": K, "warmup": args.warmup, "ms_per_step": kernel_ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": w.dtype, "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "d": w.d, "M": w.M,
+                       "variant": w.variant, "causal": w.causal,
+                       "l2": "flushed (256 MB write) before each timed step",
+                       "parallelism": f"replicas x{world}",
+                       "prefactor": PREFACTOR if args.prefactor else None},
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+            "gpu_launches": launches,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def run_sweep(args, w):
     """Forward time and device memory against N for one workload family (the paper's
     time-and-memory-versus-length comparison, our own curve only).  Per N: inputs from the
@@ -710,6 +903,8 @@ def main():
         run_reference(args, w)
     elif w.decode:
         run_decode(args, w)
+    elif w.awd:
+        run_awd(args, w)
     else:
         run_ours(args, w)
 

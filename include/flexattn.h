@@ -167,7 +167,8 @@ size_t flex_awd_workspace_bytes(const flex_shape* shape);
  * Fourier estimates and row sums can be negative) counts log(1e-6).  Computed blockwise
  * (128 x 128 tiles of scores and kernel values on the tensor cores, online softmax), never
  * materialising the N x N matrices.  q, k: [B][H][N][d] bf16 (d = 64, M in {64, 128});
- * loss: [B][H] fp32, overwritten.  ws: workspace of flex_awd_workspace_bytes() bytes.
+ * loss: [B][H] fp32, overwritten.  ws: workspace of flex_awd_workspace_bytes() bytes
+ * (it holds phi(q) and the key-weighted phi(k), written by a tensor-core feature pass).
  * Launches 4 kernels (5 with tau).  Errors: FLEX_EINVAL for NULL or misaligned pointers,
  * FLEX_EUNSUPPORTED for other shapes or fp32 storage, FLEX_EWORKSPACE. */
 int flex_awd_loss(const flex_shape* shape, const void* q, const void* k, const float* W1,

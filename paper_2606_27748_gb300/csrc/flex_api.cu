@@ -236,11 +236,13 @@ int flex_awd_loss(const flex_shape* shape, const void* q, const void* k, const f
     char* base = (char*)ws;
     float* kw = tau ? (float*)(base + w.kw) : nullptr;
     if (tau && (rc = count(1, flex::launch_key_weights(p, k, tau, kw, s)))) return rc;
-    if ((rc = count(1, flex::launch_featmap_scaled(p, q, W1, W2, nullptr, base + w.pq, s))))
+    int* status = &((flex::WsHeader*)ws)->status;
+    if ((rc = count(1, flex::launch_tc_featmap(p, q, W1, W2, nullptr, base + w.pq, status, s))))
         return rc;
-    if ((rc = count(1, flex::launch_featmap_scaled(p, k, W1, W2, kw, base + w.pk, s)))) return rc;
+    if ((rc = count(1, flex::launch_tc_featmap(p, k, W1, W2, kw, base + w.pk, status, s))))
+        return rc;
     return count(2, flex::launch_tc_awd(p, q, k, base + w.pq, base + w.pk, (float*)(base + w.part),
-                                        loss, &((flex::WsHeader*)ws)->status, s));
+                                        loss, status, s));
 }
 
 unsigned long long flex_kernel_launches(void) { return g_launches.load(); }

@@ -86,6 +86,11 @@ cudaError_t launch_tc_bwd(const Problem& p, const void* q, const void* k, const 
                           float* dW1, float* dW2, float* dtau, void* scratch, int* status,
                           cudaStream_t s);
 
+// ---- feature map on the tensor cores (bf16, d = 64, M in {64, 128}) ------------------
+bool tc_featmap_supported(const Problem& p);
+cudaError_t launch_tc_featmap(const Problem& p, const void* x, const float* W1, const float* W2,
+                              const float* rowscale, void* phi, int* status, cudaStream_t s);
+
 // ---- attention-weight distillation loss (tensor cores: bf16, d = 64, M in {64, 128}) ---
 bool tc_awd_supported(const Problem& p);
 size_t tc_awd_part_floats(const Problem& p);  // partial slots [B*H][query blocks]

@@ -39,6 +39,7 @@ class Workload:
     seed: int
     backward: bool = False
     decode: bool = False  # recurrent decode steps: one new token per sequence per step
+    awd: bool = False     # attention-weight distillation loss (q, k only)
 
     @property
     def tokens(self) -> int:
@@ -74,6 +75,11 @@ HEADLINE = ORDERED[2]
 DECODE = Workload("n_decode_bf16_B256H16_d64M128", "n", True, "bf16", 256, 16, 64, 64, 128,
                   64 ** -0.25, "normal", 6, decode=True)
 WORKLOADS[DECODE.name] = DECODE
+# The distillation setting: a 125M RoBERTa encoder (8 heads, head size 64) converted with
+# n = d = 64 frequencies, batch 32, sequences of 512 tokens (non-causal).
+AWD = Workload("n_awd_bf16_B32H8N512_d64M64", "n", False, "bf16", 32, 8, 512, 64, 64,
+               64 ** -0.25, "normal", 7, awd=True)
+WORKLOADS[AWD.name] = AWD
 
 
 def bf16_bits(x: np.ndarray) -> np.ndarray:
