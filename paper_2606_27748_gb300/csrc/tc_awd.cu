@@ -9,9 +9,10 @@
 // Entries with a non-positive R_ij count log(1e-6) (RFF estimates and row sums can be
 // negative; the logarithm is undefined there).
 //
-// One CTA per (sequence, block of 128 queries), 256 threads, phases serialised: TMA loads
-// the query tile and its features once, then per block of 128 keys the key tile and its
-// features; thread 0 issues S = Q K^T (K = d = 64) into T_S and A = phi(Q) phi~(K)^T
+// One CTA per (sequence, block of 128 queries), 256 threads: TMA loads the query tile and
+// its features once, then per block of 128 keys the key tile and its features (the next
+// block's load is issued once the MMAs have read the current one, so it overlaps the
+// epilogue); thread 0 issues S = Q K^T (K = d = 64) into T_S and A = phi(Q) phi~(K)^T
 // (K = 2M) into T_A; every thread then takes half of one query row's 128 columns and keeps
 // online statistics in base 2: the running maximum m of the scores, Z = sum 2^(s-m), and
 // for positive and negative A separately Z+- = sum 2^(s-m) and T+- = sum 2^(s-m) log2|A|,
@@ -105,18 +106,20 @@ __global__ void __launch_bounds__(kThreadsA, 1)
     const int nkb = causal ? qb + 1 : (N + kC - 1) / kC;
     bool ok = true;
 
-    for (int kb = 0; kb < nkb && ok; ++kb) {
-        if (tid == 0) {  // one arrival per phase; the first also brings the query side
-            mbar_arrive_expect_tx(&tma_bar, (1 + G2) * kTileBytes * (kb == 0 ? 2 : 1));
-            if (kb == 0) {
-                tma_load_3d(sb + L::Q, &tmap_q, 0, qb * kC, bh, &tma_bar);
-                for (int g = 0; g < G2; ++g)
-                    tma_load_3d(sb + L::PQ + g * 16384, &tmap_pq, 64 * g, qb * kC, bh, &tma_bar);
-            }
-            tma_load_3d(sb + L::K, &tmap_k, 0, kb * kC, bh, &tma_bar);
+    // key tiles of block kb (one arrival per phase; the first also brings the query side)
+    auto load_keys = [&](int kb) {
+        mbar_arrive_expect_tx(&tma_bar, (1 + G2) * kTileBytes * (kb == 0 ? 2 : 1));
+        if (kb == 0) {
+            tma_load_3d(sb + L::Q, &tmap_q, 0, qb * kC, bh, &tma_bar);
             for (int g = 0; g < G2; ++g)
-                tma_load_3d(sb + L::PK + g * 16384, &tmap_pk, 64 * g, kb * kC, bh, &tma_bar);
+                tma_load_3d(sb + L::PQ + g * 16384, &tmap_pq, 64 * g, qb * kC, bh, &tma_bar);
         }
+        tma_load_3d(sb + L::K, &tmap_k, 0, kb * kC, bh, &tma_bar);
+        for (int g = 0; g < G2; ++g)
+            tma_load_3d(sb + L::PK + g * 16384, &tmap_pk, 64 * g, kb * kC, bh, &tma_bar);
+    };
+    if (tid == 0) load_keys(0);
+    for (int kb = 0; kb < nkb && ok; ++kb) {
         ok = bar_wait(&tma_bar, tma_phase, &abort_flag, status);
         tma_phase ^= 1;
         ok = !__syncthreads_or(!ok);
@@ -138,10 +141,8 @@ __global__ void __launch_bounds__(kThreadsA, 1)
         ok = !__syncthreads_or(!ok);
         if (!ok) break;
         fence_after_sync();
-        if (tid == 0 && kb + 1 < nkb) {  // the next key block's tiles into L2
-            tma_prefetch_3d(&tmap_k, 0, (kb + 1) * kC, bh);
-            for (int g = 0; g < G2; ++g) tma_prefetch_3d(&tmap_pk, 64 * g, (kb + 1) * kC, bh);
-        }
+        // the MMAs have read the key tiles: the next block's load overlaps this epilogue
+        if (tid == 0 && kb + 1 < nkb) load_keys(kb + 1);
         // statistics over this thread's 64 columns, two rounds of 32
 #pragma unroll
         for (int b = 0; b < 2; ++b) {

@@ -3,8 +3,9 @@
 // an optional per-row factor (the key weight of the norm prefactor), into
 // phi [B*H*N][2M] bf16 (cos block, then sin block).
 //
-// One CTA per 128 rows of one sequence (one head's frequencies), 256 threads: TMA loads
-// the rows, thread 0 issues the projections x W^T (s: W1; n: U = (W1+W2)/2 and
+// One CTA per 4 blocks of 128 rows of one sequence (one head's frequencies, staged once),
+// 256 threads: TMA loads the rows (the next block while the current one is worked on),
+// thread 0 issues the projections x W^T (s: W1; n: U = (W1+W2)/2 and
 // V = (W1-W2)/2; bf16 operands, fp32 in tensor memory), one group of 64 frequencies per
 // 64 (s) or 128 (n) columns; every thread takes one row and 32 frequencies of each group:
 // hardware sin/cos, products, bf16 pack, 64-byte stores of its cos and sin runs.
@@ -18,6 +19,7 @@ using namespace tc;
 
 constexpr int kC = 128;
 constexpr int kThreadsF = 256;
+constexpr int kBlocksPerCta = 4;  // row blocks of one sequence per CTA (W staged once)
 
 template <bool NS, int G>  // G = M / 64 frequency groups
 __global__ void __launch_bounds__(kThreadsF)
@@ -26,22 +28,23 @@ __global__ void __launch_bounds__(kThreadsF)
                       const float* __restrict__ rowscale, float scale,
                       __nv_bfloat16* __restrict__ phi, int* status)
 {
-    constexpr int P = NS ? 128 : 64;  // projection rows (= tensor memory columns) per group
-    constexpr uint32_t X = 0, W = 16384;  // x tile, then G x P frequency rows
+    constexpr int P = NS ? 128 : 64;        // projection rows (= tensor memory columns) per group
+    constexpr uint32_t NCOLS = G * P;        // 64, 128 or 256: a power of two
+    constexpr uint32_t X0 = 0, W = 32768;    // two x tiles, then G x P frequency rows
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const uint32_t sb = smem_u32(sm);
     __shared__ uint32_t tmem_base_sh;
-    __shared__ __align__(8) uint64_t mbar, tma_bar;
+    __shared__ __align__(8) uint64_t mbar, tma_bar[2];
     __shared__ volatile int abort_flag;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int wg = warp >> 2, quad = warp & 3, t = 32 * quad + lane;
-    const int nblk = (N + kC - 1) / kC;
-    const int bh = blockIdx.x / nblk, blk = blockIdx.x % nblk, h = bh % H;
-    const int row = blk * kC + t;
+    const int nblk = (N + kC - 1) / kC, nchunk = (nblk + kBlocksPerCta - 1) / kBlocksPerCta;
+    const int bh = blockIdx.x / nchunk, b0 = (blockIdx.x % nchunk) * kBlocksPerCta, h = bh % H;
+    const int nb = min(kBlocksPerCta, nblk - b0);
 
-    // this head's frequency rows, bf16 K-major (n: U rows then V rows per group)
+    // this head's frequency rows, bf16 K-major (n: U rows then V rows per group), once
     for (int idx = tid; idx < G * P * 8; idx += kThreadsF) {
         const int r = idx >> 3, c = idx & 7, g = r / P, rr = r % P;
         const int f = 64 * g + (rr & 63);
@@ -61,12 +64,15 @@ __global__ void __launch_bounds__(kThreadsF)
     }
     if (tid == 0) {
         mbar_init(&mbar, 1);
-        mbar_init(&tma_bar, 1);
+        mbar_init(&tma_bar[0], 1);
+        mbar_init(&tma_bar[1], 1);
         abort_flag = 0;
         fence_mbar_init();
+        mbar_arrive_expect_tx(&tma_bar[0], kTileBytes);
+        tma_load_3d(sb + X0, &tmap_x, 0, b0 * kC, bh, &tma_bar[0]);
     }
     if (warp == 0) {
-        tmem_alloc(&tmem_base_sh, 256);
+        tmem_alloc(&tmem_base_sh, NCOLS);
         tmem_relinquish();
     }
     fence_proxy_async();
@@ -75,18 +81,23 @@ __global__ void __launch_bounds__(kThreadsF)
     fence_after_sync();
     const uint32_t tm = tmem_base_sh;
     const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
+    constexpr uint32_t I_PROJ = idesc_bf16(128, P, 0, 0);
 
-    if (tid == 0) {
-        mbar_arrive_expect_tx(&tma_bar, kTileBytes);
-        tma_load_3d(sb + X, &tmap_x, 0, blk * kC, bh, &tma_bar);
-    }
-    bool ok = bar_wait(&tma_bar, 0, &abort_flag, status);
-    ok = !__syncthreads_or(!ok);
-    if (ok) {
+    bool ok = true;
+    for (int r = 0; r < nb && ok; ++r) {
+        const int blk = b0 + r, xb = r & 1;
+        // the next tile into the other buffer (its projection finished last iteration)
+        if (tid == 0 && r + 1 < nb) {
+            mbar_arrive_expect_tx(&tma_bar[xb ^ 1], kTileBytes);
+            tma_load_3d(sb + X0 + (xb ^ 1) * 16384, &tmap_x, 0, (blk + 1) * kC, bh,
+                        &tma_bar[xb ^ 1]);
+        }
+        ok = bar_wait(&tma_bar[xb], (r >> 1) & 1, &abort_flag, status);
+        ok = !__syncthreads_or(!ok);
+        if (!ok) break;
         fence_after_sync();
         if (tid == 0) {
-            const uint64_t dX = sdesc(sb + X, 16, 1024);
-            constexpr uint32_t I_PROJ = idesc_bf16(128, P, 0, 0);
+            const uint64_t dX = sdesc(sb + X0 + xb * 16384, 16, 1024);
             for (int g = 0; g < G; ++g) {
                 const uint64_t dW = sdesc(sb + W + g * P * 128, 16, 1024);
 #pragma unroll
@@ -96,11 +107,11 @@ __global__ void __launch_bounds__(kThreadsF)
             }
             mma_commit(&mbar);
         }
-        ok = bar_wait(&mbar, 0, &abort_flag, status);
+        ok = bar_wait(&mbar, r & 1, &abort_flag, status);
         ok = !__syncthreads_or(!ok);
-    }
-    if (ok) {
+        if (!ok) break;
         fence_after_sync();
+        const int row = blk * kC + t;
         const bool valid = row < N;
         const float sc = scale * ((rowscale && valid) ? rowscale[(size_t)bh * N + row] : 1.f);
         __nv_bfloat16* out = phi + ((size_t)bh * N + (valid ? row : 0)) * 2 * M;
@@ -138,11 +149,13 @@ __global__ void __launch_bounds__(kThreadsF)
                 }
             }
         }
+        fence_before_sync();
+        __syncthreads();  // tensor memory free for the next projection
     }
     fence_before_sync();
     __syncthreads();
     fence_after_sync();
-    if (warp == 0) tmem_dealloc(tm, 256);
+    if (warp == 0) tmem_dealloc(tm, NCOLS);
 }
 
 template <bool NS, int G>
@@ -153,11 +166,12 @@ cudaError_t launch_typed(const Problem& p, const void* x, const float* W1, const
     const int BH = p.B * p.H;
     if (!make_act_map(&mx, x, BH, p.N)) return cudaErrorInvalidValue;
     constexpr int P = NS ? 128 : 64;
-    const int smem = 16384 + G * P * 128 + 1024;
+    const int smem = 32768 + G * P * 128 + 1024;
     auto kern = tc_featmap_kernel<NS, G>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    const long long blocks = (long long)BH * ((p.N + kC - 1) / kC);
+    const int nblk = (p.N + kC - 1) / kC;
+    const long long blocks = (long long)BH * ((nblk + kBlocksPerCta - 1) / kBlocksPerCta);
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
     kern<<<(unsigned)blocks, kThreadsF, smem, s>>>(mx, p.H, p.N, p.M, W1, W2, rowscale,
                                                    1.0f / sqrtf((float)p.M),
