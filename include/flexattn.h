@@ -74,8 +74,10 @@ const char* flex_strerror(int status);
 size_t flex_workspace_bytes(const flex_shape* shape, int causal, int backward);
 
 /* Feature map phi of Eq. phi_n (W2 == NULL) or Eq. phi_non (W2 != NULL), written out.
- * x: [B][H][N][d], phi: [B][H][N][2M], both in shape->dtype.  This is the only entry
- * point that writes phi to memory; the attention entry points keep it on chip. */
+ * x: [B][H][N][d], phi: [B][H][N][2M], both in shape->dtype, scaled by M^{-1/2}.  bf16
+ * with d = 64 and M in {64, 128} projects on the tensor cores (frequencies rounded to
+ * bf16); other shapes use fp32 CUDA-core arithmetic.  This and flex_awd_loss are the only
+ * entry points that write phi to memory; the attention entry points keep it on chip. */
 int flex_featmap(const flex_shape* shape, const void* x, const float* W1, const float* W2,
                  void* phi, void* stream);
 

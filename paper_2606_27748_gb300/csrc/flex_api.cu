@@ -105,6 +105,9 @@ int flex_featmap(const flex_shape* shape, const void* x, const float* W1, const 
     if (!x || !W1 || !phi) return FLEX_EINVAL;
     if (!aligned(x, 16) || !aligned(W1, 16) || !aligned(phi, 16) || (W2 && !aligned(W2, 16)))
         return FLEX_EINVAL;
+    if (flex::tc_featmap_supported(p))  // tensor-core projection (no workspace: no status)
+        return count(1, flex::launch_tc_featmap(p, x, W1, W2, nullptr, phi, nullptr,
+                                                (cudaStream_t)stream));
     return count(1, flex::launch_featmap(p, x, W1, W2, phi, (cudaStream_t)stream));
 }
 

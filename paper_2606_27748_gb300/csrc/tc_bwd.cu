@@ -76,7 +76,8 @@ __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes)
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
-template <bool NS>
+// KW: key weights of the norm prefactor given (compile-time; the plain kernel is unchanged)
+template <bool NS, bool KW>
 __global__ void __launch_bounds__(kThreadsB, 1)
     tc_bwd_kernel(const __grid_constant__ CUtensorMap tmap_q,
                   const __grid_constant__ CUtensorMap tmap_k,
@@ -109,7 +110,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     float* zr = reinterpret_cast<float*>(sm + L::ZR);
     float* crow = reinterpret_cast<float*>(sm + L::CROW);
     float* spart = reinterpret_cast<float*>(sm + L::SPART);
-    const float itau = kw ? expf(-tau[h]) : 0.f;
+    const float itau = KW ? expf(-tau[h]) : 0.f;
     float dtau_acc = 0.f;
 
     // ---- set-up: this group's projection rows, zero state, C16 ----
@@ -227,7 +228,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 const float cw0 = __cosf(w[2 * i]), cw1 = __cosf(w[2 * i + 1]);
                 c0 *= cw0; s0 *= cw0; c1 *= cw1; s1 *= cw1;
             }
-            if (kw) { c0 *= wsc; s0 *= wsc; c1 *= wsc; s1 *= wsc; }
+            if (KW) { c0 *= wsc; s0 *= wsc; c1 *= wsc; s1 *= wsc; }
             if (!valid) { c0 = s0 = c1 = s1 = 0.f; }
             pc[i] = pack_bf16(c0, c1);
             ps[i] = pack_bf16(s0, s1);
@@ -277,7 +278,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             zc[4 * j] = a4.x; zc[4 * j + 1] = a4.y; zc[4 * j + 2] = a4.z; zc[4 * j + 3] = a4.w;
             zs[4 * j] = b4.x; zs[4 * j + 1] = b4.y; zs[4 * j + 2] = b4.z; zs[4 * j + 3] = b4.w;
         }
-        const bool wt = kw && PASS == kPassR;
+        const bool wt = KW && PASS == kPassR;
         float sdot = 0.f;
         uint32_t o1[16], o2[16];
 #pragma unroll
@@ -375,7 +376,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         tmem_ld16(tm_row + L::T_A + 32 * wg, *reinterpret_cast<float(*)[16]>(&v_[0]));
         tmem_ld16(tm_row + L::T_A + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&v_[16]));
         tmem_wait_ld();
-        if (kcoef != 0.f) {
+        if (KW && kcoef != 0.f) {
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const uint4 k4 = *reinterpret_cast<const uint4*>(sm + L::K + swz128(t, 32 * wg + 8 * j));
@@ -402,7 +403,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         const int c = PASS == kPassF ? it : nch - 1 - it;
         const int t0 = c * kC, CL = min(kC, N - t0);
         const bool valid = t < CL;
-        const float wk = (kw && valid) ? kw[(size_t)bh * N + t0 + t] : 1.f;
+        const float wk = (KW && valid) ? kw[(size_t)bh * N + t0 + t] : 1.f;
         if (tid == 0) {  // the next chunk's tiles into L2 while this one is worked on
             const int cn = PASS == kPassF ? c + 1 : c - 1;
             if (cn >= 0 && cn < nch) {
@@ -607,21 +608,21 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             if (NS && !project(dK)) goto done;  // u, w of k for the chain rule
             {
                 const float sp = feature_backward(sb + L::PK, 1.0f, valid, wk);
-                if (kw) {
+                if (KW) {
                     spart[128 * wg + t] = sp;
                     dtau_acc = fmaf(-logf(wk), sp, dtau_acc);  // ln w = |k|^2 exp(-tau)
                 }
             }
             handoff();
             if (!project_back(dPK, dPKmn, dKmn, it == 0)) goto done;
-            add_rows(acc_x, t0, valid, kw ? 2.f * itau * (spart[t] + spart[128 + t]) : 0.f);
+            add_rows(acc_x, t0, valid, KW ? 2.f * itau * (spart[t] + spart[128 + t]) : 0.f);
             if (NS) dw_accumulate(it == 0);
             snapshot();
             handoff();
         }
     }
     if (!NS) dw_accumulate(true);  // s: the sum over all chunks, from T_P[64,128)
-    if (kw) {  // this CTA's dtau (pass R; 0 in pass F): warps, then in order
+    if (KW) {  // this CTA's dtau (pass R; 0 in pass F): warps, then in order
         for (int o = 16; o > 0; o >>= 1) dtau_acc += __shfl_xor_sync(0xffffffffu, dtau_acc, o);
         __syncthreads();
         if (lane == 0) spart[warp] = dtau_acc;
@@ -711,7 +712,7 @@ cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const voi
     if (!make_act_map(&mq, q, BH, p.N) || !make_act_map(&mk, k, BH, p.N) ||
         !make_act_map(&mv, v, BH, p.N))
         return cudaErrorInvalidValue;
-    auto kb = tc_bwd_kernel<NS>;
+    auto kb = tau ? tc_bwd_kernel<NS, true> : tc_bwd_kernel<NS, false>;
     if ((e = cudaFuncSetAttribute(kb, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return e;
     typedef const __nv_bfloat16* CB;
     const int units = BH * G;

@@ -117,8 +117,9 @@ __device__ __forceinline__ int segment_bound(int nch, int splits, int j)
     return (int)((2 * num + den) / (2 * den));
 }
 
-// NS: nonstationary features; CS: CTAs per cluster = frequency groups (M / 64).
-template <bool NS, int CS>
+// NS: nonstationary features; CS: CTAs per cluster = frequency groups (M / 64); KW: key
+// weights of the norm prefactor given (a compile-time switch: the plain kernel is unchanged).
+template <bool NS, int CS, bool KW>
 __global__ void __maxnreg__(96)
     tc_fwd_causal_kernel(const __grid_constant__ CUtensorMap tmap_q,
                          const __grid_constant__ CUtensorMap tmap_k,
@@ -377,7 +378,7 @@ __global__ void __maxnreg__(96)
             const bool main = c >= cb;
             const bool valid = t < min(kC, N - c * kC);
             // key weight of the norm prefactor (phi(k) scaled by it), loaded early
-            const float wk = (kw && valid) ? kw[(size_t)bh * N + (size_t)c * kC + t] : 1.f;
+            const float wk = (KW && valid) ? kw[(size_t)bh * N + (size_t)c * kC + t] : 1.f;
             for (int which = main ? 0 : 1; which < 2; ++which) {  // 0: q, 1: k
                 uint32_t pc[16], ps[16];  // [8 r + i]: frequencies 32r + 16 half + 2i, +1
 #pragma unroll
@@ -405,7 +406,7 @@ __global__ void __maxnreg__(96)
                             const float cw0 = __cosf(w[2 * i]), cw1 = __cosf(w[2 * i + 1]);
                             c0 *= cw0; s0 *= cw0; c1 *= cw1; s1 *= cw1;
                         }
-                        if (kw && which == 1) { c0 *= wk; s0 *= wk; c1 *= wk; s1 *= wk; }
+                        if (KW && which == 1) { c0 *= wk; s0 *= wk; c1 *= wk; s1 *= wk; }
                         if (!valid) { c0 = s0 = c1 = s1 = 0.f; }
                         pc[8 * r + i] = pack_bf16(c0, c1);
                         ps[8 * r + i] = pack_bf16(s0, s1);
@@ -627,7 +628,7 @@ __global__ void __maxnreg__(96)
     if (CS > 1) cluster_sync();  // no CTA leaves while its partner may still write to it
 }
 
-template <bool NS, int CS>
+template <bool NS, int CS, bool KW>
 cudaError_t launch_one(const Problem& p, const void* q, const void* k, const void* v,
                        const float* W1, const float* W2, const float* kw, void* out,
                        float* den, int* status, cudaStream_t s)
@@ -638,7 +639,7 @@ cudaError_t launch_one(const Problem& p, const void* q, const void* k, const voi
         !make_act_map(&mv, v, BH, p.N))
         return cudaErrorInvalidValue;
     const int splits = tc_fwd_splits(p, sm_count());
-    auto kern = tc_fwd_causal_kernel<NS, CS>;
+    auto kern = tc_fwd_causal_kernel<NS, CS, KW>;
     const int smem = (int)Cfg<NS>::BYTES + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
@@ -679,11 +680,18 @@ cudaError_t launch_tc_fwd(const Problem& p, const void* q, const void* k, const 
                           float* den, int* status, cudaStream_t s)
 {
     const bool pair = p.M == 128;
+    if (kw) {
+        if (p.nonstat)
+            return pair ? launch_one<true, 2, true>(p, q, k, v, W1, W2, kw, out, den, status, s)
+                        : launch_one<true, 1, true>(p, q, k, v, W1, W2, kw, out, den, status, s);
+        return pair ? launch_one<false, 2, true>(p, q, k, v, W1, W2, kw, out, den, status, s)
+                    : launch_one<false, 1, true>(p, q, k, v, W1, W2, kw, out, den, status, s);
+    }
     if (p.nonstat)
-        return pair ? launch_one<true, 2>(p, q, k, v, W1, W2, kw, out, den, status, s)
-                    : launch_one<true, 1>(p, q, k, v, W1, W2, kw, out, den, status, s);
-    return pair ? launch_one<false, 2>(p, q, k, v, W1, W2, kw, out, den, status, s)
-                : launch_one<false, 1>(p, q, k, v, W1, W2, kw, out, den, status, s);
+        return pair ? launch_one<true, 2, false>(p, q, k, v, W1, W2, kw, out, den, status, s)
+                    : launch_one<true, 1, false>(p, q, k, v, W1, W2, kw, out, den, status, s);
+    return pair ? launch_one<false, 2, false>(p, q, k, v, W1, W2, kw, out, den, status, s)
+                : launch_one<false, 1, false>(p, q, k, v, W1, W2, kw, out, den, status, s);
 }
 
 }  // namespace flex

@@ -64,7 +64,8 @@ struct NcBars {
 // partial / total [S | z] rows: [unit][group][feature 128][80 floats]
 constexpr int kRow = 80;
 
-template <int MODE, bool NS, int G>
+// KW: key weights of the norm prefactor given (compile-time; the plain kernel is unchanged)
+template <int MODE, bool NS, int G, bool KW>
 __global__ void __launch_bounds__(kThreadsNC, 1)
     tc_nc_kernel(const __grid_constant__ CUtensorMap tmap_x,
                  const __grid_constant__ CUtensorMap tmap_v, int H, int N, int M, int splits,
@@ -251,7 +252,7 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
             const int i = j / G, pb = j & 1;
             const bool valid = t < min(kC, N - (c0 + i) * kC);
             // state mode: key weight of the norm prefactor (phi(k) scaled by it)
-            const float wk = (MODE == kState && kw && valid)
+            const float wk = (MODE == kState && KW && valid)
                                  ? kw[(size_t)bh * N + (size_t)(c0 + i) * kC + t] : 1.f;
             if (!bar_wait(&bars.p_full[pb], (j >> 1) & 1, &abort_flag, status)) break;
             fence_after_sync();
@@ -277,7 +278,7 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
                     const float cw0 = __cosf(w[2 * e]), cw1 = __cosf(w[2 * e + 1]);
                     cc0 *= cw0; s0 *= cw0; cc1 *= cw1; s1 *= cw1;
                 }
-                if (MODE == kState && kw) { cc0 *= wk; s0 *= wk; cc1 *= wk; s1 *= wk; }
+                if (MODE == kState && KW) { cc0 *= wk; s0 *= wk; cc1 *= wk; s1 *= wk; }
                 if (!valid) { cc0 = s0 = cc1 = s1 = 0.f; }
                 pc[e] = pack_bf16(cc0, cc1);
                 ps[e] = pack_bf16(s0, s1);
@@ -382,8 +383,8 @@ cudaError_t launch_nc(const Problem& p, const void* q, const void* k, const void
     float* part = static_cast<float*>(scratch);
     float* total = part + (size_t)BH * splits * G * 128 * kRow;
     const int smem = (int)NcCfg<NS, G>::BYTES + 1024;
-    auto k_state = tc_nc_kernel<kState, NS, G>;
-    auto k_out = tc_nc_kernel<kOut, NS, G>;
+    auto k_state = kw ? tc_nc_kernel<kState, NS, G, true> : tc_nc_kernel<kState, NS, G, false>;
+    auto k_out = tc_nc_kernel<kOut, NS, G, false>;
     cudaError_t e = cudaFuncSetAttribute(k_state, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(k_out, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);

@@ -29,7 +29,7 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
 }
 
 // Bounded wait on one mbarrier phase.  On a time-out the CTA is told to stop (abort flag)
-// and the status word records FLEX_ETIMEOUT; every other wait then returns at once.
+// and the status word (if any) records FLEX_ETIMEOUT; every other wait then returns at once.
 __device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
                                          int* status)
 {
@@ -40,7 +40,7 @@ __device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity, volatil
         if (*abort_flag) return false;
         if (clock64() - t0 > kWaitCycles) {
             *abort_flag = 1;
-            atomicExch(status, (int)FLEX_ETIMEOUT);
+            if (status) atomicExch(status, (int)FLEX_ETIMEOUT);
             return false;
         }
     }
@@ -56,7 +56,7 @@ __device__ __forceinline__ bool bar_wait_cluster(uint64_t* bar, uint32_t parity,
         if (*abort_flag) return false;
         if (clock64() - t0 > kWaitCycles) {
             *abort_flag = 1;
-            atomicExch(status, (int)FLEX_ETIMEOUT);
+            if (status) atomicExch(status, (int)FLEX_ETIMEOUT);
             return false;
         }
     }
