@@ -143,7 +143,10 @@ __global__ void __launch_bounds__(kThreadsA, 1)
         fence_after_sync();
         // the MMAs have read the key tiles: the next block's load overlaps this epilogue
         if (tid == 0 && kb + 1 < nkb) load_keys(kb + 1);
-        // statistics over this thread's 64 columns, two rounds of 32
+        // statistics over this thread's 64 columns, two rounds of 32; a block with no
+        // masked key (not the ragged last one, not on the causal diagonal) takes the
+        // unmasked path (rows past N are computed and discarded at the end)
+        const bool full = (kb + 1) * kC <= N && (!causal || kb < qb);
 #pragma unroll
         for (int b = 0; b < 2; ++b) {
             const uint32_t col = 64 * wg + 32 * b;
@@ -153,6 +156,28 @@ __global__ void __launch_bounds__(kThreadsA, 1)
             tmem_ld16(tm_row + L::T_A + col, *reinterpret_cast<float(*)[16]>(&a[0]));
             tmem_ld16(tm_row + L::T_A + col + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
             tmem_wait_ld();
+            if (full) {  // no mask: every key of the block is valid for every row
+                float bmax = s[0];
+#pragma unroll
+                for (int e = 1; e < 32; ++e) bmax = fmaxf(bmax, s[e]);
+                bmax *= score_scale;  // > 0, so the maximum commutes with the scale
+                if (bmax > st.m) {
+                    const float f = ex2f(st.m - bmax);
+                    st.z *= f; st.zp *= f; st.zn *= f; st.tp *= f; st.tn *= f;
+                    st.m = bmax;
+                }
+                const float nm = -st.m;
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    const float p = ex2f(fmaf(s[e], score_scale, nm));
+                    const float pl = p * lg2f(fabsf(a[e]));
+                    st.z += p;
+                    st.den += a[e];
+                    if (a[e] > 0.f) { st.zp += p; st.tp += pl; }
+                    if (a[e] < 0.f) { st.zn += p; st.tn += pl; }
+                }
+                continue;
+            }
             const int j0 = kb * kC + (int)col;
             float bmax = -INFINITY;
 #pragma unroll
