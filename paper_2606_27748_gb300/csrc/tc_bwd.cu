@@ -81,7 +81,9 @@ template <bool NS, bool KW>
 __global__ void __launch_bounds__(kThreadsB, 1)
     tc_bwd_kernel(const __grid_constant__ CUtensorMap tmap_q,
                   const __grid_constant__ CUtensorMap tmap_k,
-                  const __grid_constant__ CUtensorMap tmap_v, int H, int N, int M, int G, int causal,
+                  const __grid_constant__ CUtensorMap tmap_v,
+                  const __grid_constant__ CUtensorMap tmap_do,
+                  const __grid_constant__ CUtensorMap tmap_o, int H, int N, int M, int G, int causal,
                   const __nv_bfloat16* __restrict__ q,
                   const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __restrict__ v,
                   const float* __restrict__ W1, const float* __restrict__ W2,
@@ -416,25 +418,30 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 prefetch_l2(outp + off, bytes);
             }
         }
-        // ---- loads: q, k, v tiles (TMA; rows past N read as zero); g tile and c_t from
-        // dout, out, den ----
+        // ---- loads: q, k, v, dout, out tiles (TMA; rows past N read as zero; dout and out
+        // go to [DO | O], free until pass R stores bf16(A) there later in the chunk); then
+        // the g tile and c_t from dout, out (shared memory) and den ----
         if (tid == 0) {
-            mbar_arrive_expect_tx(&tma_bar, 3 * kTileBytes);
+            mbar_arrive_expect_tx(&tma_bar, 5 * kTileBytes);
             tma_load_3d(sb + L::Q, &tmap_q, 0, t0, bh, &tma_bar);
             tma_load_3d(sb + L::K, &tmap_k, 0, t0, bh, &tma_bar);
             tma_load_3d(sb + L::V, &tmap_v, 0, t0, bh, &tma_bar);
+            tma_load_3d(sb + L::DO, &tmap_do, 0, t0, bh, &tma_bar);
+            tma_load_3d(sb + L::O, &tmap_o, 0, t0, bh, &tma_bar);
         }
+        const float den_t = (wg == 0 && valid) ? den[(size_t)bh * N + t0 + t] : 1.f;
+        if (!bar_wait(&tma_bar, tma_phase, &abort_flag, status)) goto done;
+        tma_phase ^= 1;
         if (wg == 0) {
             float gsc = 0.f, cval = 0.f;
             uint32_t gp[32];
             if (valid) {
-                const size_t row = base + (size_t)(t0 + t) * 64;
-                gsc = dscale / den[(size_t)bh * N + t0 + t];
+                gsc = dscale / den_t;
                 float dot = 0.f;
 #pragma unroll
                 for (int cc = 0; cc < 8; ++cc) {
-                    const uint4 a4 = __ldg(reinterpret_cast<const uint4*>(dout + row + cc * 8));
-                    const uint4 o4 = __ldg(reinterpret_cast<const uint4*>(outp + row + cc * 8));
+                    const uint4 a4 = *reinterpret_cast<const uint4*>(sm + L::DO + swz128(t, cc * 8));
+                    const uint4 o4 = *reinterpret_cast<const uint4*>(sm + L::O + swz128(t, cc * 8));
                     const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w}, ow[4] = {o4.x, o4.y, o4.z, o4.w};
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
@@ -462,8 +469,6 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 *reinterpret_cast<__nv_bfloat16*>(sm + L::C16 + (t >> 6) * 2048 + swz128(0, t & 63)) =
                     __float2bfloat16_rn(cval);
         }
-        if (!bar_wait(&tma_bar, tma_phase, &abort_flag, status)) goto done;
-        tma_phase ^= 1;
         handoff();
         // ---- features of q and k for this group ----
         if (!project_qk()) goto done;
@@ -708,15 +713,16 @@ cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const voi
     if (e != cudaSuccess) return e;
     if (tau && (e = launch_key_weights(p, k, tau, kw, s)) != cudaSuccess) return e;
     const int smem = (int)BwCfg<NS>::BYTES + 1024;
-    CUtensorMap mq, mk, mv;
+    CUtensorMap mq, mk, mv, mdo, mo;
     if (!make_act_map(&mq, q, BH, p.N) || !make_act_map(&mk, k, BH, p.N) ||
-        !make_act_map(&mv, v, BH, p.N))
+        !make_act_map(&mv, v, BH, p.N) || !make_act_map(&mdo, dout, BH, p.N) ||
+        !make_act_map(&mo, out, BH, p.N))
         return cudaErrorInvalidValue;
     auto kb = tau ? tc_bwd_kernel<NS, true> : tc_bwd_kernel<NS, false>;
     if ((e = cudaFuncSetAttribute(kb, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return e;
     typedef const __nv_bfloat16* CB;
     const int units = BH * G;
-    kb<<<2 * units, kThreadsB, smem, s>>>(mq, mk, mv, p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k,
+    kb<<<2 * units, kThreadsB, smem, s>>>(mq, mk, mv, mdo, mo, p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k,
                                           (CB)v, W1,
                                           W2, (CB)out, den, (CB)dout, acc_q, acc_k, acc_v, part,
                                           tau ? kw : nullptr, tau, dtau_part, units, status);
