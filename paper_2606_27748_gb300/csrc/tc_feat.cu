@@ -29,7 +29,6 @@ __global__ void __launch_bounds__(kThreadsF)
                       __nv_bfloat16* __restrict__ phi, int* status)
 {
     constexpr int P = NS ? 128 : 64;        // projection rows (= tensor memory columns) per group
-    static_assert(G * P * 8 % kThreadsF == 0, "whole pieces per thread");
     constexpr uint32_t NCOLS = G * P;        // 64, 128 or 256: a power of two
     constexpr uint32_t X0 = 0, W = 32768;    // two x tiles, then G x P frequency rows
     extern __shared__ uint8_t smem_raw[];
@@ -45,44 +44,7 @@ __global__ void __launch_bounds__(kThreadsF)
     const int bh = blockIdx.x / nchunk, b0 = (blockIdx.x % nchunk) * kBlocksPerCta, h = bh % H;
     const int nb = min(kBlocksPerCta, nblk - b0);
 
-    // this head's frequency rows, bf16 K-major (n: U rows then V rows per group), once;
-    // 8-float pieces by float4 loads, a batch of up to 4 pieces per thread in flight
-    constexpr int kPieces = G * P * 8 / kThreadsF, kBatch = kPieces < 4 ? kPieces : 4;
-    for (int i0 = 0; i0 < kPieces; i0 += kBatch) {
-        float4 a[kBatch][2], c2[kBatch][2];
-#pragma unroll
-        for (int i = 0; i < kBatch; ++i) {
-            const int idx = tid + kThreadsF * (i0 + i), r = idx >> 3, c = idx & 7;
-            const int f = 64 * (r / P) + ((r % P) & 63);
-            const float4* w1 = reinterpret_cast<const float4*>(W1 + ((size_t)h * M + f) * 64 + c * 8);
-            a[i][0] = __ldg(w1);
-            a[i][1] = __ldg(w1 + 1);
-            if (NS) {
-                const float4* w2 = reinterpret_cast<const float4*>(W2 + ((size_t)h * M + f) * 64 + c * 8);
-                c2[i][0] = __ldg(w2);
-                c2[i][1] = __ldg(w2 + 1);
-            }
-        }
-#pragma unroll
-        for (int i = 0; i < kBatch; ++i) {
-            const int idx = tid + kThreadsF * (i0 + i), r = idx >> 3, c = idx & 7;
-            const float x0[8] = {a[i][0].x, a[i][0].y, a[i][0].z, a[i][0].w,
-                                 a[i][1].x, a[i][1].y, a[i][1].z, a[i][1].w};
-            float x[8];
-            if (!NS) {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) x[e] = x0[e];
-            } else {
-                const float y0[8] = {c2[i][0].x, c2[i][0].y, c2[i][0].z, c2[i][0].w,
-                                     c2[i][1].x, c2[i][1].y, c2[i][1].z, c2[i][1].w};
-                const float sgn = (r % P) < 64 ? 1.f : -1.f;  // U = (W1+W2)/2, V = (W1-W2)/2
-#pragma unroll
-                for (int e = 0; e < 8; ++e) x[e] = 0.5f * (x0[e] + sgn * y0[e]);
-            }
-            st_shared_v4(sb + W + swz128(r, c * 8), pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]),
-                         pack_bf16(x[4], x[5]), pack_bf16(x[6], x[7]));
-        }
-    }
+    stage_freq_rows<NS, G, kThreadsF>(sb + W, W1, W2, h, M, tid);  // once per CTA
     if (tid == 0) {
         mbar_init(&mbar, 1);
         mbar_init(&tma_bar[0], 1);

@@ -99,6 +99,54 @@ inline bool make_act_map(CUtensorMap* m, const void* base, int BH, int N)
            CUDA_SUCCESS;
 }
 
+// One head's frequency rows into shared memory, bf16, K-major with 128-byte swizzle: G
+// groups of P rows (s: P = 64 rows of W1; n: P = 128, U = (W1+W2)/2 then V = (W1-W2)/2),
+// row r of group g = frequency 64 g + r % 64.  8-float pieces by float4 loads, a batch of
+// up to 4 pieces per thread in flight.  W1, W2: [H][M][64] fp32, 16-byte aligned.
+template <bool NS, int G, int NTHREADS>
+__device__ __forceinline__ void stage_freq_rows(uint32_t dst, const float* W1, const float* W2,
+                                                int h, int M, int tid)
+{
+    constexpr int P = NS ? 128 : 64;
+    static_assert(G * P * 8 % NTHREADS == 0, "whole pieces per thread");
+    constexpr int kPieces = G * P * 8 / NTHREADS, kBatch = kPieces < 4 ? kPieces : 4;
+    for (int i0 = 0; i0 < kPieces; i0 += kBatch) {
+        float4 a[kBatch][2], c2[kBatch][2];
+#pragma unroll
+        for (int i = 0; i < kBatch; ++i) {
+            const int idx = tid + NTHREADS * (i0 + i), r = idx >> 3, c = idx & 7;
+            const int f = 64 * (r / P) + ((r % P) & 63);
+            const float4* w1 = reinterpret_cast<const float4*>(W1 + ((size_t)h * M + f) * 64 + c * 8);
+            a[i][0] = __ldg(w1);
+            a[i][1] = __ldg(w1 + 1);
+            if (NS) {
+                const float4* w2 = reinterpret_cast<const float4*>(W2 + ((size_t)h * M + f) * 64 + c * 8);
+                c2[i][0] = __ldg(w2);
+                c2[i][1] = __ldg(w2 + 1);
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < kBatch; ++i) {
+            const int idx = tid + NTHREADS * (i0 + i), r = idx >> 3, c = idx & 7;
+            const float x0[8] = {a[i][0].x, a[i][0].y, a[i][0].z, a[i][0].w,
+                                 a[i][1].x, a[i][1].y, a[i][1].z, a[i][1].w};
+            float x[8];
+            if (!NS) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) x[e] = x0[e];
+            } else {
+                const float y0[8] = {c2[i][0].x, c2[i][0].y, c2[i][0].z, c2[i][0].w,
+                                     c2[i][1].x, c2[i][1].y, c2[i][1].z, c2[i][1].w};
+                const float sgn = (r % P) < 64 ? 1.f : -1.f;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) x[e] = 0.5f * (x0[e] + sgn * y0[e]);
+            }
+            st_shared_v4(dst + swz128(r, c * 8), pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]),
+                         pack_bf16(x[4], x[5]), pack_bf16(x[6], x[7]));
+        }
+    }
+}
+
 // [BH][N][F] bf16 rows of F features (F a multiple of 64), box 64 x 128, 128B swizzle:
 // a load at x = 64 g brings feature block g of 128 rows.
 inline bool make_feat_map(CUtensorMap* m, const void* base, int BH, int N, int F)
