@@ -194,7 +194,8 @@ int flex_linattn_decode(const flex_shape* shape, const void* q, const void* k, c
         return FLEX_EINVAL;
     if ((rc = check_ws(ws, ws_bytes, header_bytes() + flex::decode_ws_bytes(p)))) return rc;
     return count(2, flex::launch_decode(p, q, k, v, W1, W2, tau, S, z, out, den,
-                                        (char*)ws + header_bytes(), (cudaStream_t)stream));
+                                        (char*)ws + header_bytes(),
+                                        &((flex::WsHeader*)ws)->status, (cudaStream_t)stream));
 }
 
 // Distillation-loss workspace: header, phi(q), phi~(k) [B*H*N][2M] bf16, key weights

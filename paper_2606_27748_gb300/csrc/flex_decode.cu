@@ -24,11 +24,14 @@
 //                    summed in a fixed order (bit-exact repeatable).  A state of more than
 //                    64 KB per (b, h) (M d > 8192) goes through shared memory in row
 //                    chunks.
+#include <cuda.h>
 #include <cuda_bf16.h>
 
 #include <algorithm>
 
 #include "flex_internal.h"
+#include "tc_common.cuh"
+#include "tc_util.cuh"
 
 namespace flex {
 namespace {
@@ -187,6 +190,132 @@ __global__ void __launch_bounds__(kThreadsF, 4)
     }
 }
 
+// The same features on the tensor cores for bf16 token vectors with d = 64: one CTA per
+// (head, 128 sequences, q or k, group of 64 frequencies); the 128 rows arrive by TMA (a
+// strided view of [B][H][64]); the projection x W^T runs on tcgen05 with W split into
+// bf16 high and low parts (x is exactly bf16, so the two MMAs give the fp32 product to
+// about 2^-17) into 64 (s) or 128 (n) tensor-memory columns; every thread takes one
+// sequence and 32 frequencies: sin/cos after the reduction by 2 pi, for k the key weight
+// of the norm prefactor from its row in shared memory, fp32 phi to the workspace.
+template <bool NS, int G>
+__global__ void __launch_bounds__(256)
+    decode_features_tc(const __grid_constant__ CUtensorMap tmap_q,
+                       const __grid_constant__ CUtensorMap tmap_k, int B, int H, int M,
+                       const float* __restrict__ W1, const float* __restrict__ W2,
+                       const float* __restrict__ tau, float* __restrict__ phi, int* status)
+{
+    using namespace tc;
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+    constexpr int P = NS ? 128 : 64;
+    constexpr uint32_t X = 0, WH = 16384, WL = WH + P * 128;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const uint32_t sb = smem_u32(sm);
+    __shared__ uint32_t tmem_base_sh;
+    __shared__ __align__(8) uint64_t mbar, tma_bar;
+    __shared__ volatile int abort_flag;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int wg = warp >> 2, quad = warp & 3, t = 32 * quad + lane;
+    const int nblk = (B + 127) / 128;
+    int u = blockIdx.x;
+    const int g = u % G; u /= G;
+    const int which = u % 2; u /= 2;  // 0: q, 1: k
+    const int blk = u % nblk, h = u / nblk, b0 = blk * 128;
+
+    stage_freq_rows_split<NS, 1, 256>(sb + WH, sb + WL, W1, W2, h, M, tid, 64 * g);
+    if (tid == 0) {
+        mbar_init(&mbar, 1);
+        mbar_init(&tma_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+        mbar_arrive_expect_tx(&tma_bar, kTileBytes);
+        tma_load_3d(sb + X, which ? &tmap_k : &tmap_q, 0, h, b0, &tma_bar);
+    }
+    if (warp == 0) {
+        tmem_alloc(&tmem_base_sh, P);
+        tmem_relinquish();
+    }
+    fence_proxy_async();
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    const uint32_t tm = tmem_base_sh;
+    const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
+
+    bool ok = bar_wait(&tma_bar, 0, &abort_flag, status);
+    ok = !__syncthreads_or(!ok);
+    if (ok) {
+        fence_after_sync();
+        if (tid == 0) {
+            constexpr uint32_t I_PROJ = idesc_bf16(128, P, 0, 0);
+            const uint64_t dX = sdesc(sb + X, 16, 1024);
+            const uint64_t dH = sdesc(sb + WH, 16, 1024), dL = sdesc(sb + WL, 16, 1024);
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks)
+                mma_bf16(tm, dX + ((ks * 32) >> 4), dH + ((ks * 32) >> 4), I_PROJ, ks > 0);
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks)
+                mma_bf16(tm, dX + ((ks * 32) >> 4), dL + ((ks * 32) >> 4), I_PROJ, 1u);
+            mma_commit(&mbar);
+        }
+        ok = bar_wait(&mbar, 0, &abort_flag, status);
+        ok = !__syncthreads_or(!ok);
+    }
+    if (ok) {
+        fence_after_sync();
+        const int b = b0 + t, F = 2 * M;
+        const bool valid = b < B;
+        float wsc = rsqrtf((float)M);
+        if (which == 1 && tau) {  // key weight exp(|k|^2 exp(-tau)) from this k row
+            float n2 = 0.f;
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const uint4 q4 = *reinterpret_cast<const uint4*>(sm + X + swz128(t, 8 * c));
+                const uint32_t wv[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float lo = __uint_as_float(wv[e] << 16), hi = __uint_as_float(wv[e] & 0xffff0000u);
+                    n2 = fmaf(lo, lo, fmaf(hi, hi, n2));
+                }
+            }
+            wsc *= expf(n2 * expf(-tau[h]));
+        }
+        float a[32], w[32];
+        const uint32_t col = tm_row + 32 * wg;
+        tmem_ld16(col, *reinterpret_cast<float(*)[16]>(&a[0]));
+        tmem_ld16(col + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+        if (NS) {
+            tmem_ld16(col + 64, *reinterpret_cast<float(*)[16]>(&w[0]));
+            tmem_ld16(col + 80, *reinterpret_cast<float(*)[16]>(&w[16]));
+        }
+        tmem_wait_ld();
+        float pc[32], ps[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+            float su, cu, sw, cw = 1.f;
+            sincos_reduced(a[i], &su, &cu);
+            if (NS) sincos_reduced(w[i], &sw, &cw);
+            pc[i] = cu * cw * wsc;
+            ps[i] = su * cw * wsc;
+        }
+        if (valid) {
+            float* dst = phi + (((size_t)b * H + h) * 2 + which) * F + 64 * g + 32 * wg;
+            float4* dc = reinterpret_cast<float4*>(dst);
+            float4* ds = reinterpret_cast<float4*>(dst + M);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                dc[j] = make_float4(pc[4 * j], pc[4 * j + 1], pc[4 * j + 2], pc[4 * j + 3]);
+                ds[j] = make_float4(ps[4 * j], ps[4 * j + 1], ps[4 * j + 2], ps[4 * j + 3]);
+            }
+        }
+    }
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    if (warp == 0) tmem_dealloc(tm, P);
+}
+
 template <typename T>
 __global__ void __launch_bounds__(kThreadsD, 3)
     decode_state(int d, int M, const T* __restrict__ v, const float* phi,
@@ -281,25 +410,53 @@ __global__ void __launch_bounds__(kThreadsD, 3)
     }
 }
 
+template <bool NS, int G>
+cudaError_t launch_features_tc(const Problem& p, const void* q, const void* k, const float* W1,
+                               const float* W2, const float* tau, float* phi, int* status,
+                               cudaStream_t s)
+{
+    CUtensorMap mq, mk;
+    if (!tc::make_head_rows_map(&mq, q, p.B, p.H) || !tc::make_head_rows_map(&mk, k, p.B, p.H))
+        return cudaErrorInvalidValue;
+    constexpr int P = NS ? 128 : 64;
+    const int smem = 16384 + 2 * P * 128 + 1024;
+    auto kern = decode_features_tc<NS, G>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    const long long ctas = (long long)p.H * ((p.B + 127) / 128) * 2 * G;
+    if (ctas > 0x7fffffffLL) return cudaErrorInvalidValue;
+    kern<<<(unsigned)ctas, 256, smem, s>>>(mq, mk, p.B, p.H, p.M, W1, W2, tau, phi, status);
+    return cudaGetLastError();
+}
+
 template <typename T, bool NS>
 cudaError_t launch_typed(const Problem& p, const void* q, const void* k, const void* v,
                          const float* W1, const float* W2, const float* tau, float* S,
-                         float* z, void* out, float* den, float* phi, cudaStream_t s)
+                         float* z, void* out, float* den, float* phi, int* status,
+                         cudaStream_t s)
 {
     const long long fctas = (long long)p.H * ((p.B + kG - 1) / kG) * ((p.M + kTF - 1) / kTF);
     const long long sctas = (long long)p.B * p.H;
     if (fctas > 0x7fffffffLL || sctas > 0x7fffffffLL) return cudaErrorInvalidValue;
 
-    const size_t fsmem = ((size_t)kTF * (p.d + 4) * 2 + 2 * kG * p.d + 2 * kG) * sizeof(float);
-    auto fk = p.d == 32    ? decode_features<T, NS, 8>
-              : p.d == 64  ? decode_features<T, NS, 16>
-              : p.d == 128 ? decode_features<T, NS, 32>
-                           : decode_features<T, NS, 0>;
-    cudaError_t e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fsmem);
-    if (e != cudaSuccess) return e;
-    fk<<<(unsigned)fctas, kThreadsF, fsmem, s>>>(p.B, p.H, p.d, p.M, (const T*)q, (const T*)k,
-                                                W1, W2, tau, phi);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    cudaError_t e;
+    if (p.bf16 && p.d == 64 && (p.M == 64 || p.M == 128)) {  // tensor-core features
+        e = p.M == 64 ? launch_features_tc<NS, 1>(p, q, k, W1, W2, tau, phi, status, s)
+                      : launch_features_tc<NS, 2>(p, q, k, W1, W2, tau, phi, status, s);
+        if (e != cudaSuccess) return e;
+    } else {
+        const size_t fsmem =
+            ((size_t)kTF * (p.d + 4) * 2 + 2 * kG * p.d + 2 * kG) * sizeof(float);
+        auto fk = p.d == 32    ? decode_features<T, NS, 8>
+                  : p.d == 64  ? decode_features<T, NS, 16>
+                  : p.d == 128 ? decode_features<T, NS, 32>
+                               : decode_features<T, NS, 0>;
+        e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fsmem);
+        if (e != cudaSuccess) return e;
+        fk<<<(unsigned)fctas, kThreadsF, fsmem, s>>>(p.B, p.H, p.d, p.M, (const T*)q,
+                                                    (const T*)k, W1, W2, tau, phi);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
 
     const size_t ssmem = (size_t)std::min(2 * p.M, kSBuf / p.d) * p.d * sizeof(float);
     auto sk = decode_state<T>;
@@ -326,16 +483,19 @@ size_t decode_ws_bytes(const Problem& p) { return (size_t)p.B * p.H * 2 * 2 * p.
 
 cudaError_t launch_decode(const Problem& p, const void* q, const void* k, const void* v,
                           const float* W1, const float* W2, const float* tau, float* S,
-                          float* z, void* out, float* den, void* scratch, cudaStream_t s)
+                          float* z, void* out, float* den, void* scratch, int* status,
+                          cudaStream_t s)
 {
     float* phi = (float*)scratch;
     if (p.bf16)
         return p.nonstat ? launch_typed<__nv_bfloat16, true>(p, q, k, v, W1, W2, tau, S, z, out,
-                                                             den, phi, s)
+                                                             den, phi, status, s)
                          : launch_typed<__nv_bfloat16, false>(p, q, k, v, W1, W2, tau, S, z,
-                                                              out, den, phi, s);
-    return p.nonstat ? launch_typed<float, true>(p, q, k, v, W1, W2, tau, S, z, out, den, phi, s)
-                     : launch_typed<float, false>(p, q, k, v, W1, W2, tau, S, z, out, den, phi, s);
+                                                              out, den, phi, status, s);
+    return p.nonstat
+               ? launch_typed<float, true>(p, q, k, v, W1, W2, tau, S, z, out, den, phi, status, s)
+               : launch_typed<float, false>(p, q, k, v, W1, W2, tau, S, z, out, den, phi, status,
+                                            s);
 }
 
 }  // namespace flex

@@ -61,7 +61,8 @@ cudaError_t launch_key_weights(const Problem& p, const void* k, const float* tau
 size_t decode_ws_bytes(const Problem& p);  // phi(q), phi(k) of the step, fp32
 cudaError_t launch_decode(const Problem& p, const void* q, const void* k, const void* v,
                           const float* W1, const float* W2, const float* tau, float* S,
-                          float* z, void* out, float* den, void* scratch, cudaStream_t s);
+                          float* z, void* out, float* den, void* scratch, int* status,
+                          cudaStream_t s);
 
 // ---- tensor-core path (bf16 storage, d = 64, M in {64, 128}) ------------------------
 bool tc_fwd_supported(const Problem& p);

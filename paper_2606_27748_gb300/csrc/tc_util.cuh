@@ -147,6 +147,43 @@ __device__ __forceinline__ void stage_freq_rows(uint32_t dst, const float* W1, c
     }
 }
 
+// The same rows split into bf16 high and low parts (x = hi + lo to about 2^-17): hi at
+// dst_hi, lo at dst_lo, both in the layout above; frequencies from f0 on.  Two MMAs (hi, lo) against an exactly
+// representable bf16 operand reproduce the fp32 product to that accuracy.
+template <bool NS, int G, int NTHREADS>
+__device__ __forceinline__ void stage_freq_rows_split(uint32_t dst_hi, uint32_t dst_lo,
+                                                      const float* W1, const float* W2, int h,
+                                                      int M, int tid, int f0 = 0)
+{
+    constexpr int P = NS ? 128 : 64;
+    static_assert(G * P * 8 % NTHREADS == 0, "whole pieces per thread");
+    constexpr int kPieces = G * P * 8 / NTHREADS;
+    for (int i = 0; i < kPieces; ++i) {
+        const int idx = tid + NTHREADS * i, r = idx >> 3, c = idx & 7;
+        const int f = f0 + 64 * (r / P) + ((r % P) & 63);
+        const float4* w1 = reinterpret_cast<const float4*>(W1 + ((size_t)h * M + f) * 64 + c * 8);
+        const float4 a0 = __ldg(w1), a1 = __ldg(w1 + 1);
+        float x[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+        if (NS) {
+            const float4* w2 = reinterpret_cast<const float4*>(W2 + ((size_t)h * M + f) * 64 + c * 8);
+            const float4 b0 = __ldg(w2), b1 = __ldg(w2 + 1);
+            const float y[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+            const float sgn = (r % P) < 64 ? 1.f : -1.f;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) x[e] = 0.5f * (x[e] + sgn * y[e]);
+        }
+        uint32_t hi[4], lo[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            hi[e] = pack_bf16(x[2 * e], x[2 * e + 1]);
+            const float h0 = __uint_as_float(hi[e] << 16), h1 = __uint_as_float(hi[e] & 0xffff0000u);
+            lo[e] = pack_bf16(x[2 * e] - h0, x[2 * e + 1] - h1);
+        }
+        st_shared_v4(dst_hi + swz128(r, c * 8), hi[0], hi[1], hi[2], hi[3]);
+        st_shared_v4(dst_lo + swz128(r, c * 8), lo[0], lo[1], lo[2], lo[3]);
+    }
+}
+
 // [BH][N][F] bf16 rows of F features (F a multiple of 64), box 64 x 128, 128B swizzle:
 // a load at x = 64 g brings feature block g of 128 rows.
 inline bool make_feat_map(CUtensorMap* m, const void* base, int BH, int N, int F)
@@ -156,6 +193,22 @@ inline bool make_feat_map(CUtensorMap* m, const void* base, int BH, int N, int F
     cuuint64_t dims[3] = {(cuuint64_t)F, (cuuint64_t)N, (cuuint64_t)BH};
     cuuint64_t strides[2] = {(cuuint64_t)F * 2, (cuuint64_t)N * F * 2};
     cuuint32_t box[3] = {64, 128, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+               box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
+}
+
+// [B][H][64] bf16 token vectors of one step, viewed per head: box (64, 1 head, 128 batch
+// entries), 128B swizzle: a load at (0, h, b0) brings 128 rows of head h.
+inline bool make_head_rows_map(CUtensorMap* m, const void* base, int B, int H)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {64, (cuuint64_t)H, (cuuint64_t)B};
+    cuuint64_t strides[2] = {128, (cuuint64_t)H * 128};
+    cuuint32_t box[3] = {64, 1, 128};
     cuuint32_t es[3] = {1, 1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
                box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
