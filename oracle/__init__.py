@@ -72,8 +72,10 @@ class Oracle:
         lib.oracle_linattn_decode.argtypes = [i, i, i, i, dp, dp, dp, dp, dp, dp, dp, dp, dp,
                                               dp]
         lib.oracle_awd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, i, dp]
+        lib.oracle_awd_bwd.argtypes = [i, i, i, i, i, dp, dp, dp, dp, dp, i, dp, dp, dp, dp]
         for fn in (lib.oracle_featmap, lib.oracle_featmap_sumform, lib.oracle_linattn_fwd,
-                   lib.oracle_linattn_bwd, lib.oracle_linattn_decode, lib.oracle_awd):
+                   lib.oracle_linattn_bwd, lib.oracle_linattn_decode, lib.oracle_awd,
+                   lib.oracle_awd_bwd):
             fn.restype = ctypes.c_int
         self._lib = lib
         self.path = path
@@ -183,6 +185,24 @@ class Oracle:
             raise ValueError("oracle_awd: bad shape")
         return loss
 
+    def awd_bwd(self, q, k, W1, W2=None, causal=False, tau=None, dloss=None):
+        """Gradient of sum_{b,h} dloss[b, h] * awd(...)[b, h] with respect to the kernel's
+        parameters: (dW1 [H, M, d], dW2 [H, M, d] or None, dtau [H] or None).  dloss
+        defaults to ones."""
+        q, k, W1, W2, tau = (self._f64(a) for a in (q, k, W1, W2, tau))
+        B, H, N, d = q.shape
+        M = W1.shape[1]
+        dl = self._f64(np.ones((B, H)) if dloss is None else np.broadcast_to(dloss, (B, H)))
+        dW1 = np.empty_like(W1)
+        dW2 = None if W2 is None else np.empty_like(W2)
+        dtau = None if tau is None else np.empty(H)
+        rc = self._lib.oracle_awd_bwd(B, H, N, d, M, self._p(q), self._p(k), self._p(W1),
+                                      self._p(W2), self._p(tau), int(bool(causal)),
+                                      self._p(dl), self._p(dW1), self._p(dW2), self._p(dtau))
+        if rc != 0:
+            raise ValueError("oracle_awd_bwd: bad shape")
+        return dW1, dW2, dtau
+
 
 def load() -> Oracle:
     """The oracle built from ``flex_oracle.c`` (compiled on first use if needed)."""
@@ -213,3 +233,7 @@ def decode(q, k, v, W1, W2, S, z, tau=None):
 
 def awd(q, k, W1, W2=None, causal=False, tau=None):
     return load().awd(q, k, W1, W2, causal, tau)
+
+
+def awd_bwd(q, k, W1, W2=None, causal=False, tau=None, dloss=None):
+    return load().awd_bwd(q, k, W1, W2, causal, tau, dloss)

@@ -511,6 +511,106 @@ int oracle_awd(int B, int H, int N, int d, int M, const double* q, const double*
     return 0;
 }
 
+/* Gradient of the distillation loss with respect to the kernel's parameters (the
+ * distillation trains only the feature map: W1, W2 and tau; q and k are frozen).
+ * For an entry with R_ij > 0, log R_ij = log|A~_ij| - log|D_i|; entries with R_ij <= 0
+ * are constant.  With c_i = sum of P_ij over the entries with R_ij > 0 and the upstream
+ * gradient dl of this sequence's loss:
+ *   dL/dA~_ij = -(dl/N) ( [R_ij > 0] P_ij / A~_ij  -  c_i / D_i )     (j in the row)
+ * (the second term from D_i = sum_j A~_ij), then
+ *   dphi(q_i) = sum_j dA~_ij phi~(k_j),   dphi~(k_j) = sum_i dA~_ij phi(q_i),
+ *   dphi(k_j) = w_j dphi~(k_j),   dtau += -(phi~(k_j) . dphi~(k_j)) |k_j|^2 exp(-tau)
+ * (from dw_j/dtau = -w_j |k_j|^2 exp(-tau)), and the feature map's chain rule into dA, dB
+ * ([M][d], as in the attention backward). */
+static void awd_grad_seq(int N, int d, int M, int causal, const double* q, const double* k,
+                         const double* W1, const double* W2, double itau, double dl,
+                         double* dA, double* dB, double* dtau)
+{
+    const int D = 2 * M;
+    double* PQ = malloc(sizeof(double) * (size_t)N * D);
+    double* PK = malloc(sizeof(double) * (size_t)N * D);
+    double* dPQ = calloc((size_t)N * D, sizeof(double));
+    double* dPK = calloc((size_t)N * D, sizeof(double));
+    double* wk = malloc(sizeof(double) * (size_t)N);
+    double* sc = malloc(sizeof(double) * (size_t)N);
+    double* at = malloc(sizeof(double) * (size_t)N);
+    double* P = malloc(sizeof(double) * (size_t)N);
+    double* dx = calloc((size_t)d, sizeof(double));  /* dq, dk: not needed, discarded */
+    for (int i = 0; i < N; ++i) {
+        feature(d, M, q + (size_t)i * d, W1, W2, PQ + (size_t)i * D);
+        feature(d, M, k + (size_t)i * d, W1, W2, PK + (size_t)i * D);
+        wk[i] = key_weight(d, k + (size_t)i * d, itau);
+        for (int f = 0; f < D; ++f) PK[(size_t)i * D + f] *= wk[i];
+    }
+    for (int i = 0; i < N; ++i) {
+        const int J = causal ? i + 1 : N;
+        double smax = -INFINITY, Dn = 0.0, Z = 0.0, ci = 0.0;
+        for (int j = 0; j < J; ++j) {
+            sc[j] = dot(d, q + (size_t)i * d, k + (size_t)j * d) / sqrt((double)d);
+            at[j] = dot(D, PQ + (size_t)i * D, PK + (size_t)j * D);
+            if (sc[j] > smax) smax = sc[j];
+            Dn += at[j];
+        }
+        for (int j = 0; j < J; ++j) Z += exp(sc[j] - smax);
+        for (int j = 0; j < J; ++j) {
+            P[j] = exp(sc[j] - smax) / Z;
+            if (at[j] / Dn > 0.0) ci += P[j];
+        }
+        for (int j = 0; j < J; ++j) {
+            const double first = at[j] / Dn > 0.0 ? P[j] / at[j] : 0.0;
+            const double g = -(dl / N) * (first - ci / Dn);
+            for (int f = 0; f < D; ++f) {
+                dPQ[(size_t)i * D + f] += g * PK[(size_t)j * D + f];
+                dPK[(size_t)j * D + f] += g * PQ[(size_t)i * D + f];
+            }
+        }
+    }
+    for (int i = 0; i < N; ++i) {
+        feature_backward(d, M, q + (size_t)i * d, W1, W2, dPQ + (size_t)i * D, dx, dA, dB);
+        const double* kj = k + (size_t)i * d;
+        double s = dot(D, PK + (size_t)i * D, dPK + (size_t)i * D);
+        if (dtau) *dtau += -s * dot(d, kj, kj) * itau;
+        for (int f = 0; f < D; ++f) dPK[(size_t)i * D + f] *= wk[i];
+        feature_backward(d, M, kj, W1, W2, dPK + (size_t)i * D, dx, dA, dB);
+    }
+    free(PQ); free(PK); free(dPQ); free(dPK); free(wk); free(sc); free(at); free(P); free(dx);
+}
+
+/* dW1, dW2 [H][M][d] (dW2 only with W2) and dtau [H] (only with tau): the gradient of
+ * sum_{b,h} dloss[b][h] L[b][h] with L the distillation loss of oracle_awd. */
+int oracle_awd_bwd(int B, int H, int N, int d, int M, const double* q, const double* k,
+                   const double* W1, const double* W2, const double* tau, int causal,
+                   const double* dloss, double* dW1, double* dW2, double* dtau)
+{
+    if (bad_shape(B, H, N, d, M)) return -1;
+    const size_t per = (size_t)M * d;
+    double* dA = malloc(sizeof(double) * per);
+    double* dB = malloc(sizeof(double) * per);
+    for (int h = 0; h < H; ++h) {
+        memset(dA, 0, sizeof(double) * per);
+        memset(dB, 0, sizeof(double) * per);
+        double dt = 0.0;
+        const double* w1 = W1 + (size_t)h * per;
+        const double* w2 = W2 ? W2 + (size_t)h * per : NULL;
+        for (int b = 0; b < B; ++b) {
+            const size_t u = (size_t)b * H + h, off = u * N * d;
+            awd_grad_seq(N, d, M, causal, q + off, k + off, w1, w2, tau ? exp(-tau[h]) : 0.0,
+                         dloss[u], dA, dB, tau ? &dt : NULL);
+        }
+        for (size_t t = 0; t < per; ++t) {
+            if (W2 == NULL) {
+                dW1[h * per + t] = dA[t];
+            } else {               /* U = (W1+W2)/2, V = (W1-W2)/2 */
+                dW1[h * per + t] = 0.5 * (dA[t] + dB[t]);
+                dW2[h * per + t] = 0.5 * (dA[t] - dB[t]);
+            }
+        }
+        if (tau) dtau[h] = dt;
+    }
+    free(dA); free(dB);
+    return 0;
+}
+
 /* One step of the causal recurrence behind Eq. (linear att) with j <= i: the running sums
  * S = sum_j phi(k_j) v_j^T and z = sum_j phi(k_j) absorb the new token (inclusive), then
  * out = phi(q)^T S / den with den = phi(q)^T z.  Per (b, h): q, k, v, out [d]; S [2M][d]

@@ -33,6 +33,9 @@ Facts used (none is the oracle's own formula retyped):
     0; d = 1, M = 1 in closed form (cos kernel, softmax teacher); Gibbs' inequality
     (loss >= the teacher's entropy); keys of equal norm make tau irrelevant; entries with
     a non-positive normalised weight count log 1e-6 in both forms.
+  * its gradient with respect to W1, W2 and tau: central finite differences of the numpy
+    form (cases with negative kernel entries); one key gives 0; keys of equal norm give
+    dtau = 0; W2 = W1 gives dW1 + dW2 = the stationary gradient.
 """
 from __future__ import annotations
 
@@ -399,6 +402,83 @@ def pin_awd_nonpositive_entries(orc):
     assert _rel(orc.awd(q, k, W1), brute.awd_loss(q, k, W1)) < 1e-12, "awd clamp"
 
 
+# -------------------------------------------------------------------------------------
+# Gradient of the distillation loss with respect to the kernel's parameters (W1, W2,
+# tau): the distillation trains only the feature map, q and k are frozen.
+# -------------------------------------------------------------------------------------
+def _awd_case(variant):
+    """Small case with negative kernel estimates (and, for s, negative row sums) but no
+    normalised weight near 0, so central differences do not straddle the clamp."""
+    seed = 124 if variant == "s" else 109
+    q, k, _, W1, W2 = _case(seed, 2, 2, 6, 3, 4, variant, qk_scale=1.0)
+    return q, k, W1 * 1.5, None if W2 is None else W2 * 1.5
+
+
+def pin_awd_grad_finite_differences(orc):
+    """dW1, dW2, dtau against central differences of the numpy explicit-matrix loss
+    (sum form of the nonstationary features, prefactor on queries and keys as printed),
+    weighted by a random upstream gradient per sequence."""
+    h = 1e-6
+    dl = _rng(75).standard_normal((2, 2))
+    for variant in ("s", "n"):
+        q, k, W1, W2 = _awd_case(variant)
+        K = brute.kernel_matrix(q, k, W1, W2)
+        assert np.any(K < 0), "the case needs negative kernel entries"
+        for causal in (False, True):
+            for tau in (None, _TAU.copy()):
+                def total():
+                    return float(np.sum(dl * brute.awd_loss(q, k, W1, W2, causal, tau=tau)))
+                grads = orc.awd_bwd(q, k, W1, W2, causal, tau=tau, dloss=dl)
+                params = [(W1, grads[0])]
+                if W2 is not None:
+                    params.append((W2, grads[1]))
+                if tau is not None:
+                    params.append((tau, grads[2]))
+                for idx, (p, gp) in enumerate(params):
+                    fd = np.zeros_like(p)
+                    it = np.nditer(p, flags=["multi_index"])
+                    for _ in it:
+                        mi = it.multi_index
+                        old = p[mi]
+                        p[mi] = old + h
+                        lp = total()
+                        p[mi] = old - h
+                        lm = total()
+                        p[mi] = old
+                        fd[mi] = (lp - lm) / (2 * h)
+                    err = np.linalg.norm(gp - fd) / np.linalg.norm(fd)
+                    assert err < 1e-6, (f"awd grad FD {variant} causal={causal} "
+                                        f"tau={tau is not None} #{idx}: {err:.2e}")
+
+
+def pin_awd_grad_single_key(orc):
+    """One key: R = 1 whatever the parameters, so every gradient is exactly 0."""
+    q, k, _, W1, W2 = _case(76, 2, 2, 1, 5, 7, "n")
+    dW1, dW2, dtau = orc.awd_bwd(q, k, W1, W2, tau=_TAU)
+    assert np.all(dW1 == 0.0) and np.all(dW2 == 0.0) and np.all(dtau == 0.0), "awd grad N=1"
+
+
+def pin_awd_grad_equal_key_norms(orc):
+    """Keys of one norm: the prefactor is a common factor of each row of R, so the loss
+    does not depend on tau and dtau = 0 (the -c_i/D_i term must cancel the P/A term)."""
+    for causal in (False, True):
+        q, k, _, W1, W2 = _case(77, 2, 2, 19, 5, 7, "n")
+        k = k / np.linalg.norm(k, axis=-1, keepdims=True) * 1.3
+        dW1, _, dtau = orc.awd_bwd(q, k, W1, W2, causal, tau=_TAU)
+        assert np.all(np.abs(dtau) < 1e-11 * np.abs(dW1).sum()), "awd dtau, equal norms"
+        assert np.abs(dW1).sum() > 1e-6, "the case needs a nonzero gradient"
+
+
+def pin_awd_grad_tied_frequencies(orc):
+    """W2 = W1 reduces Flexformer_n to Flexformer_s at W1, so moving both together is
+    moving the stationary frequencies: dW1_n + dW2_n = dW_s."""
+    for causal in (False, True):
+        q, k, _, W1, _ = _case(78, 2, 2, 13, 5, 7, "s")
+        dn1, dn2, _ = orc.awd_bwd(q, k, W1, W1.copy(), causal)
+        ds, _, _ = orc.awd_bwd(q, k, W1, None, causal)
+        assert _rel(dn1 + dn2, ds) < 1e-12, "awd grad W2 = W1"
+
+
 ALL_PINS = [
     pin_origin_features, pin_stationary_unit_norm, pin_sum_to_product, pin_w2_equals_w1,
     pin_bochner, pin_yaglom, pin_linear_equals_brute, pin_decode_equals_brute,
@@ -408,5 +488,6 @@ ALL_PINS = [
     pin_prefactor_vanishes_as_tau_grows, pin_prefactor_equal_key_norms,
     pin_prefactor_finite_differences, pin_prefactor_scaling_identity, pin_prefactor_decode,
     pin_awd_equals_brute, pin_awd_single_key, pin_awd_closed_form_d1, pin_awd_gibbs,
-    pin_awd_equal_key_norms, pin_awd_nonpositive_entries,
+    pin_awd_equal_key_norms, pin_awd_nonpositive_entries, pin_awd_grad_finite_differences,
+    pin_awd_grad_single_key, pin_awd_grad_equal_key_norms, pin_awd_grad_tied_frequencies,
 ]

@@ -60,6 +60,26 @@ MUTATIONS = [
     ("awd_unweighted_keys", "for (int f = 0; f < D; ++f) PK[(size_t)i * D + f] *= wk;\n    }\n    double loss",
      "for (int f = 0; f < D; ++f) PK[(size_t)i * D + f] *= 1.0;\n    }\n    double loss", 0),
     ("awd_clamp_value", "(r > 0.0 ? log(r) : log(AWD_EPS))", "(r > 0.0 ? log(r) : log(1e-3))", 0),
+    ("awdgrad_drop_row_sum_term", "const double g = -(dl / N) * (first - ci / Dn);",
+     "const double g = -(dl / N) * (first);", 0),
+    ("awdgrad_no_clamp_mask", "const double first = at[j] / Dn > 0.0 ? P[j] / at[j] : 0.0;",
+     "const double first = P[j] / at[j];", 0),
+    ("awdgrad_c_over_all_entries", "if (at[j] / Dn > 0.0) ci += P[j];", "ci += P[j];", 0),
+    ("awdgrad_dtau_sign", "if (dtau) *dtau += -s * dot(d, kj, kj) * itau;",
+     "if (dtau) *dtau += s * dot(d, kj, kj) * itau;", 0),
+    ("awdgrad_key_chain_unweighted", "for (int f = 0; f < D; ++f) dPK[(size_t)i * D + f] *= wk[i];",
+     "for (int f = 0; f < D; ++f) dPK[(size_t)i * D + f] *= 1.0;", 0),
+    ("awdgrad_dtau_weight_twice", "double s = dot(D, PK + (size_t)i * D, dPK + (size_t)i * D);",
+     "double s = dot(D, PK + (size_t)i * D, dPK + (size_t)i * D) * wk[i];", 0),
+    ("awdgrad_causal_mask_exclusive",
+     "const int J = causal ? i + 1 : N;\n        double smax = -INFINITY, Dn = 0.0, Z = 0.0, ci",
+     "const int J = causal ? (i > 0 ? i : 1) : N;\n        double smax = -INFINITY, Dn = 0.0, Z = 0.0, ci", 0),
+    ("awdgrad_ignores_dloss", "const double g = -(dl / N)", "const double g = -(1.0 / N)", 0),
+    ("awdgrad_w2_sign", "dW2[h * per + t] = 0.5 * (dA[t] - dB[t]);",
+     "dW2[h * per + t] = 0.5 * (dB[t] - dA[t]);", 0),
+    ("awdgrad_drop_query_side",
+     "feature_backward(d, M, q + (size_t)i * d, W1, W2, dPQ + (size_t)i * D, dx, dA, dB);",
+     "(void)dPQ;", 0),
 ]
 
 
