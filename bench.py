@@ -38,6 +38,8 @@ METRIC_DECODE = ("RFF linear-attn recurrent decode tokens/s (one new token per s
                  "running state) & % of HBM roofline")
 METRIC_AWD = ("RFF attention-weight distillation loss tokens/s (softmax teacher vs kernel "
               "weights, blockwise N x N) & % of roofline")
+METRIC_AWD_TRAIN = ("RFF attention-weight distillation training-step tokens/s (loss and its "
+                    "gradient w.r.t. the frequencies, blockwise N x N) & % of roofline")
 L2_BYTES = 129e6
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
@@ -286,7 +288,8 @@ def run_reference(args, w):
                    for _ in range(args.steps)) / args.steps
         value = nseq * w.N / w.H / step
         print(json.dumps({
-            "metric": METRIC_AWD, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "metric": METRIC_AWD_TRAIN if w.backward else METRIC_AWD, "value": value,
+            "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
@@ -664,20 +667,29 @@ def run_decode(args, w):
 # Attention-weight distillation loss: a step is the loss of every sequence of the batch.
 # ---------------------------------------------------------------------------------------
 def awd_work(w):
-    """(bytes, flops, sin/cos+exp/log) per step: q, k read, the loss written; the score and
-    kernel contractions over the (masked) pairs plus the feature projections; per pair one
-    exp and one log, per token and frequency 2 (s) or 3 (n) sin/cos for q and for k."""
+    """(bytes, flops, sin/cos+exp/log/reciprocal) per step: q, k read, the loss written; the
+    score and kernel contractions over the (masked) pairs plus the feature projections; per
+    pair one exp and one log, per token and frequency 2 (s) or 3 (n) sin/cos for q and for
+    k.  A training step (w.backward) adds the gradient: W read and dW written; per pair and
+    side the score and kernel contractions again and G phi (2M features), one exp and one
+    reciprocal; per token and side the projection and dW' = da^T x (2 P d each, P = M (s)
+    or 2M (n)) and the sin/cos of the chain rule."""
     bh, N = w.B * w.H, w.N
     pairs = bh * (N * (N + 1) // 2 if w.causal else N * N)
     c = 2 if w.variant == "n" else 1
     nbytes = bh * N * w.d * elem_bytes(w) * 2 + bh * 4
     flops = 2 * pairs * (w.d + 2 * w.M) + 2 * bh * N * 2 * w.d * w.M * c
     ops = 2 * pairs + bh * N * 2 * w.M * (3 if w.variant == "n" else 2)
+    if w.backward:
+        nbytes += 2 * c * w.H * w.M * w.d * 4
+        flops += 2 * (2 * pairs * (w.d + 4 * w.M)) + 2 * (2 * bh * N * 2 * c * w.M * w.d)
+        ops += 2 * (2 * pairs) + 2 * bh * N * w.M * (4 if w.variant == "n" else 2)
     return nbytes, flops, ops
 
 
 def oracle_awd_sample(w, nseq, prefactor=False):
-    """Seconds of the oracle loss over the first `nseq` sequences (one thread)."""
+    """Seconds of the oracle loss (and, for a training step, its gradient) over the first
+    `nseq` sequences (one thread)."""
     import oracle
     nb = -(-nseq // w.H)
     ins = workloads.make_inputs(w, bs=range(nb))
@@ -688,6 +700,8 @@ def oracle_awd_sample(w, nseq, prefactor=False):
     tau = workloads.draw_tau(w)[heads] if prefactor else None
     t0 = time.perf_counter()
     oracle.awd(q, k, W1, W2, w.causal, tau=tau)
+    if w.backward:
+        oracle.awd_bwd(q, k, W1, W2, w.causal, tau=tau)
     return time.perf_counter() - t0
 
 
@@ -718,13 +732,24 @@ def run_awd(args, w):
     del ins
     tau = torch.from_numpy(workloads.draw_tau(w)).to(dev) if args.prefactor else None
     shape = flexattn.shape_of(q, W1)
-    ws = flexattn.awd_workspace(shape, dev)
+    train = w.backward  # loss and its gradient (mean over the sequences) per step
+    ws = (flexattn.awd_bwd_workspace if train else flexattn.awd_workspace)(shape, dev)
     loss = torch.empty(w.B, w.H, dtype=torch.float32, device=dev)
+    dloss = torch.full((w.B, w.H), 1.0 / (w.B * w.H), dtype=torch.float32, device=dev)
+    grads = [torch.empty_like(W1)] + ([torch.empty_like(W2)] if W2 is not None else [])
+    dtau = torch.empty_like(tau) if tau is not None else None
+    if dtau is not None:
+        grads.append(dtau)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > L2: a cold step
     stream = torch.cuda.current_stream()
 
     def step():
-        flexattn.awd_loss(q, k, W1, W2, w.causal, tau=tau, loss=loss, ws=ws)
+        if train:
+            flexattn.awd_loss_bwd(q, k, W1, W2, w.causal, tau=tau, dloss=dloss, loss=loss,
+                                  dW1=grads[0], dW2=grads[1] if W2 is not None else None,
+                                  dtau=dtau, ws=ws)
+        else:
+            flexattn.awd_loss(q, k, W1, W2, w.causal, tau=tau, loss=loss, ws=ws)
 
     def barrier():
         if world > 1:
@@ -757,14 +782,16 @@ def run_awd(args, w):
     value = job_value(world, w.tokens, kernel_ms)
 
     e2e = None
-    if not args.no_e2e:  # q, k from pinned host memory, the losses back
-        host_out = torch.empty(loss.shape, dtype=loss.dtype).pin_memory()
+    if not args.no_e2e:  # q, k from pinned host memory, the losses (and gradients) back
+        results = [loss] + (grads if train else [])
+        host_outs = [torch.empty(r.shape, dtype=r.dtype).pin_memory() for r in results]
 
         def e2e_step():
             q.copy_(host["q"], non_blocking=True)
             k.copy_(host["k"], non_blocking=True)
             step()
-            host_out.copy_(loss, non_blocking=True)
+            for ho, r in zip(host_outs, results):
+                ho.copy_(r, non_blocking=True)
 
         for _ in range(max(3, args.warmup)):
             e2e_step()
@@ -783,7 +810,7 @@ def run_awd(args, w):
         e2e_ms = max_over_ranks([tot / K], world, dev)[0]
         e2e = {"value": job_value(world, w.tokens, e2e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": sum(t.numel() * t.element_size() for t in host.values()),
-               "d2h_bytes_per_step": host_out.numel() * host_out.element_size()}
+               "d2h_bytes_per_step": sum(t.numel() * t.element_size() for t in host_outs)}
 
     peaks, peaks_src = load_peaks()
     nbytes, flops, ops = awd_work(w)
@@ -801,13 +828,13 @@ def run_awd(args, w):
             "algorithmic_flops_per_launch": flops, "sfu_ops_per_launch": ops,
             "time_at_peak_us": {r: v[3] * 1e6 for r, v in roofs.items()},
             "fracs": {r: v[0] / v[1] for r, v in roofs.items()},
-            "alu_peak_note": f"{SFU_PER_CLK_PER_SM} MUFU results (ex2, lg2, sin, cos) per clock "
+            "alu_peak_note": f"{SFU_PER_CLK_PER_SM} MUFU results (ex2, lg2, rcp, sin, cos) per clock "
                              f"per SM x {sms} SMs x {peaks.get('sm_max_mhz', 2070.0):.0f} MHz",
             "kernel_ms": kernel_ms}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        nseq = w.B * w.H  # the whole batch: ~10 s of one core
+        nseq = w.B * w.H // (4 if train else 1)  # ~10 s of one core
         t = oracle_awd_sample(w, nseq, args.prefactor)
         cpu = {"value": nseq * w.N / w.H / t, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                "sample": f"{nseq} of {w.B * w.H} sequences of N={w.N} (fp64 C oracle, one "
@@ -815,7 +842,8 @@ def run_awd(args, w):
 
     if rank == 0:
         line = {
-            "metric": METRIC_AWD, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "metric": METRIC_AWD_TRAIN if train else METRIC_AWD, "value": value,
+            "unit": "tokens/s", "n_gpus": world,
             "steps": K, "warmup": args.warmup, "ms_per_step": kernel_ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": w.dtype, "data": "synthetic",

@@ -177,6 +177,34 @@ int flex_awd_loss(const flex_shape* shape, const void* q, const void* k, const f
                   const float* W2, const float* tau, int causal, float* loss, void* ws,
                   size_t ws_bytes, void* stream);
 
+/* Workspace bytes needed by flex_awd_loss_bwd for this shape; 0 if the shape is invalid
+ * or unsupported. */
+size_t flex_awd_bwd_workspace_bytes(const flex_shape* shape);
+
+/* One distillation step's loss and gradient.  The distillation trains only the kernel's
+ * parameters (appendix "Attention Distillation Setting": the Transformer is frozen), so
+ * the gradient of sum_{b,h} dloss[b][h] loss[b][h] (loss as in flex_awd_loss) is taken
+ * with respect to W1, W2 and tau, not q and k.  An entry with R_ij <= 0 is constant
+ * (log 1e-6) and has no gradient; on an entry with R_ij > 0,
+ *   d loss / d A~_ij = -(1/N) (P_ij / A~_ij - c_i / D_i),
+ * c_i the teacher mass on row i's entries with R_ij > 0 and D_i the row sum.  Near
+ * A~_ij = 0 the first term has a pole, so where some estimates are negative the gradient
+ * is ill-conditioned; the computation is meant for inputs whose weights are positive.
+ * q, k: [B][H][N][d] bf16 (d = 64, M in {64, 128}); dloss: [B][H] fp32 (device);
+ * loss: NULL or [B][H] fp32, overwritten; dW1, dW2: [H][M][d] fp32, overwritten (dW2 given
+ * exactly when W2 is); dtau: [H] fp32, overwritten (given exactly when tau is).
+ * ws: workspace of flex_awd_bwd_workspace_bytes() bytes.  Launches 6 kernels (5 without
+ * loss, one more with tau): the feature passes, the loss kernel (which also records each
+ * row's softmax normaliser, row-sum sign and c_i / D_i), its reduction, one gradient kernel
+ * (a query side and a key side, blockwise on the tensor cores; the chain rule through the
+ * feature map runs in the same kernel) and a fixed-order reduction, so the result does not
+ * depend on scheduling.  Errors as for flex_awd_loss, and FLEX_EINVAL when dW2 or dtau is
+ * given without W2 or tau (or missing with it). */
+int flex_awd_loss_bwd(const flex_shape* shape, const void* q, const void* k, const float* W1,
+                      const float* W2, const float* tau, int causal, const float* dloss,
+                      float* loss, float* dW1, float* dW2, float* dtau, void* ws,
+                      size_t ws_bytes, void* stream);
+
 /* Cumulative number of kernels this library has enqueued in this process (all entry
  * points, all devices).  Lets a caller count the launches inside a timed region. */
 unsigned long long flex_kernel_launches(void);

@@ -199,11 +199,12 @@ int flex_linattn_decode(const flex_shape* shape, const void* q, const void* k, c
 }
 
 // Distillation-loss workspace: header, phi(q), phi~(k) [B*H*N][2M] bf16, key weights
-// [B*H*N] fp32, partial sums [B*H][query blocks] fp32.
+// [B*H*N] fp32, partial sums [B*H][query blocks] fp32; for the gradient also the row
+// statistics [B*H*N] float4, the dW slots and the dtau partials [2*B*H] fp32.
 struct AwdWs {
-    size_t pq, pk, kw, part, total;
+    size_t pq, pk, kw, part, rowstat, slots, dtau_part, total;
 };
-AwdWs awd_ws(const Problem& p)
+AwdWs awd_ws(const Problem& p, bool grad)
 {
     const size_t rows = (size_t)p.B * p.H * p.N, feat = flex::align_up(rows * 2 * p.M * 2, 256);
     AwdWs w;
@@ -211,7 +212,10 @@ AwdWs awd_ws(const Problem& p)
     w.pk = w.pq + feat;
     w.kw = w.pk + feat;
     w.part = w.kw + flex::align_up(rows * sizeof(float), 256);
-    w.total = w.part + flex::align_up(flex::tc_awd_part_floats(p) * sizeof(float), 256);
+    w.rowstat = w.part + flex::align_up(flex::tc_awd_part_floats(p) * sizeof(float), 256);
+    w.slots = w.rowstat + (grad ? flex::align_up(rows * 16, 256) : 0);
+    w.dtau_part = w.slots + (grad ? flex::align_up(flex::tc_awd_slot_floats(p) * 4, 256) : 0);
+    w.total = w.dtau_part + (grad ? flex::align_up((size_t)2 * p.B * p.H * 4, 256) : 0);
     return w;
 }
 
@@ -219,7 +223,7 @@ size_t flex_awd_workspace_bytes(const flex_shape* shape)
 {
     Problem p;
     if (make_problem(shape, nullptr, 0, &p) != FLEX_OK || !flex::tc_awd_supported(p)) return 0;
-    return awd_ws(p).total;
+    return awd_ws(p, false).total;
 }
 
 int flex_awd_loss(const flex_shape* shape, const void* q, const void* k, const float* W1,
@@ -234,7 +238,7 @@ int flex_awd_loss(const flex_shape* shape, const void* q, const void* k, const f
         if (!aligned(t, 16)) return FLEX_EINVAL;
     if ((W2 && !aligned(W2, 16)) || (tau && !aligned(tau, 4))) return FLEX_EINVAL;
     if (!flex::tc_awd_supported(p)) return FLEX_EUNSUPPORTED;
-    const AwdWs w = awd_ws(p);
+    const AwdWs w = awd_ws(p, false);
     if ((rc = check_ws(ws, ws_bytes, w.total))) return rc;
     cudaStream_t s = (cudaStream_t)stream;
     char* base = (char*)ws;
@@ -247,6 +251,48 @@ int flex_awd_loss(const flex_shape* shape, const void* q, const void* k, const f
         return rc;
     return count(2, flex::launch_tc_awd(p, q, k, base + w.pq, base + w.pk, (float*)(base + w.part),
                                         loss, status, s));
+}
+
+size_t flex_awd_bwd_workspace_bytes(const flex_shape* shape)
+{
+    Problem p;
+    if (make_problem(shape, nullptr, 0, &p) != FLEX_OK || !flex::tc_awd_supported(p)) return 0;
+    return awd_ws(p, true).total;
+}
+
+int flex_awd_loss_bwd(const flex_shape* shape, const void* q, const void* k, const float* W1,
+                      const float* W2, const float* tau, int causal, const float* dloss,
+                      float* loss, float* dW1, float* dW2, float* dtau, void* ws,
+                      size_t ws_bytes, void* stream)
+{
+    Problem p;
+    int rc = make_problem(shape, W2, causal, &p);
+    if (rc) return rc;
+    if (!q || !k || !W1 || !dloss || !dW1) return FLEX_EINVAL;
+    if ((W2 != nullptr) != (dW2 != nullptr) || (tau != nullptr) != (dtau != nullptr))
+        return FLEX_EINVAL;
+    for (const void* t : {q, k, (const void*)W1, (const void*)dW1})
+        if (!aligned(t, 16)) return FLEX_EINVAL;
+    if ((W2 && (!aligned(W2, 16) || !aligned(dW2, 16))) || (tau && !aligned(tau, 4)) ||
+        (loss && !aligned(loss, 4)) || !aligned(dloss, 4) || (dtau && !aligned(dtau, 4)))
+        return FLEX_EINVAL;
+    if (!flex::tc_awd_supported(p)) return FLEX_EUNSUPPORTED;
+    const AwdWs w = awd_ws(p, true);
+    if ((rc = check_ws(ws, ws_bytes, w.total))) return rc;
+    cudaStream_t s = (cudaStream_t)stream;
+    char* base = (char*)ws;
+    float* kw = tau ? (float*)(base + w.kw) : nullptr;
+    if (tau && (rc = count(1, flex::launch_key_weights(p, k, tau, kw, s)))) return rc;
+    int* status = &((flex::WsHeader*)ws)->status;
+    if ((rc = count(1, flex::launch_tc_featmap(p, q, W1, W2, nullptr, base + w.pq, status, s))))
+        return rc;
+    if ((rc = count(1, flex::launch_tc_featmap(p, k, W1, W2, kw, base + w.pk, status, s))))
+        return rc;
+    return count(loss ? 4 : 3,
+                 flex::launch_tc_awd_bwd(p, q, k, base + w.pq, base + w.pk, W1, W2, kw, tau, dloss,
+                                         (float*)(base + w.part), loss,
+                                         (float4*)(base + w.rowstat), (float*)(base + w.slots),
+                                         (float*)(base + w.dtau_part), dW1, dW2, dtau, status, s));
 }
 
 unsigned long long flex_kernel_launches(void) { return g_launches.load(); }

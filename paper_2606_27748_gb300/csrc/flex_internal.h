@@ -98,5 +98,15 @@ size_t tc_awd_part_floats(const Problem& p);  // partial slots [B*H][query block
 // pq, pk: phi(q) and the key-weighted phi(k), [B*H][N][2M] bf16; loss [B*H] fp32
 cudaError_t launch_tc_awd(const Problem& p, const void* q, const void* k, const void* pq,
                           const void* pk, float* part, float* loss, int* status, cudaStream_t s);
+// Loss (loss may be NULL) and its gradient with respect to W1, W2, tau, weighted by dloss
+// [B*H]: the loss kernel writes per-row statistics rowstat [B*H*N], then the gradient
+// kernel fills slots [tc_awd_slot_floats] and dtau_part [2*B*H], reduced into dW1, dW2,
+// dtau.  kw: key weights (with tau) or NULL.
+size_t tc_awd_slot_floats(const Problem& p);
+cudaError_t launch_tc_awd_bwd(const Problem& p, const void* q, const void* k, const void* pq,
+                              const void* pk, const float* W1, const float* W2, const float* kw,
+                              const float* tau, const float* dloss, float* part, float* loss,
+                              float4* rowstat, float* slots, float* dtau_part, float* dW1,
+                              float* dW2, float* dtau, int* status, cudaStream_t s);
 
 }  // namespace flex

@@ -19,7 +19,8 @@
 // and D = sum A.  At the end the two halves merge and, by the sign of D,
 //   L_i = -(ln2 T_sign - Z_sign ln|D| + (Z - Z_sign) ln 1e-6) / Z,
 // which is the definition with the reading above applied.  Block sums of L_i go to
-// partial slots, summed per sequence in a fixed order.  Every wait is bounded.
+// partial slots, summed per sequence in a fixed order.  Every wait is bounded.  For the
+// gradient the same kernel also writes each row's statistics (below).
 #include <algorithm>
 
 #include "flex_internal.h"
@@ -64,7 +65,8 @@ __global__ void __launch_bounds__(kThreadsA, 1)
                   const __grid_constant__ CUtensorMap tmap_k,
                   const __grid_constant__ CUtensorMap tmap_pq,
                   const __grid_constant__ CUtensorMap tmap_pk, int N, int causal,
-                  float score_scale, int nqb, float* __restrict__ part, int* status)
+                  float score_scale, int nqb, float* __restrict__ part,
+                  float4* __restrict__ rowstat, int* status)
 {
     using L = AwdCfg<G2>;
     extern __shared__ uint8_t smem_raw[];
@@ -238,6 +240,12 @@ __global__ void __launch_bounds__(kThreadsA, 1)
             else
                 li = -kLnEps;
             lsum = li;
+            if (rowstat) {  // what the gradient needs of this row (see the gradient kernel)
+                const float sg = den > 0.f ? 1.f : (den < 0.f ? -1.f : 0.f);
+                const float zs = den > 0.f ? zp : zn;
+                const float e = sg != 0.f ? (zs / z) / den : 0.f;
+                rowstat[(size_t)bh * N + row] = make_float4(m + log2f(z), sg, e, 0.f);
+            }
         }
     }
     // block sum in a fixed order
@@ -265,9 +273,356 @@ __global__ void awd_reduce_kernel(int BH, int nqb, int N, const float* __restric
     }
 }
 
+// ---- gradient with respect to the kernel's parameters ------------------------------------
+//
+// The distillation trains only the feature map, so the gradient is taken with respect to
+// W1, W2 and tau.  With the row statistics of the loss kernel (l_i = log2 of the softmax
+// normaliser in the scaled base-2 scores, the sign of D_i, e_i = c_i / D_i where c_i is the
+// teacher mass on the entries with R_ij > 0) and sigma = -dloss / N:
+//   dL/dA~_ij = sigma G_ij,   G_ij = [A~_ij sign(D_i) > 0] P_ij / A~_ij - e_i   (j in row i)
+//   dphi(q_i) = sigma sum_j G_ij phi~(k_j),   dphi~(k_j) = sigma sum_i G_ij phi(q_i).
+// One CTA per (sequence, side): the query side holds a block of 128 queries and streams
+// the key blocks, the key side holds 128 keys and streams the query blocks.  Per streamed
+// block thread 0 issues S = X_own X_other^T and A = Phi_own Phi_other^T into tensor memory;
+// each thread turns half of its row into G (two SFU operations per entry: ex2, divide),
+// writes it as bf16 in place over A, and G Phi_other (A operand in tensor memory, features
+// MN-major) accumulates into T_D.  Then, per group of 64 frequencies, the chain rule through
+// the feature map runs on the tensor cores: the projection X_own W'^T is recomputed, the
+// epilogue forms da (du | dw for Flexformer_n) from T_D, and dW' += da^T X_own.  The rows
+// of dW' are added into this CTA's slot (fixed order); a reduction sums the slots over the
+// batch and both sides in a fixed order.  On the key side, with the prefactor, the chain
+// rule takes dphi(k_j) = w_j dphi~(k_j) and dtau gains -(phi~(k_j) . dphi~(k_j)) |k_j|^2
+// exp(-tau).  Every wait is bounded.
+template <int G2>
+struct AwdBwCfg {
+    static constexpr uint32_t XO = 0, XT = 16384, PO = 32768, PT = PO + G2 * 16384;
+    static constexpr uint32_t BYTES = PT + G2 * 16384;
+    static constexpr uint32_t WG = XT;  // after the streamed blocks: one group's W' rows
+    static constexpr uint32_t DA = PT;  // and the da tiles [du | dw]
+    static constexpr uint32_t T_S = 0, T_A = 128, T_D = 256;
+    static_assert(G2 >= 2 && BYTES + 1024 <= 232448, "shared memory budget");
+};
+
+template <int G2, bool NS, bool KW>
+__global__ void __launch_bounds__(kThreadsA, 1)
+    tc_awd_bwd_kernel(const __grid_constant__ CUtensorMap tmap_q,
+                      const __grid_constant__ CUtensorMap tmap_k,
+                      const __grid_constant__ CUtensorMap tmap_pq,
+                      const __grid_constant__ CUtensorMap tmap_pk, int BH, int H, int N, int M,
+                      int causal, float score_scale, const float4* __restrict__ rowstat,
+                      const float* __restrict__ dloss, const float* __restrict__ W1,
+                      const float* __restrict__ W2, const float* __restrict__ kw,
+                      const float* __restrict__ tau, float* __restrict__ slots,
+                      float* __restrict__ dtau_part, int* status)
+{
+    using L = AwdBwCfg<G2>;
+    constexpr int P = NS ? 128 : 64;  // projection rows per group of 64 frequencies
+    constexpr int G = G2 / 2;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const uint32_t sb = smem_u32(sm);
+    __shared__ uint32_t tmem_base_sh;
+    __shared__ __align__(8) uint64_t mbar, tma_bar;
+    __shared__ volatile int abort_flag;
+    __shared__ float4 ostat[kC];  // key side: statistics of the streamed query rows
+    __shared__ float wsum[kThreadsA / 32];
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int wg = warp >> 2, quad = warp & 3, t = 32 * quad + lane;
+    const bool kside = (int)blockIdx.x >= BH;
+    const int bh = (int)blockIdx.x % BH, h = bh % H;
+    const CUtensorMap* x_own = kside ? &tmap_k : &tmap_q;
+    const CUtensorMap* x_oth = kside ? &tmap_q : &tmap_k;
+    const CUtensorMap* f_own = kside ? &tmap_pk : &tmap_pq;
+    const CUtensorMap* f_oth = kside ? &tmap_pq : &tmap_pk;
+    const int nblk = (N + kC - 1) / kC;
+    const float sigma = -dloss[bh] / (float)N;
+    const float itau = KW ? expf(-tau[h]) : 0.f;
+    const float cM = rsqrtf((float)M);
+    float dtau_acc = 0.f;
+
+    if (tid == 0) {
+        mbar_init(&mbar, 1);
+        mbar_init(&tma_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(&tmem_base_sh, 512);
+        tmem_relinquish();
+    }
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    const uint32_t tm = tmem_base_sh;
+    const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
+    uint32_t phase = 0, tma_phase = 0;
+    auto adv = [](uint64_t dsc, uint32_t bytes) { return dsc + (bytes >> 4); };
+    const uint64_t dXO = sdesc(sb + L::XO, 16, 1024), dXT = sdesc(sb + L::XT, 16, 1024);
+    const uint64_t dPO = sdesc(sb + L::PO, 16, 1024), dPT = sdesc(sb + L::PT, 16, 1024);
+    const uint64_t dPTmn = sdesc(sb + L::PT, 16384, 1024);
+    const uint64_t dWg = sdesc(sb + L::WG, 16, 1024);
+    const uint64_t dDAmn = sdesc(sb + L::DA, 16384, 1024), dXOmn = sdesc(sb + L::XO, 16384, 1024);
+    constexpr uint32_t I_KK128 = idesc_bf16(128, 128, 0, 0);
+    constexpr uint32_t I_DPHI = idesc_bf16(128, 64 * G2, 0, 1);  // N = 2M features
+    constexpr uint32_t I_PROJ = idesc_bf16(128, P, 0, 0);
+    constexpr uint32_t I_DW = idesc_bf16(128, 64, 1, 1);
+
+    auto handoff = [&]() {
+        fence_proxy_async();
+        fence_before_sync();
+        __syncthreads();
+    };
+    auto commit_wait = [&]() -> bool {  // thread 0 has issued MMAs: commit, all wait
+        if (tid == 0) mma_commit(&mbar);
+        bool ok_ = bar_wait(&mbar, phase, &abort_flag, status);
+        phase ^= 1;
+        ok_ = !__syncthreads_or(!ok_);
+        fence_after_sync();
+        return ok_;
+    };
+    // the streamed block ot (and first the held block ob): one arrival per phase
+    auto load = [&](int ob, int ot, bool own_too) {
+        mbar_arrive_expect_tx(&tma_bar, (1 + G2) * kTileBytes * (own_too ? 2 : 1));
+        if (own_too) {
+            tma_load_3d(sb + L::XO, x_own, 0, ob * kC, bh, &tma_bar);
+            for (int g = 0; g < G2; ++g)
+                tma_load_3d(sb + L::PO + g * 16384, f_own, 64 * g, ob * kC, bh, &tma_bar);
+        }
+        tma_load_3d(sb + L::XT, x_oth, 0, ot * kC, bh, &tma_bar);
+        for (int g = 0; g < G2; ++g)
+            tma_load_3d(sb + L::PT + g * 16384, f_oth, 64 * g, ot * kC, bh, &tma_bar);
+    };
+    // streamed blocks of held block ob: causal queries see keys j <= i
+    auto first_other = [&](int ob) { return (kside && causal) ? ob : 0; };
+    auto last_other = [&](int ob) { return (!kside && causal) ? ob : nblk - 1; };
+
+    bool ok = true;
+    if (tid == 0) load(0, first_other(0), true);
+    for (int ob = 0; ob < nblk && ok; ++ob) {
+        const int own_row = ob * kC + t;
+        const bool own_valid = own_row < N;
+        float4 qs = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (!kside && own_valid) qs = rowstat[(size_t)bh * N + own_row];
+        const int o0 = first_other(ob), o1 = last_other(ob);
+        for (int ot = o0; ot <= o1; ++ot) {
+            if (kside && tid < kC) {
+                const int r = ot * kC + tid;
+                ostat[tid] = r < N ? rowstat[(size_t)bh * N + r] : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            ok = bar_wait(&tma_bar, tma_phase, &abort_flag, status);
+            tma_phase ^= 1;
+            ok = !__syncthreads_or(!ok);
+            if (!ok) break;
+            fence_after_sync();
+            if (tid == 0) {
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_bf16(tm + L::T_S, adv(dXO, ks * 32), adv(dXT, ks * 32), I_KK128, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 4 * G2; ++ks) {
+                    const uint32_t kofs = (ks >> 2) * 16384 + (ks & 3) * 32;
+                    mma_bf16(tm + L::T_A, adv(dPO, kofs), adv(dPT, kofs), I_KK128, ks > 0);
+                }
+            }
+            if (!(ok = commit_wait())) break;
+            // G over this thread's 64 columns, two rounds of 32, bf16 in place over A
+#pragma unroll
+            for (int b = 0; b < 2; ++b) {
+                const uint32_t col = 64 * wg + 32 * b;
+                float sv[32], av[32];
+                tmem_ld16(tm_row + L::T_S + col, *reinterpret_cast<float(*)[16]>(&sv[0]));
+                tmem_ld16(tm_row + L::T_S + col + 16, *reinterpret_cast<float(*)[16]>(&sv[16]));
+                tmem_ld16(tm_row + L::T_A + col, *reinterpret_cast<float(*)[16]>(&av[0]));
+                tmem_ld16(tm_row + L::T_A + col + 16, *reinterpret_cast<float(*)[16]>(&av[16]));
+                tmem_wait_ld();
+                uint32_t pk[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    float gv[2];
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        const int c = (int)col + 2 * i + e, orow = ot * kC + c;
+                        const int qi = kside ? orow : own_row, kj = kside ? own_row : orow;
+                        const bool in = own_valid && orow < N && (!causal || kj <= qi);
+                        const float4 st = kside ? ostat[c] : qs;
+                        const float a = av[2 * i + e];
+                        const float p = ex2f(fmaf(sv[2 * i + e], score_scale, -st.x));
+                        const float first = a * st.y > 0.f ? __fdividef(p, a) : 0.f;
+                        gv[e] = in ? first - st.z : 0.f;
+                    }
+                    pk[i] = pack_bf16(gv[0], gv[1]);
+                }
+                tmem_st16(tm_row + L::T_A + 64 * wg + 16 * b, pk);
+            }
+            tmem_wait_st();
+            handoff();
+            if (tid == 0) {
+                fence_after_sync();
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_bf16_tmem_a(tm + L::T_D, tm + L::T_A + 64 * (ks >> 2) + 8 * (ks & 3),
+                                    adv(dPTmn, ks * 2048), I_DPHI, (ot > o0 || ks > 0) ? 1u : 0u);
+            }
+            if (!(ok = commit_wait())) break;
+            if (tid == 0 && ot < o1) load(ob, ot + 1, false);
+        }
+        if (!ok) break;
+
+        // chain rule through the feature map, one group of 64 frequencies at a time
+        const float wk = (KW && kside && own_valid) ? kw[(size_t)bh * N + own_row] : 1.f;
+        const float scl = sigma * wk;  // dphi(x) = scl T_D (key side: dphi = w dphi~)
+        float sdot = 0.f;              // key side: phi(k) . T_D over this thread's features
+        float kk = 0.f;                // key side: |k_j|^2 from the held tile (read before
+        if (KW && kside) {             // the group loop: the next block's load reuses it)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const uint4 k4 = *reinterpret_cast<const uint4*>(sm + L::XO + swz128(t, 8 * j));
+                const uint32_t kw4[4] = {k4.x, k4.y, k4.z, k4.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float k0 = __uint_as_float(kw4[e] << 16);
+                    const float k1 = __uint_as_float(kw4[e] & 0xFFFF0000u);
+                    kk = fmaf(k0, k0, fmaf(k1, k1, kk));
+                }
+            }
+        }
+        for (int g = 0; g < G && ok; ++g) {
+            stage_freq_rows<NS, 1, kThreadsA>(sb + L::WG, W1, W2, h, M, tid, 64 * g);
+            handoff();
+            if (tid == 0) {
+                fence_after_sync();
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_bf16(tm + L::T_S, adv(dXO, ks * 32), adv(dWg, ks * 32), I_PROJ, ks > 0);
+            }
+            if (!(ok = commit_wait())) break;
+            float dc[32], ds[32], u[32], w[32];
+            tmem_ld16(tm_row + L::T_D + 64 * g + 32 * wg, *reinterpret_cast<float(*)[16]>(&dc[0]));
+            tmem_ld16(tm_row + L::T_D + 64 * g + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&dc[16]));
+            tmem_ld16(tm_row + L::T_D + M + 64 * g + 32 * wg, *reinterpret_cast<float(*)[16]>(&ds[0]));
+            tmem_ld16(tm_row + L::T_D + M + 64 * g + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&ds[16]));
+            tmem_ld16(tm_row + L::T_S + 32 * wg, *reinterpret_cast<float(*)[16]>(&u[0]));
+            tmem_ld16(tm_row + L::T_S + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&u[16]));
+            if (NS) {
+                tmem_ld16(tm_row + L::T_S + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]));
+                tmem_ld16(tm_row + L::T_S + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
+            }
+            tmem_wait_ld();
+            uint32_t o1[16], o2[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                float r1[2], r2[2];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int f = 2 * i + e;
+                    float su, cu;
+                    __sincosf(u[f], &su, &cu);
+                    float cw = 1.f, sw = 0.f;
+                    if (NS) __sincosf(w[f], &sw, &cw);
+                    const float dpc = scl * dc[f], dps = scl * ds[f];
+                    r1[e] = cM * cw * (-su * dpc + cu * dps);
+                    r2[e] = NS ? -cM * sw * (cu * dpc + su * dps) : 0.f;
+                    if (KW) sdot = fmaf(cu * cw, dc[f], fmaf(su * cw, ds[f], sdot));
+                    if (!own_valid) r1[e] = r2[e] = 0.f;
+                }
+                o1[i] = pack_bf16(r1[0], r1[1]);
+                o2[i] = pack_bf16(r2[0], r2[1]);
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const uint32_t off = swz128(t, (4 * wg + j) * 8);
+                st_shared_v4(sb + L::DA + off, o1[4 * j], o1[4 * j + 1], o1[4 * j + 2], o1[4 * j + 3]);
+                st_shared_v4(sb + L::DA + 16384 + off, o2[4 * j], o2[4 * j + 1], o2[4 * j + 2],
+                             o2[4 * j + 3]);
+            }
+            handoff();
+            if (tid == 0) {
+                fence_after_sync();
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_bf16(tm + L::T_A, adv(dDAmn, ks * 2048), adv(dXOmn, ks * 2048), I_DW, ks > 0);
+            }
+            if (!(ok = commit_wait())) break;
+            // rows of dW' (lane = projection row) added into this CTA's slot
+            float v[32];
+            tmem_ld16(tm_row + L::T_A + 32 * wg, *reinterpret_cast<float(*)[16]>(&v[0]));
+            tmem_ld16(tm_row + L::T_A + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&v[16]));
+            tmem_wait_ld();
+            float4* dst = reinterpret_cast<float4*>(
+                slots + (((size_t)blockIdx.x * G + g) * 128 + t) * 64 + 32 * wg);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const float4 old = ob == 0 ? make_float4(0.f, 0.f, 0.f, 0.f) : dst[j];
+                dst[j] = make_float4(old.x + v[4 * j], old.y + v[4 * j + 1], old.z + v[4 * j + 2],
+                                     old.w + v[4 * j + 3]);
+            }
+            // tensor memory, the W' rows and the da tiles are free once every thread is here
+            fence_before_sync();
+            __syncthreads();
+        }
+        if (!ok) break;
+        if (KW && kside && own_valid)  // s_j = phi~(k_j) . dphi~(k_j) = w cM sigma sdot
+            dtau_acc -= wk * cM * sigma * sdot * kk * itau;
+        if (tid == 0 && ob + 1 < nblk) load(ob + 1, first_other(ob + 1), true);
+    }
+
+    // dtau partial of this CTA, summed in a fixed order
+    float dsum = dtau_acc;
+    for (int o = 16; o > 0; o >>= 1) dsum += __shfl_xor_sync(0xffffffffu, dsum, o);
+    if (lane == 0) wsum[warp] = dsum;
+    __syncthreads();
+    if (tid == 0) {
+        float tot = 0.f;
+        for (int w8 = 0; w8 < kThreadsA / 32; ++w8) tot += wsum[w8];
+        dtau_part[blockIdx.x] = tot;
+    }
+    fence_before_sync();
+    __syncthreads();
+    fence_after_sync();
+    if (warp == 0) tmem_dealloc(tm, 512);
+}
+
+// dW1, dW2 [H][M][64] and dtau [H] from the slots [2 sides][B*H][G][128 rows][64]: sum over
+// the sides and the batch in a fixed order; Flexformer_n rows 0-63 of a group are dU, rows
+// 64-127 dV (U = (W1+W2)/2, V = (W1-W2)/2), so dW1 = (dU+dV)/2, dW2 = (dU-dV)/2.
+__global__ void awd_dw_reduce_kernel(int B, int H, int M, int nonstat,
+                                     const float* __restrict__ slots,
+                                     const float* __restrict__ dtau_part, float* __restrict__ dW1,
+                                     float* __restrict__ dW2, float* __restrict__ dtau)
+{
+    const int BH = B * H, G = M / 64;
+    const size_t total = (size_t)H * M * 64;
+    for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
+         idx += (size_t)gridDim.x * blockDim.x) {
+        const int c = (int)(idx % 64), f = (int)((idx / 64) % M), h = (int)(idx / ((size_t)64 * M));
+        const int g = f / 64, r = f % 64;
+        float su = 0.f, sv = 0.f;
+        for (int side = 0; side < 2; ++side)
+            for (int b = 0; b < B; ++b) {
+                const float* sl = slots + (((size_t)(side * BH + b * H + h) * G + g) * 128) * 64;
+                su += sl[r * 64 + c];
+                if (nonstat) sv += sl[(64 + r) * 64 + c];
+            }
+        if (nonstat) {
+            dW1[idx] = 0.5f * (su + sv);
+            dW2[idx] = 0.5f * (su - sv);
+        } else {
+            dW1[idx] = su;
+        }
+    }
+    if (dtau && blockIdx.x == 0)
+        for (int h = threadIdx.x; h < H; h += blockDim.x) {
+            float sd = 0.f;
+            for (int b = 0; b < B; ++b) sd += dtau_part[BH + b * H + h];  // key side
+            dtau[h] = sd;
+        }
+}
+
 template <int G2>
 cudaError_t launch_typed(const Problem& p, const void* q, const void* k, const void* pq,
-                         const void* pk, float* part, float* loss, int* status, cudaStream_t s)
+                         const void* pk, float* part, float* loss, float4* rowstat, int* status,
+                         cudaStream_t s)
 {
     const int BH = p.B * p.H, nqb = (p.N + kC - 1) / kC;
     CUtensorMap mq, mk, mpq, mpk;
@@ -280,10 +635,61 @@ cudaError_t launch_typed(const Problem& p, const void* q, const void* k, const v
     if (e != cudaSuccess) return e;
     const float score_scale = 1.4426950408889634f / sqrtf((float)p.d);  // log2(e) / sqrt(d)
     kern<<<BH * nqb, kThreadsA, smem, s>>>(mq, mk, mpq, mpk, p.N, p.causal, score_scale, nqb,
-                                           part, status);
+                                           part, rowstat, status);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (!loss) return cudaSuccess;
     awd_reduce_kernel<<<(BH + 255) / 256, 256, 0, s>>>(BH, nqb, p.N, part, loss);
     return cudaGetLastError();
+}
+
+template <int G2, bool NS, bool KW>
+cudaError_t launch_bwd_typed(const Problem& p, const void* q, const void* k, const void* pq,
+                             const void* pk, const float* W1, const float* W2, const float* kw,
+                             const float* tau, const float* dloss, const float4* rowstat,
+                             float* slots, float* dtau_part, float* dW1, float* dW2, float* dtau,
+                             int* status, cudaStream_t s)
+{
+    const int BH = p.B * p.H;
+    CUtensorMap mq, mk, mpq, mpk;
+    if (!make_act_map(&mq, q, BH, p.N) || !make_act_map(&mk, k, BH, p.N) ||
+        !make_feat_map(&mpq, pq, BH, p.N, 2 * p.M) || !make_feat_map(&mpk, pk, BH, p.N, 2 * p.M))
+        return cudaErrorInvalidValue;
+    const int smem = (int)AwdBwCfg<G2>::BYTES + 1024;
+    auto kern = tc_awd_bwd_kernel<G2, NS, KW>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    const float score_scale = 1.4426950408889634f / sqrtf((float)p.d);
+    kern<<<2 * BH, kThreadsA, smem, s>>>(mq, mk, mpq, mpk, BH, p.H, p.N, p.M, p.causal,
+                                         score_scale, rowstat, dloss, W1, W2, kw, tau, slots,
+                                         dtau_part, status);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const size_t total = (size_t)p.H * p.M * 64;
+    const int grid = (int)std::min<size_t>((total + 255) / 256, 152 * 8);
+    awd_dw_reduce_kernel<<<grid, 256, 0, s>>>(p.B, p.H, p.M, p.nonstat, slots, dtau_part, dW1,
+                                              dW2, tau ? dtau : nullptr);
+    return cudaGetLastError();
+}
+
+template <int G2>
+cudaError_t launch_bwd_g2(const Problem& p, const void* q, const void* k, const void* pq,
+                          const void* pk, const float* W1, const float* W2, const float* kw,
+                          const float* tau, const float* dloss, const float4* rowstat,
+                          float* slots, float* dtau_part, float* dW1, float* dW2, float* dtau,
+                          int* status, cudaStream_t s)
+{
+    if (p.nonstat)
+        return tau ? launch_bwd_typed<G2, true, true>(p, q, k, pq, pk, W1, W2, kw, tau, dloss,
+                                                      rowstat, slots, dtau_part, dW1, dW2, dtau,
+                                                      status, s)
+                   : launch_bwd_typed<G2, true, false>(p, q, k, pq, pk, W1, W2, kw, tau, dloss,
+                                                       rowstat, slots, dtau_part, dW1, dW2, dtau,
+                                                       status, s);
+    return tau ? launch_bwd_typed<G2, false, true>(p, q, k, pq, pk, W1, W2, kw, tau, dloss,
+                                                   rowstat, slots, dtau_part, dW1, dW2, dtau,
+                                                   status, s)
+               : launch_bwd_typed<G2, false, false>(p, q, k, pq, pk, W1, W2, kw, tau, dloss,
+                                                    rowstat, slots, dtau_part, dW1, dW2, dtau,
+                                                    status, s);
 }
 
 }  // namespace
@@ -298,11 +704,31 @@ size_t tc_awd_part_floats(const Problem& p)
     return (size_t)p.B * p.H * ((p.N + kC - 1) / kC);
 }
 
+size_t tc_awd_slot_floats(const Problem& p)
+{
+    return (size_t)2 * p.B * p.H * (p.M / 64) * 128 * 64;
+}
+
 cudaError_t launch_tc_awd(const Problem& p, const void* q, const void* k, const void* pq,
                           const void* pk, float* part, float* loss, int* status, cudaStream_t s)
 {
-    return p.M == 64 ? launch_typed<2>(p, q, k, pq, pk, part, loss, status, s)
-                     : launch_typed<4>(p, q, k, pq, pk, part, loss, status, s);
+    return p.M == 64 ? launch_typed<2>(p, q, k, pq, pk, part, loss, nullptr, status, s)
+                     : launch_typed<4>(p, q, k, pq, pk, part, loss, nullptr, status, s);
+}
+
+cudaError_t launch_tc_awd_bwd(const Problem& p, const void* q, const void* k, const void* pq,
+                              const void* pk, const float* W1, const float* W2, const float* kw,
+                              const float* tau, const float* dloss, float* part, float* loss,
+                              float4* rowstat, float* slots, float* dtau_part, float* dW1,
+                              float* dW2, float* dtau, int* status, cudaStream_t s)
+{
+    cudaError_t e = p.M == 64 ? launch_typed<2>(p, q, k, pq, pk, part, loss, rowstat, status, s)
+                              : launch_typed<4>(p, q, k, pq, pk, part, loss, rowstat, status, s);
+    if (e != cudaSuccess) return e;
+    return p.M == 64 ? launch_bwd_g2<2>(p, q, k, pq, pk, W1, W2, kw, tau, dloss, rowstat, slots,
+                                        dtau_part, dW1, dW2, dtau, status, s)
+                     : launch_bwd_g2<4>(p, q, k, pq, pk, W1, W2, kw, tau, dloss, rowstat, slots,
+                                        dtau_part, dW1, dW2, dtau, status, s);
 }
 
 }  // namespace flex

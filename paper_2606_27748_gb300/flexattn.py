@@ -22,8 +22,8 @@ FLEX_OK, FLEX_EINVAL, FLEX_EUNSUPPORTED, FLEX_EWORKSPACE, FLEX_ECUDA, FLEX_ETIME
 
 EXPORTS = ("flex_strerror", "flex_workspace_bytes", "flex_featmap", "flex_linattn_fwd",
            "flex_linattn_bwd", "flex_decode_workspace_bytes", "flex_linattn_decode",
-           "flex_awd_workspace_bytes", "flex_awd_loss", "flex_kernel_launches",
-           "flex_check_status")
+           "flex_awd_workspace_bytes", "flex_awd_loss", "flex_awd_bwd_workspace_bytes",
+           "flex_awd_loss_bwd", "flex_kernel_launches", "flex_check_status")
 
 
 class FlexShape(ctypes.Structure):
@@ -68,11 +68,16 @@ def load(path: str = LIBRARY) -> ctypes.CDLL:
         lib.flex_awd_workspace_bytes.argtypes = [shp]
         lib.flex_awd_workspace_bytes.restype = sz
         lib.flex_awd_loss.argtypes = [shp, vp, vp, vp, vp, vp, ip, vp, vp, sz, vp]
+        lib.flex_awd_bwd_workspace_bytes.argtypes = [shp]
+        lib.flex_awd_bwd_workspace_bytes.restype = sz
+        lib.flex_awd_loss_bwd.argtypes = [shp, vp, vp, vp, vp, vp, ip, vp, vp, vp, vp, vp, vp,
+                                          sz, vp]
         lib.flex_check_status.argtypes = [vp, vp]
         lib.flex_kernel_launches.argtypes = []
         lib.flex_kernel_launches.restype = ctypes.c_ulonglong
         for fn in (lib.flex_featmap, lib.flex_linattn_fwd, lib.flex_linattn_bwd,
-                   lib.flex_linattn_decode, lib.flex_awd_loss, lib.flex_check_status):
+                   lib.flex_linattn_decode, lib.flex_awd_loss, lib.flex_awd_loss_bwd,
+                   lib.flex_check_status):
             fn.restype = ip
         _lib = lib
         return lib
@@ -236,6 +241,43 @@ def awd_loss(q, k, W1, W2=None, causal=False, tau=None, loss=None, ws=None, stre
                                 _ptr(tau), int(bool(causal)), _ptr(loss), _ptr(ws),
                                 ws.numel(), _stream(stream)), "flex_awd_loss")
     return loss
+
+
+def awd_bwd_workspace(shape: FlexShape, device=None) -> torch.Tensor:
+    """A caller-owned workspace for flex_awd_loss_bwd."""
+    n = int(load().flex_awd_bwd_workspace_bytes(ctypes.byref(shape)))
+    if n == 0:
+        raise FlexError(FLEX_EUNSUPPORTED, "flex_awd_bwd_workspace_bytes")
+    return torch.zeros(n, dtype=torch.uint8, device=device or "cuda")
+
+
+def awd_loss_bwd(q, k, W1, W2=None, causal=False, tau=None, dloss=None, loss=None,
+                 dW1=None, dW2=None, dtau=None, ws=None, stream=None, want_loss=True):
+    """Distillation loss [B, H] (None unless want_loss) and its gradient with respect to the
+    kernel's parameters, weighted by dloss [B, H] (default ones): (loss, dW1, dW2, dtau);
+    dW2 is None without W2, dtau None without tau."""
+    shape = shape_of(q, W1)
+    dev = q.device
+    if dloss is None:
+        dloss = torch.ones(q.shape[:2], dtype=torch.float32, device=dev)
+    if want_loss and loss is None:
+        loss = torch.empty(q.shape[:2], dtype=torch.float32, device=dev)
+    if dW1 is None:
+        dW1 = torch.empty_like(W1)
+    if W2 is not None and dW2 is None:
+        dW2 = torch.empty_like(W2)
+    if tau is not None and dtau is None:
+        dtau = torch.empty_like(tau)
+    if ws is None:
+        ws = awd_bwd_workspace(shape, dev)
+    _check(load().flex_awd_loss_bwd(ctypes.byref(shape), _ptr(q), _ptr(k), _ptr(W1), _ptr(W2),
+                                    _ptr(tau), int(bool(causal)), _ptr(dloss),
+                                    _ptr(loss if want_loss else None), _ptr(dW1),
+                                    _ptr(dW2 if W2 is not None else None),
+                                    _ptr(dtau if tau is not None else None), _ptr(ws),
+                                    ws.numel(), _stream(stream)), "flex_awd_loss_bwd")
+    return (loss if want_loss else None), dW1, (dW2 if W2 is not None else None), (
+        dtau if tau is not None else None)
 
 
 def check_status(ws, stream=None):

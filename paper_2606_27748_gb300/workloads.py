@@ -80,6 +80,10 @@ WORKLOADS[DECODE.name] = DECODE
 AWD = Workload("n_awd_bf16_B32H8N512_d64M64", "n", False, "bf16", 32, 8, 512, 64, 64,
                64 ** -0.25, "normal", 7, awd=True)
 WORKLOADS[AWD.name] = AWD
+# One distillation training step on the same batch: the loss and its gradient with respect
+# to the kernel's parameters (W1, W2; tau with the prefactor).
+AWD_TRAIN = AWD.replace(name="n_awd_train_bf16_B32H8N512_d64M64", backward=True)
+WORKLOADS[AWD_TRAIN.name] = AWD_TRAIN
 
 
 def bf16_bits(x: np.ndarray) -> np.ndarray:

@@ -129,3 +129,30 @@ def test_awd_host_validation_without_gpu(lib):
                              None) == FLEX_EWORKSPACE
     assert lib.flex_awd_loss(ctypes.byref(ok), p, p, p, None, ctypes.c_void_p(4098), 0, p, p,
                              need, None) == FLEX_EINVAL
+
+
+def test_awd_bwd_host_validation_without_gpu(lib):
+    from paper_2606_27748_gb300.flexattn import (FlexShape, FLEX_EINVAL, FLEX_EUNSUPPORTED,
+                                                 FLEX_EWORKSPACE)
+    p = ctypes.c_void_p(4096)  # never dereferenced: validation fails first
+    ok = FlexShape(2, 3, 300, 64, 64, 1)
+    f32 = FlexShape(2, 3, 300, 64, 64, 0)
+    need = lib.flex_awd_bwd_workspace_bytes(ctypes.byref(ok))
+    assert need > lib.flex_awd_workspace_bytes(ctypes.byref(ok))
+    assert lib.flex_awd_bwd_workspace_bytes(ctypes.byref(f32)) == 0
+    f = lib.flex_awd_loss_bwd
+    # (shape, q, k, W1, W2, tau, causal, dloss, loss, dW1, dW2, dtau, ws, ws_bytes, stream)
+    assert f(ctypes.byref(ok), p, p, p, None, None, 0, None, p, p, None, None, p, need,
+             None) == FLEX_EINVAL                                   # no dloss
+    assert f(ctypes.byref(ok), p, p, p, p, None, 0, p, p, p, None, None, p, need,
+             None) == FLEX_EINVAL                                   # W2 without dW2
+    assert f(ctypes.byref(ok), p, p, p, None, None, 0, p, p, p, p, None, p, need,
+             None) == FLEX_EINVAL                                   # dW2 without W2
+    assert f(ctypes.byref(ok), p, p, p, None, p, 0, p, p, p, None, None, p, need,
+             None) == FLEX_EINVAL                                   # tau without dtau
+    assert f(ctypes.byref(f32), p, p, p, None, None, 0, p, p, p, None, None, p, need,
+             None) == FLEX_EUNSUPPORTED
+    assert f(ctypes.byref(ok), p, p, p, None, None, 0, p, p, p, None, None, p, need - 1,
+             None) == FLEX_EWORKSPACE
+    assert f(ctypes.byref(ok), p, p, p, None, None, 0, p, p, ctypes.c_void_p(4100), None, None,
+             p, need, None) == FLEX_EINVAL                          # misaligned dW1
