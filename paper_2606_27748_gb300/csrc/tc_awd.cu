@@ -281,61 +281,71 @@ __global__ void awd_reduce_kernel(int BH, int nqb, int N, const float* __restric
 // teacher mass on the entries with R_ij > 0) and sigma = -dloss / N:
 //   dL/dA~_ij = sigma G_ij,   G_ij = [A~_ij sign(D_i) > 0] P_ij / A~_ij - e_i   (j in row i)
 //   dphi(q_i) = sigma sum_j G_ij phi~(k_j),   dphi~(k_j) = sigma sum_i G_ij phi(q_i).
-// One CTA per (sequence, side): the query side holds a block of 128 queries and streams
-// the key blocks, the key side holds 128 keys and streams the query blocks.  Per streamed
-// block thread 0 issues S = X_own X_other^T and A = Phi_own Phi_other^T into tensor memory;
-// each thread turns half of its row into G (two SFU operations per entry: ex2, divide),
-// writes it as bf16 in place over A, and G Phi_other (A operand in tensor memory, features
-// MN-major) accumulates into T_D.  Then, per group of 64 frequencies, the chain rule through
-// the feature map runs on the tensor cores: the projection X_own W'^T is recomputed, the
-// epilogue forms da (du | dw for Flexformer_n) from T_D, and dW' += da^T X_own.  The rows
-// of dW' are added into this CTA's slot (fixed order); a reduction sums the slots over the
-// batch and both sides in a fixed order.  On the key side, with the prefactor, the chain
-// rule takes dphi(k_j) = w_j dphi~(k_j) and dtau gains -(phi~(k_j) . dphi~(k_j)) |k_j|^2
-// exp(-tau).  Every wait is bounded.
+// A sequence's query side holds blocks of 128 queries and streams the key blocks; its key
+// side holds blocks of 128 keys and streams the query blocks; each side's held blocks are
+// split over `hsplit` CTAs.  Per streamed block thread 0 issues S = X_own X_other^T and
+// A = Phi_own Phi_other^T into tensor memory; 16 warps (four per lane quadrant, each on 32
+// of the 128 columns) turn their part of the rows into G (two SFU operations per entry:
+// ex2 and a divide), write it as bf16 in place over the columns they read, and G Phi_other
+// (A operand in tensor memory, features MN-major) accumulates into T_D.  With M = 64 the
+// streamed tiles are double-buffered: the next block's load is issued as soon as the
+// current one has landed.  Then, per group of 64 frequencies, the chain rule through the
+// feature map runs on the tensor cores: the projection X_own W'^T is recomputed, the
+// epilogue forms da (du | dw for Flexformer_n) from T_D, and dW' += da^T X_own.  The rows of
+// dW' are added into this CTA's slot; a reduction sums the slots over the sides, the batch
+// and the splits in a fixed order, so the result does not depend on scheduling.  On the
+// key side, with the prefactor, the chain rule takes dphi(k_j) = w_j dphi~(k_j) and dtau
+// gains -(phi~(k_j) . dphi~(k_j)) |k_j|^2 exp(-tau).  Every wait is bounded.
+constexpr int kThreadsG = 512;
+
 template <int G2>
 struct AwdBwCfg {
-    static constexpr uint32_t XO = 0, XT = 16384, PO = 32768, PT = PO + G2 * 16384;
-    static constexpr uint32_t BYTES = PT + G2 * 16384;
-    static constexpr uint32_t WG = XT;  // after the streamed blocks: one group's W' rows
-    static constexpr uint32_t DA = PT;  // and the da tiles [du | dw]
+    static constexpr int STAGES = G2 == 2 ? 2 : 1;          // streamed tiles in flight
+    static constexpr uint32_t XO = 0, PO = 16384, ST0 = PO + G2 * 16384;
+    static constexpr uint32_t STAGE_BYTES = (1 + G2) * 16384;  // x tile, then features
+    static constexpr uint32_t WG = ST0 + STAGES * STAGE_BYTES;  // W' rows of every group
+    static constexpr uint32_t BYTES = WG + (G2 / 2) * 16384;   // (at most 16 KB a group)
+    static constexpr uint32_t DA = ST0 + 16384;  // after the streamed blocks: da [du | dw]
     static constexpr uint32_t T_S = 0, T_A = 128, T_D = 256;
     static_assert(G2 >= 2 && BYTES + 1024 <= 232448, "shared memory budget");
 };
 
 template <int G2, bool NS, bool KW>
-__global__ void __launch_bounds__(kThreadsA, 1)
+__global__ void __launch_bounds__(kThreadsG, 1)
     tc_awd_bwd_kernel(const __grid_constant__ CUtensorMap tmap_q,
                       const __grid_constant__ CUtensorMap tmap_k,
                       const __grid_constant__ CUtensorMap tmap_pq,
                       const __grid_constant__ CUtensorMap tmap_pk, int BH, int H, int N, int M,
-                      int causal, float score_scale, const float4* __restrict__ rowstat,
-                      const float* __restrict__ dloss, const float* __restrict__ W1,
-                      const float* __restrict__ W2, const float* __restrict__ kw,
-                      const float* __restrict__ tau, float* __restrict__ slots,
-                      float* __restrict__ dtau_part, int* status)
+                      int causal, int hsplit, float score_scale,
+                      const float4* __restrict__ rowstat, const float* __restrict__ dloss,
+                      const float* __restrict__ W1, const float* __restrict__ W2,
+                      const float* __restrict__ kw, const float* __restrict__ tau,
+                      float* __restrict__ slots, float* __restrict__ dtau_part, int* status)
 {
     using L = AwdBwCfg<G2>;
     constexpr int P = NS ? 128 : 64;  // projection rows per group of 64 frequencies
     constexpr int G = G2 / 2;
+    constexpr int S = L::STAGES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const uint32_t sb = smem_u32(sm);
     __shared__ uint32_t tmem_base_sh;
-    __shared__ __align__(8) uint64_t mbar, tma_bar;
+    __shared__ __align__(8) uint64_t mbar, tma_bar[S];
     __shared__ volatile int abort_flag;
     __shared__ float4 ostat[kC];  // key side: statistics of the streamed query rows
-    __shared__ float wsum[kThreadsA / 32];
+    __shared__ float wsum[kThreadsG / 32];
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int wg = warp >> 2, quad = warp & 3, t = 32 * quad + lane;
-    const bool kside = (int)blockIdx.x >= BH;
-    const int bh = (int)blockIdx.x % BH, h = bh % H;
+    const int qd = warp >> 2, quad = warp & 3, t = 32 * quad + lane;  // qd: column quarter
+    const int seq = (int)blockIdx.x / hsplit, split = (int)blockIdx.x % hsplit;
+    const bool kside = seq >= BH;
+    const int bh = seq % BH, h = bh % H;
     const CUtensorMap* x_own = kside ? &tmap_k : &tmap_q;
     const CUtensorMap* x_oth = kside ? &tmap_q : &tmap_k;
     const CUtensorMap* f_own = kside ? &tmap_pk : &tmap_pq;
     const CUtensorMap* f_oth = kside ? &tmap_pq : &tmap_pk;
     const int nblk = (N + kC - 1) / kC;
+    const int hb0 = split * nblk / hsplit, hb1 = (split + 1) * nblk / hsplit;
     const float sigma = -dloss[bh] / (float)N;
     const float itau = KW ? expf(-tau[h]) : 0.f;
     const float cM = rsqrtf((float)M);
@@ -343,7 +353,7 @@ __global__ void __launch_bounds__(kThreadsA, 1)
 
     if (tid == 0) {
         mbar_init(&mbar, 1);
-        mbar_init(&tma_bar, 1);
+        for (int s = 0; s < S; ++s) mbar_init(&tma_bar[s], 1);
         abort_flag = 0;
         fence_mbar_init();
     }
@@ -356,12 +366,10 @@ __global__ void __launch_bounds__(kThreadsA, 1)
     fence_after_sync();
     const uint32_t tm = tmem_base_sh;
     const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
-    uint32_t phase = 0, tma_phase = 0;
+    uint32_t phase = 0, tph = 0;  // tph: bit st = parity of stage st's barrier
     auto adv = [](uint64_t dsc, uint32_t bytes) { return dsc + (bytes >> 4); };
-    const uint64_t dXO = sdesc(sb + L::XO, 16, 1024), dXT = sdesc(sb + L::XT, 16, 1024);
-    const uint64_t dPO = sdesc(sb + L::PO, 16, 1024), dPT = sdesc(sb + L::PT, 16, 1024);
-    const uint64_t dPTmn = sdesc(sb + L::PT, 16384, 1024);
-    const uint64_t dWg = sdesc(sb + L::WG, 16, 1024);
+    auto xt = [](int st) { return L::ST0 + (uint32_t)st * L::STAGE_BYTES; };
+    const uint64_t dXO = sdesc(sb + L::XO, 16, 1024), dPO = sdesc(sb + L::PO, 16, 1024);
     const uint64_t dDAmn = sdesc(sb + L::DA, 16384, 1024), dXOmn = sdesc(sb + L::XO, 16384, 1024);
     constexpr uint32_t I_KK128 = idesc_bf16(128, 128, 0, 0);
     constexpr uint32_t I_DPHI = idesc_bf16(128, 64 * G2, 0, 1);  // N = 2M features
@@ -381,41 +389,51 @@ __global__ void __launch_bounds__(kThreadsA, 1)
         fence_after_sync();
         return ok_;
     };
-    // the streamed block ot (and first the held block ob): one arrival per phase
-    auto load = [&](int ob, int ot, bool own_too) {
-        mbar_arrive_expect_tx(&tma_bar, (1 + G2) * kTileBytes * (own_too ? 2 : 1));
+    // streamed block ot into stage st (and first the held block ob): one arrival per phase
+    auto load = [&](int ob, int ot, int st, bool own_too) {
+        mbar_arrive_expect_tx(&tma_bar[st], (1 + G2) * kTileBytes * (own_too ? 2 : 1));
         if (own_too) {
-            tma_load_3d(sb + L::XO, x_own, 0, ob * kC, bh, &tma_bar);
+            tma_load_3d(sb + L::XO, x_own, 0, ob * kC, bh, &tma_bar[st]);
             for (int g = 0; g < G2; ++g)
-                tma_load_3d(sb + L::PO + g * 16384, f_own, 64 * g, ob * kC, bh, &tma_bar);
+                tma_load_3d(sb + L::PO + g * 16384, f_own, 64 * g, ob * kC, bh, &tma_bar[st]);
         }
-        tma_load_3d(sb + L::XT, x_oth, 0, ot * kC, bh, &tma_bar);
+        tma_load_3d(sb + xt(st), x_oth, 0, ot * kC, bh, &tma_bar[st]);
         for (int g = 0; g < G2; ++g)
-            tma_load_3d(sb + L::PT + g * 16384, f_oth, 64 * g, ot * kC, bh, &tma_bar);
+            tma_load_3d(sb + xt(st) + 16384 + g * 16384, f_oth, 64 * g, ot * kC, bh,
+                        &tma_bar[st]);
     };
     // streamed blocks of held block ob: causal queries see keys j <= i
     auto first_other = [&](int ob) { return (kside && causal) ? ob : 0; };
     auto last_other = [&](int ob) { return (!kside && causal) ? ob : nblk - 1; };
 
     bool ok = true;
-    if (tid == 0) load(0, first_other(0), true);
-    for (int ob = 0; ob < nblk && ok; ++ob) {
+    if (tid == 0) load(hb0, first_other(hb0), 0, true);
+    // this head's W' rows, all groups, once (overlaps the first load; made visible to the
+    // tensor cores by the fence here and the barrier at the first wait)
+    stage_freq_rows<NS, G, kThreadsG>(sb + L::WG, W1, W2, h, M, tid);
+    fence_proxy_async();
+    for (int ob = hb0; ob < hb1 && ok; ++ob) {
         const int own_row = ob * kC + t;
         const bool own_valid = own_row < N;
         float4 qs = make_float4(0.f, 0.f, 0.f, 0.f);
         if (!kside && own_valid) qs = rowstat[(size_t)bh * N + own_row];
         const int o0 = first_other(ob), o1 = last_other(ob);
         for (int ot = o0; ot <= o1; ++ot) {
+            const int st = S == 2 ? (ot - o0) & 1 : 0;
             if (kside && tid < kC) {
                 const int r = ot * kC + tid;
                 ostat[tid] = r < N ? rowstat[(size_t)bh * N + r] : make_float4(0.f, 0.f, 0.f, 0.f);
             }
-            ok = bar_wait(&tma_bar, tma_phase, &abort_flag, status);
-            tma_phase ^= 1;
+            ok = bar_wait(&tma_bar[st], (tph >> st) & 1u, &abort_flag, status);
+            tph ^= 1u << st;
             ok = !__syncthreads_or(!ok);
             if (!ok) break;
             fence_after_sync();
             if (tid == 0) {
+                // the other stage was last read by the previous block's MMAs, now complete
+                if (S == 2 && ot < o1) load(ob, ot + 1, st ^ 1, false);
+                const uint64_t dXT = sdesc(sb + xt(st), 16, 1024);
+                const uint64_t dPT = sdesc(sb + xt(st) + 16384, 16, 1024);
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
                     mma_bf16(tm + L::T_S, adv(dXO, ks * 32), adv(dXT, ks * 32), I_KK128, ks > 0);
@@ -426,46 +444,52 @@ __global__ void __launch_bounds__(kThreadsA, 1)
                 }
             }
             if (!(ok = commit_wait())) break;
-            // G over this thread's 64 columns, two rounds of 32, bf16 in place over A
+            // G over this thread's 32 columns (two rounds of 16), bf16 in place over A in
+            // the first 16 of them; a block with no masked entry skips the mask tests
+            const bool full = (ot + 1) * kC <= N && (ob + 1) * kC <= N &&
+                              (!causal || (kside ? ot > ob : ot < ob));
 #pragma unroll
             for (int b = 0; b < 2; ++b) {
-                const uint32_t col = 64 * wg + 32 * b;
-                float sv[32], av[32];
-                tmem_ld16(tm_row + L::T_S + col, *reinterpret_cast<float(*)[16]>(&sv[0]));
-                tmem_ld16(tm_row + L::T_S + col + 16, *reinterpret_cast<float(*)[16]>(&sv[16]));
-                tmem_ld16(tm_row + L::T_A + col, *reinterpret_cast<float(*)[16]>(&av[0]));
-                tmem_ld16(tm_row + L::T_A + col + 16, *reinterpret_cast<float(*)[16]>(&av[16]));
+                const uint32_t col = 32 * qd + 16 * b;
+                float sv[16], av[16];
+                tmem_ld16(tm_row + L::T_S + col, sv);
+                tmem_ld16(tm_row + L::T_A + col, av);
                 tmem_wait_ld();
-                uint32_t pk[16];
+                uint32_t pk[8];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
+                for (int i = 0; i < 8; ++i) {
                     float gv[2];
 #pragma unroll
                     for (int e = 0; e < 2; ++e) {
-                        const int c = (int)col + 2 * i + e, orow = ot * kC + c;
-                        const int qi = kside ? orow : own_row, kj = kside ? own_row : orow;
-                        const bool in = own_valid && orow < N && (!causal || kj <= qi);
-                        const float4 st = kside ? ostat[c] : qs;
+                        const int c = (int)col + 2 * i + e;
+                        const float4 sts = kside ? ostat[c] : qs;
                         const float a = av[2 * i + e];
-                        const float p = ex2f(fmaf(sv[2 * i + e], score_scale, -st.x));
-                        const float first = a * st.y > 0.f ? __fdividef(p, a) : 0.f;
-                        gv[e] = in ? first - st.z : 0.f;
+                        const float p = ex2f(fmaf(sv[2 * i + e], score_scale, -sts.x));
+                        const float g = (a * sts.y > 0.f ? __fdividef(p, a) : 0.f) - sts.z;
+                        if (full) {
+                            gv[e] = g;
+                        } else {
+                            const int orow = ot * kC + c;
+                            const int qi = kside ? orow : own_row, kj = kside ? own_row : orow;
+                            gv[e] = (own_valid && orow < N && (!causal || kj <= qi)) ? g : 0.f;
+                        }
                     }
                     pk[i] = pack_bf16(gv[0], gv[1]);
                 }
-                tmem_st16(tm_row + L::T_A + 64 * wg + 16 * b, pk);
+                tmem_st8(tm_row + L::T_A + 32 * qd + 8 * b, pk);
             }
             tmem_wait_st();
             handoff();
             if (tid == 0) {
                 fence_after_sync();
+                const uint64_t dPTmn = sdesc(sb + xt(st) + 16384, 16384, 1024);
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks)
-                    mma_bf16_tmem_a(tm + L::T_D, tm + L::T_A + 64 * (ks >> 2) + 8 * (ks & 3),
+                for (int ks = 0; ks < 8; ++ks)  // K = streamed rows 16 ks .. 16 ks + 15
+                    mma_bf16_tmem_a(tm + L::T_D, tm + L::T_A + 32 * (ks >> 1) + 8 * (ks & 1),
                                     adv(dPTmn, ks * 2048), I_DPHI, (ot > o0 || ks > 0) ? 1u : 0u);
             }
             if (!(ok = commit_wait())) break;
-            if (tid == 0 && ot < o1) load(ob, ot + 1, false);
+            if (S == 1 && tid == 0 && ot < o1) load(ob, ot + 1, 0, false);
         }
         if (!ok) break;
 
@@ -488,30 +512,24 @@ __global__ void __launch_bounds__(kThreadsA, 1)
             }
         }
         for (int g = 0; g < G && ok; ++g) {
-            stage_freq_rows<NS, 1, kThreadsA>(sb + L::WG, W1, W2, h, M, tid, 64 * g);
-            handoff();
             if (tid == 0) {
-                fence_after_sync();
+                fence_after_sync();  // after the previous group's barrier
+                const uint64_t dWg = sdesc(sb + L::WG + (uint32_t)g * P * 128, 16, 1024);
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
                     mma_bf16(tm + L::T_S, adv(dXO, ks * 32), adv(dWg, ks * 32), I_PROJ, ks > 0);
             }
             if (!(ok = commit_wait())) break;
-            float dc[32], ds[32], u[32], w[32];
-            tmem_ld16(tm_row + L::T_D + 64 * g + 32 * wg, *reinterpret_cast<float(*)[16]>(&dc[0]));
-            tmem_ld16(tm_row + L::T_D + 64 * g + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&dc[16]));
-            tmem_ld16(tm_row + L::T_D + M + 64 * g + 32 * wg, *reinterpret_cast<float(*)[16]>(&ds[0]));
-            tmem_ld16(tm_row + L::T_D + M + 64 * g + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&ds[16]));
-            tmem_ld16(tm_row + L::T_S + 32 * wg, *reinterpret_cast<float(*)[16]>(&u[0]));
-            tmem_ld16(tm_row + L::T_S + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&u[16]));
-            if (NS) {
-                tmem_ld16(tm_row + L::T_S + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]));
-                tmem_ld16(tm_row + L::T_S + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
-            }
+            // this thread's 16 frequencies of the group: 64 g + 16 qd + [0, 16)
+            float dc[16], ds[16], u[16], w[16];
+            tmem_ld16(tm_row + L::T_D + 64 * g + 16 * qd, dc);
+            tmem_ld16(tm_row + L::T_D + M + 64 * g + 16 * qd, ds);
+            tmem_ld16(tm_row + L::T_S + 16 * qd, u);
+            if (NS) tmem_ld16(tm_row + L::T_S + 64 + 16 * qd, w);
             tmem_wait_ld();
-            uint32_t o1[16], o2[16];
+            uint32_t o1[8], o2[8];
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
+            for (int i = 0; i < 8; ++i) {
                 float r1[2], r2[2];
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
@@ -530,8 +548,8 @@ __global__ void __launch_bounds__(kThreadsA, 1)
                 o2[i] = pack_bf16(r2[0], r2[1]);
             }
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const uint32_t off = swz128(t, (4 * wg + j) * 8);
+            for (int j = 0; j < 2; ++j) {
+                const uint32_t off = swz128(t, (2 * qd + j) * 8);
                 st_shared_v4(sb + L::DA + off, o1[4 * j], o1[4 * j + 1], o1[4 * j + 2], o1[4 * j + 3]);
                 st_shared_v4(sb + L::DA + 16384 + off, o2[4 * j], o2[4 * j + 1], o2[4 * j + 2],
                              o2[4 * j + 3]);
@@ -544,16 +562,15 @@ __global__ void __launch_bounds__(kThreadsA, 1)
                     mma_bf16(tm + L::T_A, adv(dDAmn, ks * 2048), adv(dXOmn, ks * 2048), I_DW, ks > 0);
             }
             if (!(ok = commit_wait())) break;
-            // rows of dW' (lane = projection row) added into this CTA's slot
-            float v[32];
-            tmem_ld16(tm_row + L::T_A + 32 * wg, *reinterpret_cast<float(*)[16]>(&v[0]));
-            tmem_ld16(tm_row + L::T_A + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&v[16]));
+            // rows of dW' (lane = projection row), this thread's 16 columns, into the slot
+            float v[16];
+            tmem_ld16(tm_row + L::T_A + 16 * qd, v);
             tmem_wait_ld();
             float4* dst = reinterpret_cast<float4*>(
-                slots + (((size_t)blockIdx.x * G + g) * 128 + t) * 64 + 32 * wg);
+                slots + (((size_t)blockIdx.x * G + g) * 128 + t) * 64 + 16 * qd);
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const float4 old = ob == 0 ? make_float4(0.f, 0.f, 0.f, 0.f) : dst[j];
+            for (int j = 0; j < 4; ++j) {
+                const float4 old = ob == hb0 ? make_float4(0.f, 0.f, 0.f, 0.f) : dst[j];
                 dst[j] = make_float4(old.x + v[4 * j], old.y + v[4 * j + 1], old.z + v[4 * j + 2],
                                      old.w + v[4 * j + 3]);
             }
@@ -564,7 +581,7 @@ __global__ void __launch_bounds__(kThreadsA, 1)
         if (!ok) break;
         if (KW && kside && own_valid)  // s_j = phi~(k_j) . dphi~(k_j) = w cM sigma sdot
             dtau_acc -= wk * cM * sigma * sdot * kk * itau;
-        if (tid == 0 && ob + 1 < nblk) load(ob + 1, first_other(ob + 1), true);
+        if (tid == 0 && ob + 1 < hb1) load(ob + 1, first_other(ob + 1), 0, true);
     }
 
     // dtau partial of this CTA, summed in a fixed order
@@ -574,7 +591,7 @@ __global__ void __launch_bounds__(kThreadsA, 1)
     __syncthreads();
     if (tid == 0) {
         float tot = 0.f;
-        for (int w8 = 0; w8 < kThreadsA / 32; ++w8) tot += wsum[w8];
+        for (int w8 = 0; w8 < kThreadsG / 32; ++w8) tot += wsum[w8];
         dtau_part[blockIdx.x] = tot;
     }
     fence_before_sync();
@@ -583,39 +600,70 @@ __global__ void __launch_bounds__(kThreadsA, 1)
     if (warp == 0) tmem_dealloc(tm, 512);
 }
 
-// dW1, dW2 [H][M][64] and dtau [H] from the slots [2 sides][B*H][G][128 rows][64]: sum over
-// the sides and the batch in a fixed order; Flexformer_n rows 0-63 of a group are dU, rows
-// 64-127 dV (U = (W1+W2)/2, V = (W1-W2)/2), so dW1 = (dU+dV)/2, dW2 = (dU-dV)/2.
-__global__ void awd_dw_reduce_kernel(int B, int H, int M, int nonstat,
-                                     const float* __restrict__ slots,
-                                     const float* __restrict__ dtau_part, float* __restrict__ dW1,
-                                     float* __restrict__ dW2, float* __restrict__ dtau)
+// dW1, dW2 [H][M][64] and dtau [H] from the slots [2 sides][B*H][hsplit][G][128 rows][64].
+// One block of 512 threads per (head, frequency): column c = tid % 64, lane = tid / 64 sums
+// the slots s = lane, lane + 8, ... (s in (side, batch entry, split) order), eight loads in
+// flight; the eight lane sums are then added in lane order, so the order is fixed.  For
+// Flexformer_n rows 0-63 of a group are dU, rows 64-127 dV (U = (W1+W2)/2, V = (W1-W2)/2),
+// so dW1 = (dU+dV)/2, dW2 = (dU-dV)/2.
+constexpr int kReduceLanes = 8;
+__global__ void __launch_bounds__(64 * kReduceLanes)
+    awd_dw_reduce_kernel(int B, int H, int M, int nonstat, int hsplit,
+                         const float* __restrict__ slots, const float* __restrict__ dtau_part,
+                         float* __restrict__ dW1, float* __restrict__ dW2,
+                         float* __restrict__ dtau)
 {
-    const int BH = B * H, G = M / 64;
-    const size_t total = (size_t)H * M * 64;
-    for (size_t idx = (size_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-         idx += (size_t)gridDim.x * blockDim.x) {
-        const int c = (int)(idx % 64), f = (int)((idx / 64) % M), h = (int)(idx / ((size_t)64 * M));
-        const int g = f / 64, r = f % 64;
-        float su = 0.f, sv = 0.f;
-        for (int side = 0; side < 2; ++side)
-            for (int b = 0; b < B; ++b) {
-                const float* sl = slots + (((size_t)(side * BH + b * H + h) * G + g) * 128) * 64;
-                su += sl[r * 64 + c];
-                if (nonstat) sv += sl[(64 + r) * 64 + c];
+    __shared__ float part[2][kReduceLanes][64];
+    const int BH = B * H, G = M / 64, per_side = B * hsplit, nslot = 2 * per_side;
+    const size_t slot_floats = (size_t)G * 128 * 64;
+    const int c = threadIdx.x % 64, lane = threadIdx.x / 64;
+    const int f = blockIdx.x % M, h = blockIdx.x / M;
+    const float* base = slots + ((size_t)(f / 64) * 128 + f % 64) * 64 + c;
+    float su = 0.f, sv = 0.f;
+    for (int s0 = lane; s0 < nslot; s0 += 8 * kReduceLanes) {
+        float a[8], bq[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int s = s0 + e * kReduceLanes;
+            a[e] = bq[e] = 0.f;
+            if (s < nslot) {
+                const int side = s / per_side, rem = s % per_side;
+                const size_t cta = (size_t)(side * BH + (rem / hsplit) * H + h) * hsplit +
+                                   rem % hsplit;
+                a[e] = base[cta * slot_floats];
+                if (nonstat) bq[e] = base[cta * slot_floats + 64 * 64];
             }
+        }
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            su += a[e];
+            sv += bq[e];
+        }
+    }
+    part[0][lane][c] = su;
+    part[1][lane][c] = sv;
+    __syncthreads();
+    if (lane == 0) {
+        float tu = 0.f, tv = 0.f;
+        for (int l = 0; l < kReduceLanes; ++l) {
+            tu += part[0][l][c];
+            tv += part[1][l][c];
+        }
+        const size_t idx = ((size_t)h * M + f) * 64 + c;
         if (nonstat) {
-            dW1[idx] = 0.5f * (su + sv);
-            dW2[idx] = 0.5f * (su - sv);
+            dW1[idx] = 0.5f * (tu + tv);
+            dW2[idx] = 0.5f * (tu - tv);
         } else {
-            dW1[idx] = su;
+            dW1[idx] = tu;
         }
     }
     if (dtau && blockIdx.x == 0)
-        for (int h = threadIdx.x; h < H; h += blockDim.x) {
+        for (int hh = threadIdx.x; hh < H; hh += blockDim.x) {
             float sd = 0.f;
-            for (int b = 0; b < B; ++b) sd += dtau_part[BH + b * H + h];  // key side
-            dtau[h] = sd;
+            for (int b = 0; b < B; ++b)
+                for (int r = 0; r < hsplit; ++r)  // key side
+                    sd += dtau_part[(size_t)(BH + b * H + hh) * hsplit + r];
+            dtau[hh] = sd;
         }
 }
 
@@ -642,6 +690,16 @@ cudaError_t launch_typed(const Problem& p, const void* q, const void* k, const v
     return cudaGetLastError();
 }
 
+// CTAs per (side, sequence) of the gradient kernel: held blocks are split until the grid
+// covers the GPU about four times over (whole blocks per CTA).
+int awd_hsplit(const Problem& p)
+{
+    const int nblk = (p.N + kC - 1) / kC;
+    int hs = 1;
+    while (hs * 2 <= nblk && 2LL * p.B * p.H * hs < 4LL * 152) hs *= 2;
+    return hs;
+}
+
 template <int G2, bool NS, bool KW>
 cudaError_t launch_bwd_typed(const Problem& p, const void* q, const void* k, const void* pq,
                              const void* pk, const float* W1, const float* W2, const float* kw,
@@ -659,14 +717,13 @@ cudaError_t launch_bwd_typed(const Problem& p, const void* q, const void* k, con
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     const float score_scale = 1.4426950408889634f / sqrtf((float)p.d);
-    kern<<<2 * BH, kThreadsA, smem, s>>>(mq, mk, mpq, mpk, BH, p.H, p.N, p.M, p.causal,
-                                         score_scale, rowstat, dloss, W1, W2, kw, tau, slots,
-                                         dtau_part, status);
+    const int hs = awd_hsplit(p);
+    kern<<<2 * BH * hs, kThreadsG, smem, s>>>(mq, mk, mpq, mpk, BH, p.H, p.N, p.M, p.causal, hs,
+                                              score_scale, rowstat, dloss, W1, W2, kw, tau, slots,
+                                              dtau_part, status);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    const size_t total = (size_t)p.H * p.M * 64;
-    const int grid = (int)std::min<size_t>((total + 255) / 256, 152 * 8);
-    awd_dw_reduce_kernel<<<grid, 256, 0, s>>>(p.B, p.H, p.M, p.nonstat, slots, dtau_part, dW1,
-                                              dW2, tau ? dtau : nullptr);
+    awd_dw_reduce_kernel<<<p.H * p.M, 64 * kReduceLanes, 0, s>>>(
+        p.B, p.H, p.M, p.nonstat, hs, slots, dtau_part, dW1, dW2, tau ? dtau : nullptr);
     return cudaGetLastError();
 }
 
@@ -706,7 +763,7 @@ size_t tc_awd_part_floats(const Problem& p)
 
 size_t tc_awd_slot_floats(const Problem& p)
 {
-    return (size_t)2 * p.B * p.H * (p.M / 64) * 128 * 64;
+    return (size_t)2 * p.B * p.H * awd_hsplit(p) * (p.M / 64) * 128 * 64;
 }
 
 cudaError_t launch_tc_awd(const Problem& p, const void* q, const void* k, const void* pq,
