@@ -101,11 +101,11 @@ inline bool make_act_map(CUtensorMap* m, const void* base, int BH, int N)
 
 // One head's frequency rows into shared memory, bf16, K-major with 128-byte swizzle: G
 // groups of P rows (s: P = 64 rows of W1; n: P = 128, U = (W1+W2)/2 then V = (W1-W2)/2),
-// row r of group g = frequency f0 + 64 g + r % 64.  8-float pieces by float4 loads, a batch
-// of up to 4 pieces per thread in flight.  W1, W2: [H][M][64] fp32, 16-byte aligned.
+// row r of group g = frequency 64 g + r % 64.  8-float pieces by float4 loads, a batch of
+// up to 4 pieces per thread in flight.  W1, W2: [H][M][64] fp32, 16-byte aligned.
 template <bool NS, int G, int NTHREADS>
 __device__ __forceinline__ void stage_freq_rows(uint32_t dst, const float* W1, const float* W2,
-                                                int h, int M, int tid, int f0 = 0)
+                                                int h, int M, int tid)
 {
     constexpr int P = NS ? 128 : 64;
     static_assert(G * P * 8 % NTHREADS == 0, "whole pieces per thread");
@@ -115,7 +115,7 @@ __device__ __forceinline__ void stage_freq_rows(uint32_t dst, const float* W1, c
 #pragma unroll
         for (int i = 0; i < kBatch; ++i) {
             const int idx = tid + NTHREADS * (i0 + i), r = idx >> 3, c = idx & 7;
-            const int f = f0 + 64 * (r / P) + ((r % P) & 63);
+            const int f = 64 * (r / P) + ((r % P) & 63);
             const float4* w1 = reinterpret_cast<const float4*>(W1 + ((size_t)h * M + f) * 64 + c * 8);
             a[i][0] = __ldg(w1);
             a[i][1] = __ldg(w1 + 1);
