@@ -34,8 +34,9 @@ Facts used (none is the oracle's own formula retyped):
     (loss >= the teacher's entropy); keys of equal norm make tau irrelevant; entries with
     a non-positive normalised weight count log 1e-6 in both forms.
   * its gradient with respect to W1, W2 and tau: central finite differences of the numpy
-    form (cases with negative kernel entries); one key gives 0; keys of equal norm give
-    dtau = 0; W2 = W1 gives dW1 + dW2 = the stationary gradient.
+    form (cases with negative kernel entries); d = 1, M = 1 in closed form; one key gives
+    0; keys of equal norm give dtau = 0; W2 = W1 gives dW1 + dW2 = the stationary
+    gradient.
 """
 from __future__ import annotations
 
@@ -451,6 +452,29 @@ def pin_awd_grad_finite_differences(orc):
                                         f"tau={tau is not None} #{idx}: {err:.2e}")
 
 
+def pin_awd_grad_closed_form_d1(orc):
+    """d = 1, M = 1, stationary: A_ij is proportional to cos(w D_ij), D_ij = q_i - k_j, so
+    dL/dw = -(1/N) sum_i [ sum_j P_ij (-D_ij tan(w D_ij))  -  c_i (sum_j -D_ij sin(w D_ij))
+    / (sum_j cos(w D_ij)) ]  with every entry positive here (c_i = 1), written out."""
+    q = np.array([0.3, -0.4, 0.2, 0.5]).reshape(1, 1, 4, 1)
+    k = np.array([0.1, 0.25, -0.3, 0.0]).reshape(1, 1, 4, 1)
+    w = 0.7
+    for causal in (False, True):
+        dW1, _, _ = orc.awd_bwd(q, k, np.array([[[w]]]), None, causal)
+        qq, kk = q.reshape(4, 1), k.reshape(1, 4)
+        Dl = qq - kk
+        mask = np.tril(np.ones((4, 4), bool)) if causal else np.ones((4, 4), bool)
+        s = np.where(mask, qq * kk, -np.inf)
+        P = np.exp(s - s.max(1, keepdims=True))
+        P /= P.sum(1, keepdims=True)
+        A = np.where(mask, np.cos(w * Dl), 0.0)
+        dA = np.where(mask, -Dl * np.sin(w * Dl), 0.0)
+        assert np.all(A[mask] > 0), "the case needs positive weights"
+        g = np.sum(P * np.where(mask, dA / np.where(mask, A, 1.0), 0.0), 1) - (
+            dA.sum(1) / A.sum(1))
+        assert abs(dW1[0, 0, 0] - (-np.sum(g) / 4)) < 1e-14, "awd grad closed form"
+
+
 def pin_awd_grad_single_key(orc):
     """One key: R = 1 whatever the parameters, so every gradient is exactly 0."""
     q, k, _, W1, W2 = _case(76, 2, 2, 1, 5, 7, "n")
@@ -490,4 +514,5 @@ ALL_PINS = [
     pin_awd_equals_brute, pin_awd_single_key, pin_awd_closed_form_d1, pin_awd_gibbs,
     pin_awd_equal_key_norms, pin_awd_nonpositive_entries, pin_awd_grad_finite_differences,
     pin_awd_grad_single_key, pin_awd_grad_equal_key_norms, pin_awd_grad_tied_frequencies,
+    pin_awd_grad_closed_form_d1,
 ]
