@@ -63,17 +63,11 @@ __device__ __forceinline__ void cp_async_wait_all()
     asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;\n" ::: "memory");
 }
 
-// sin and cos of x: Cody-Waite reduction by 2 pi (the fp32 value of 2 pi plus the fp32
-// value of the remainder, both computed from the mathematical constant) to |r| <= pi, then
-// the hardware approximations, whose absolute error on [-pi, pi] is a few 1e-7.
+// sin and cos of x: Cody-Waite reduction by 2 pi to |r| <= pi (tc::reduce_2pi), then the
+// hardware approximations, whose absolute error on [-pi, pi] is a few 1e-7.
 __device__ __forceinline__ void sincos_reduced(float x, float* s, float* c)
 {
-    constexpr float kInv2Pi = 0.15915493667125702f;
-    constexpr float k2PiHi = 6.2831854820251465f;
-    constexpr float k2PiLo = -1.7484555314695172e-07f;
-    const float n = rintf(x * kInv2Pi);
-    const float r = fmaf(-n, k2PiLo, fmaf(-n, k2PiHi, x));
-    __sincosf(r, s, c);
+    __sincosf(tc::reduce_2pi(x), s, c);
 }
 
 __device__ __forceinline__ float to_f32(float x) { return x; }

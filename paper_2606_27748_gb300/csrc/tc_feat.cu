@@ -6,9 +6,15 @@
 // One CTA per 4 blocks of 128 rows of one sequence (one head's frequencies, staged once),
 // 256 threads: TMA loads the rows (the next block while the current one is worked on),
 // thread 0 issues the projections x W^T (s: W1; n: U = (W1+W2)/2 and
-// V = (W1-W2)/2; bf16 operands, fp32 in tensor memory), one group of 64 frequencies per
-// 64 (s) or 128 (n) columns; every thread takes one row and 32 frequencies of each group:
-// hardware sin/cos, products, bf16 pack, 64-byte stores of its cos and sin runs.
+// V = (W1-W2)/2), one group of 64 frequencies per 64 (s) or 128 (n) columns; every thread
+// takes one row and 32 frequencies of each group: arguments reduced by 2 pi, hardware
+// sin/cos, products, bf16 pack, 64-byte stores of its cos and sin runs.
+//
+// The frequencies enter the projection split into bf16 high and low parts (two MMAs into
+// one fp32 accumulator): x is exactly bf16, so the projection carries the fp32
+// frequencies to about 2^-17 instead of bf16's 2^-9.  The phase error of a single bf16
+// rounding grows with the argument (|x . w| 2^-9), which would dominate the feature error
+// once trained frequencies push arguments past ~10.
 #include "flex_internal.h"
 #include "tc_common.cuh"
 #include "tc_util.cuh"
@@ -31,6 +37,7 @@ __global__ void __launch_bounds__(kThreadsF)
     constexpr int P = NS ? 128 : 64;        // projection rows (= tensor memory columns) per group
     constexpr uint32_t NCOLS = G * P;        // 64, 128 or 256: a power of two
     constexpr uint32_t X0 = 0, W = 32768;    // two x tiles, then G x P frequency rows
+    constexpr uint32_t WLO = W + G * P * 128; // their low parts
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const uint32_t sb = smem_u32(sm);
@@ -44,7 +51,7 @@ __global__ void __launch_bounds__(kThreadsF)
     const int bh = blockIdx.x / nchunk, b0 = (blockIdx.x % nchunk) * kBlocksPerCta, h = bh % H;
     const int nb = min(kBlocksPerCta, nblk - b0);
 
-    stage_freq_rows<NS, G, kThreadsF>(sb + W, W1, W2, h, M, tid);  // once per CTA
+    stage_freq_rows_split<NS, G, kThreadsF>(sb + W, sb + WLO, W1, W2, h, M, tid);  // once
     if (tid == 0) {
         mbar_init(&mbar, 1);
         mbar_init(&tma_bar[0], 1);
@@ -83,10 +90,15 @@ __global__ void __launch_bounds__(kThreadsF)
             const uint64_t dX = sdesc(sb + X0 + xb * 16384, 16, 1024);
             for (int g = 0; g < G; ++g) {
                 const uint64_t dW = sdesc(sb + W + g * P * 128, 16, 1024);
+                const uint64_t dWlo = sdesc(sb + WLO + g * P * 128, 16, 1024);
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
                     mma_bf16(tm + g * P, dX + ((ks * 32) >> 4), dW + ((ks * 32) >> 4), I_PROJ,
                              ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_bf16(tm + g * P, dX + ((ks * 32) >> 4), dWlo + ((ks * 32) >> 4), I_PROJ,
+                             1u);
             }
             mma_commit(&mbar);
         }
@@ -108,6 +120,8 @@ __global__ void __launch_bounds__(kThreadsF)
                 tmem_ld16(col + 80, *reinterpret_cast<float(*)[16]>(&w[16]));
             }
             tmem_wait_ld();
+            reduce_2pi_if_needed(a);
+            if (NS) reduce_2pi_if_needed(w);
             uint32_t pc[16], ps[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
@@ -149,7 +163,7 @@ cudaError_t launch_typed(const Problem& p, const void* x, const float* W1, const
     const int BH = p.B * p.H;
     if (!make_act_map(&mx, x, BH, p.N)) return cudaErrorInvalidValue;
     constexpr int P = NS ? 128 : 64;
-    const int smem = 32768 + G * P * 128 + 1024;
+    const int smem = 32768 + 2 * G * P * 128 + 1024;
     auto kern = tc_featmap_kernel<NS, G>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;

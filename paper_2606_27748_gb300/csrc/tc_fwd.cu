@@ -397,6 +397,8 @@ __global__ void __maxnreg__(96)
                         __syncwarp();
                         if (lane == 0) mbar_arrive(&bars.p_free);
                     }
+                    reduce_2pi_if_needed(a);
+                    if (NS) reduce_2pi_if_needed(w);
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
                         float s0, c0, s1, c1;

@@ -28,6 +28,41 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
                  : "memory");
 }
 
+// ---- sin/cos arguments ----------------------------------------------------------------
+// The hardware sin/cos (MUFU, reached through __sincosf / __cosf) is accurate to about
+// 2^-21 absolute on [-pi, pi]; beyond it the error grows with |x| (measured on GB300 over
+// 2^16 points per range: 2^-19.6 for |x| <= 10, 2^-17.8 for |x| <= 30, 2^-12.9 for
+// |x| <= 1000).  Projection values reach that range once the frequencies are trained
+// (Sec. 3.2: the spectral frequencies are learned), so arguments are first reduced by
+// 2 pi with a two-constant Cody-Waite step: n = rint(x / 2 pi), r = (x - n C1) - n C2,
+// C1 the fp32 value of 2 pi and C2 the fp32 value of 2 pi - C1, each fma rounding once;
+// measured after the reduction: 2^-21 for every |x| <= 2000.
+constexpr float kPi = 3.14159265358979f;
+constexpr float kInv2Pi = 0.15915493667125702f;
+constexpr float k2PiHi = 6.2831854820251465f;
+constexpr float k2PiLo = -1.7484555314695172e-07f;
+
+__device__ __forceinline__ float reduce_2pi(float x)
+{
+    const float n = rintf(x * kInv2Pi);
+    return fmaf(-n, k2PiLo, fmaf(-n, k2PiHi, x));
+}
+
+// Reduces every value of v when any lane of the warp holds one beyond [-pi, pi]; the test
+// costs one max per value, so inputs inside the range (the common case) skip the step.
+// Warp-collective: all 32 lanes call it together.
+template <int n>
+__device__ __forceinline__ void reduce_2pi_if_needed(float (&v)[n])
+{
+    float m = 0.f;
+#pragma unroll
+    for (int i = 0; i < n; ++i) m = fmaxf(m, fabsf(v[i]));
+    if (__any_sync(0xffffffffu, m > kPi)) {
+#pragma unroll
+        for (int i = 0; i < n; ++i) v[i] = reduce_2pi(v[i]);
+    }
+}
+
 // Bounded wait on one mbarrier phase.  On a time-out the CTA is told to stop (abort flag)
 // and the status word (if any) records FLEX_ETIMEOUT; every other wait then returns at once.
 __device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,

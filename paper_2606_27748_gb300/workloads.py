@@ -11,8 +11,9 @@ classification (LRA, N = 1K-4K, d = 64; Sec. 4.1) settings, extended to longer N
 Draw recipe: every (tensor, b, h) slice has its own PCG64 stream, seeded by
 ``(seed, tensor_id, b, h)`` (frequencies: ``(seed, tensor_id, h)``), so any subset of
 sequences can be regenerated without drawing the rest.  Tensor ids follow the draw order
-q=0, k=1, v=2, W1=3, W2=4, dO=5.  Values are drawn in float32; bf16 workloads are then
-rounded once to bf16 (round to nearest even) and the rounded values are what both sides use.
+q=0, k=1, v=2, W1=3, W2=4, dO=5 (6: the q/k offset of large-argument inputs).  Values are
+drawn in float32; bf16 workloads are then rounded once to bf16 (round to nearest even) and
+the rounded values are what both sides use.
 """
 from __future__ import annotations
 
@@ -20,7 +21,7 @@ import dataclasses
 
 import numpy as np
 
-Q, K, V, W1, W2, DO = range(6)
+Q, K, V, W1, W2, DO, OFFSET = range(7)
 
 
 @dataclasses.dataclass(frozen=True)
@@ -40,6 +41,11 @@ class Workload:
     backward: bool = False
     decode: bool = False  # recurrent decode steps: one new token per sequence per step
     awd: bool = False     # attention-weight distillation loss (q, k only)
+    # Large projection arguments |x . w| (the regime of trained frequencies): q and k of
+    # head h share an offset vector m_h ~ N(0, qk_offset^2 I) (every batch entry), and the
+    # frequencies are drawn with standard deviation w_scale / sqrt(d).
+    qk_offset: float = 0.0
+    w_scale: float = 1.0
 
     @property
     def tokens(self) -> int:
@@ -104,10 +110,24 @@ def _stream(*key):
 def _draw_seq(w: Workload, tensor: int, b: int, h: int, N: int) -> np.ndarray:
     g = _stream(w.seed, tensor, b, h)
     if tensor in (Q, K):
-        return g.standard_normal((N, w.d), dtype=np.float32) * np.float32(w.qk_scale)
+        x = g.standard_normal((N, w.d), dtype=np.float32) * np.float32(w.qk_scale)
+        if w.qk_offset:
+            x += draw_offset(w, [h])[0]
+        return x
     if tensor == V and w.v_dist == "uniform":
         return g.uniform(-1.0, 1.0, (N, w.d)).astype(np.float32)
     return g.standard_normal((N, w.d), dtype=np.float32)
+
+
+def draw_offset(w: Workload, hs=None) -> np.ndarray:
+    """float32 [len(hs), d]: the offset m_h shared by q and k of head h (zeros if none)."""
+    hs = range(w.H) if hs is None else hs
+    out = np.zeros((len(hs), w.d), dtype=np.float32)
+    if w.qk_offset:
+        for j, h in enumerate(hs):
+            out[j] = _stream(w.seed, OFFSET, h).standard_normal(w.d, dtype=np.float32)
+        out *= np.float32(w.qk_offset)
+    return out
 
 
 def draw_activation(w: Workload, tensor: int, bs=None, hs=None, N=None) -> np.ndarray:
@@ -125,12 +145,12 @@ def draw_activation(w: Workload, tensor: int, bs=None, hs=None, N=None) -> np.nd
 
 
 def draw_frequencies(w: Workload, tensor: int, hs=None) -> np.ndarray:
-    """float32 [len(hs), M, d] with entries ~ N(0, 1/d)."""
+    """float32 [len(hs), M, d] with entries ~ N(0, w_scale^2 / d)."""
     hs = range(w.H) if hs is None else hs
     out = np.empty((len(hs), w.M, w.d), dtype=np.float32)
     for j, h in enumerate(hs):
         out[j] = _stream(w.seed, tensor, h).standard_normal((w.M, w.d), dtype=np.float32)
-    return out * np.float32(1.0 / np.sqrt(w.d))
+    return out * np.float32(w.w_scale / np.sqrt(w.d))
 
 
 def draw_tau(w: Workload, hs=None) -> np.ndarray:

@@ -9,6 +9,7 @@ import torch
 F32_REL_L2 = 1e-4
 BF16_REL_L2 = 2e-2
 BF16_MAX_ABS = 5e-2
+ZERO_ABS = 1e-5  # an exactly-zero result
 
 
 def to_dev(a, dtype):
@@ -38,12 +39,13 @@ def assert_close(x, ref, dtype, what, max_abs_scale=1.0):
     """
     assert np.all(np.isfinite(x)), f"{what}: non-finite values"
     if np.linalg.norm(ref.ravel()) <= 1e-12 * np.sqrt(ref.size):
-        # The exact result is zero (e.g. dq at a causal sequence of length 1, whose
-        # output v_0 does not depend on q); relative error is undefined, so only the
-        # absolute bound applies: fp32 rounding noise, or the stated bf16 max-abs bound.
+        # The exact result is zero (e.g. dq, dk and dW at a sequence of length 1, whose
+        # output v_0 depends on neither q, k nor W); relative error is undefined.  The
+        # kernels form the two cancelling terms from the same rounded operands (g and
+        # c = -(g . out) from the bf16 g that feeds the MMAs), so the zero comes out to
+        # fp32 rounding for either storage type.
         m = float(np.max(np.abs(x)))
-        bound = 1e-5 if dtype == "f32" else BF16_MAX_ABS * max_abs_scale
-        assert m <= bound, f"{what}: exact zero expected, max |x| = {m:.3e}"
+        assert m <= ZERO_ABS, f"{what}: exact zero expected, max |x| = {m:.3e}"
         return 0.0
     r = rel_l2(x, ref)
     if dtype == "f32":
@@ -53,3 +55,33 @@ def assert_close(x, ref, dtype, what, max_abs_scale=1.0):
         assert r <= BF16_REL_L2, f"{what}: rel L2 {r:.3e} > {BF16_REL_L2}"
         assert m <= BF16_MAX_ABS, f"{what}: max-abs {m:.3e} > {BF16_MAX_ABS}"
     return r
+
+
+def assert_close_offset_split(x, ref, x0_rms, offsets, dtype, what):
+    """dW1/dW2 [H, M, d] of inputs whose q and k of head h share a large offset m_h.
+
+    dW_h = sum_t da_t x_t^T with x_t = m_h + x0_t.  Its component along m_h,
+    (sum_t da_t) |m_h|, is a sum whose terms cancel (exactly, for the stationary kernel:
+    phi_s(q + m) . phi_s(k + m) = phi_s(q) . phi_s(k)), so with bf16 operands its error
+    grows with the condition number kappa = |m_h| / rms |x0_t| of that sum, not with the
+    result.  The component orthogonal to m_h is held to the stated bound; the component
+    along m_h to the stated relative bound times kappa.
+    """
+    scale = float(np.sqrt(np.mean(ref * ref)))
+    mh = offsets / np.linalg.norm(offsets, axis=1, keepdims=True)  # [H, d]
+    err = x - ref
+    along = np.einsum("hfd,hd->hf", err, mh)
+    perp = err - along[..., None] * mh[:, None, :]
+    rn = float(np.linalg.norm(ref))
+    kappa = float(np.linalg.norm(offsets, axis=1).max() / x0_rms)
+    tol = F32_REL_L2 if dtype == "f32" else BF16_REL_L2
+    r_perp = float(np.linalg.norm(perp)) / rn
+    r_along = float(np.linalg.norm(along)) / rn
+    assert np.all(np.isfinite(x)), f"{what}: non-finite values"
+    assert r_perp <= tol, f"{what}: orthogonal part rel L2 {r_perp:.3e} > {tol}"
+    if dtype != "f32":
+        m = float(np.abs(perp).max()) / scale
+        assert m <= BF16_MAX_ABS, f"{what}: orthogonal part max-abs {m:.3e} > {BF16_MAX_ABS}"
+    assert r_along <= tol * kappa, (
+        f"{what}: part along the offset rel L2 {r_along:.3e} > {tol} x kappa {kappa:.1f}")
+    return r_perp, r_along, kappa
