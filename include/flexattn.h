@@ -119,15 +119,18 @@ int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, cons
  * must not call cudaMalloc/cudaFree, which can synchronise the device.  (The paper has
  * no counterpart; this is a convenience of this library.)
  * Same arguments, layouts and results as flex_linattn_bwd without the norm prefactor,
- * minus tau, dtau, ws and ws_bytes.  The
- * scratch is one array of 4 MiB (2^20 floats) in the library's own device memory, which
- * every GPU that loads the library keeps until the process exits; it must hold
- * B * H * (Mc * d + 1) floats (Mc = M, or 2M when W2 is given), else FLEX_EWORKSPACE is
- * returned and nothing runs.  Nothing is allocated or freed.  All calls on a device
+ * minus tau, dtau, ws and ws_bytes.  It always runs the fp32 CUDA-core backward (two
+ * kernels), never the tensor-core one, so for bf16 storage its results agree with
+ * flex_linattn_bwd's within the bf16 tolerance rather than bit for bit, and its speed
+ * differs.  The scratch is one array of 4 MiB (2^20 floats) in the library's own device
+ * memory, which every GPU that loads the library keeps until the process exits; it must
+ * hold B * H * (Mc * d + 1) floats (Mc = M, or 2M when W2 is given), else FLEX_EWORKSPACE
+ * is returned and nothing runs.  Nothing is allocated or freed.  All calls on a device
  * share that array and it keeps the last call's contents, so two calls whose work may
  * overlap on the GPU (different streams, or different host threads) race and must be
- * ordered by the caller.  The first call on each device looks the array's address up
- * (with that device current); make that first call before any stream capture. */
+ * ordered by the caller.  The first call on a device (and the first after its context
+ * was replaced, e.g. by cudaDeviceReset) looks the array's address up with that device
+ * current; make that first call before any stream capture. */
 int flex_linattn_bwd_noalloc(const flex_shape* shape, const void* q, const void* k,
                              const void* v, const float* W1, const float* W2, int causal,
                              const void* out, const float* den, const void* dout, void* dq,
@@ -213,6 +216,18 @@ unsigned long long flex_kernel_launches(void);
  * on a bounded wait since the workspace was last checked, FLEX_ECUDA on a pending CUDA
  * error, else FLEX_OK.  Clears the recorded status. */
 int flex_check_status(void* ws, void* stream);
+
+/* Diagnostic of the bounded waits (the paper has no counterpart).  Enqueues on `stream`
+ * a write of `cycles` into the header of workspace `ws` (ws_bytes >= 256).  While it is
+ * nonzero, every CTA of the causal tensor-core forward (flex_linattn_fwd with causal = 1,
+ * bf16, d = 64, M in {64, 128}) first waits at most `cycles` clocks, during its set-up and
+ * before it issues any copy or tensor-core operation, on an mbarrier that nothing arrives
+ * on; the wait runs out as a wait for a lost arrival would (FLEX_ETIMEOUT recorded in
+ * `ws`, reported by flex_check_status), the CTA frees its tensor memory and exits, and
+ * `out`/`den` are left unwritten.  flex_debug_stall(ws, ws_bytes, 0, stream) restores
+ * normal operation.  Other entry points ignore the value.  Errors: FLEX_EINVAL (NULL or
+ * misaligned ws, cycles < 0), FLEX_EWORKSPACE, FLEX_ECUDA. */
+int flex_debug_stall(void* ws, size_t ws_bytes, int cycles, void* stream);
 
 #ifdef __cplusplus
 }

@@ -72,6 +72,8 @@ int count(int n, cudaError_t e)
 
 }  // namespace
 
+void flex::add_launches(int n) { g_launches += (unsigned long long)n; }
+
 extern "C" {
 
 const char* flex_strerror(int status)
@@ -296,6 +298,18 @@ int flex_awd_loss_bwd(const flex_shape* shape, const void* q, const void* k, con
 }
 
 unsigned long long flex_kernel_launches(void) { return g_launches.load(); }
+
+int flex_debug_stall(void* ws, size_t ws_bytes, int cycles, void* stream)
+{
+    if (!ws || !aligned(ws, 256) || cycles < 0) return FLEX_EINVAL;
+    if (ws_bytes < header_bytes()) return FLEX_EWORKSPACE;
+    // from pageable host memory: the value is staged before the call returns
+    int* word = (int*)ws + flex::kStallWord;
+    return cudaMemcpyAsync(word, &cycles, sizeof(int), cudaMemcpyHostToDevice,
+                           (cudaStream_t)stream) == cudaSuccess
+               ? FLEX_OK
+               : FLEX_ECUDA;
+}
 
 int flex_check_status(void* ws, void* stream)
 {

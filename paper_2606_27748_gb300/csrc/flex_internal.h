@@ -16,9 +16,14 @@ struct WsHeader {
     int status;          // FLEX_OK or FLEX_ETIMEOUT, set by kernels, cleared by check
     int timeout_where;   // diagnostic: which wait gave up
     unsigned int ticket; // dynamic work counter of persistent kernels
-    unsigned int pad[61];
+    int stall_cycles;    // diagnostic (flex_debug_stall): 0, or the limit of a wait that
+                         // nothing ends, taken by the causal forward before any work
+    unsigned int pad[60];
 };
 static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
+// Kernels receive &header.status; the stall limit is the fourth int of the header.
+constexpr int kStallWord = 3;
+static_assert(offsetof(WsHeader, stall_cycles) == kStallWord * sizeof(int), "header layout");
 
 struct Problem {
     int B, H, N, d, M;
@@ -28,6 +33,9 @@ struct Problem {
 };
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Adds n to the count of kernels enqueued by the library (flex_kernel_launches).
+void add_launches(int n);
 
 // ---- SIMT path (fp32 arithmetic; any supported dtype) --------------------------------
 size_t simt_fwd_smem_bytes(const Problem& p, int chunk);

@@ -527,8 +527,10 @@ __global__ void __launch_bounds__(kThreadsG, 1)
             tmem_ld16(tm_row + L::T_S + 16 * qd, u);
             if (NS) tmem_ld16(tm_row + L::T_S + 64 + 16 * qd, w);
             tmem_wait_ld();
-            reduce_2pi_if_needed(u);
-            if (NS) reduce_2pi_if_needed(w);
+            if (NS)
+                reduce_2pi_if_needed(u, w);
+            else
+                reduce_2pi_if_needed(u);
             uint32_t o1[8], o2[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) {

@@ -220,8 +220,10 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             tmem_ld16(tm_row + tcol + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
         }
         tmem_wait_ld();
-        reduce_2pi_if_needed(a);
-        if (NS) reduce_2pi_if_needed(w);
+        if (NS)
+            reduce_2pi_if_needed(a, w);
+        else
+            reduce_2pi_if_needed(a);
         uint32_t pc[16], ps[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
@@ -263,10 +265,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             tmem_ld16(tm_row + L::T_P + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
         }
         tmem_wait_ld();
-        if (NS) {
-            reduce_2pi_if_needed(a);
-            reduce_2pi_if_needed(w);
-        }
+        if (NS) reduce_2pi_if_needed(a, w);
         uint32_t cpair[16], spair[16];  // s: this thread's cos / sin features, bf16 pairs
         if (!NS) {
 #pragma unroll

@@ -120,8 +120,10 @@ __global__ void __launch_bounds__(kThreadsF)
                 tmem_ld16(col + 80, *reinterpret_cast<float(*)[16]>(&w[16]));
             }
             tmem_wait_ld();
-            reduce_2pi_if_needed(a);
-            if (NS) reduce_2pi_if_needed(w);
+            if (NS)
+                reduce_2pi_if_needed(a, w);
+            else
+                reduce_2pi_if_needed(a);
             uint32_t pc[16], ps[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i) {

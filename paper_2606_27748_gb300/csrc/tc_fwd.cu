@@ -107,6 +107,7 @@ struct Bars {
     uint64_t p_full, p_free, phiq_full, phik_full, phiq_free, phik_free;
     uint64_t attn_done, s_done, a_ready, sx_ready, o_ready, epi_done[2];
     uint64_t xch_full[2];  // the partner's four block copies have landed in XCH (tx count)
+    uint64_t never;        // nothing arrives on it (the diagnostic stall)
 };
 
 // First chunk of segment j of `splits` (lengths proportional to 2^-j), rounded.
@@ -193,8 +194,10 @@ __global__ void __maxnreg__(96)
         mbar_init(&bars.o_ready, 1);
         mbar_init(&bars.xch_full[0], 1);
         mbar_init(&bars.xch_full[1], 1);
+        mbar_init(&bars.never, 1);
         abort_flag = 0;
         fence_mbar_init();
+        diagnostic_stall(&bars.never, &abort_flag, status);  // normally returns at once
         if (CS > 1) {  // the first exchange into each buffer
             mbar_arrive_expect_tx(&bars.xch_full[0], L::XBUF);
             mbar_arrive_expect_tx(&bars.xch_full[1], L::XBUF);
@@ -213,7 +216,9 @@ __global__ void __maxnreg__(96)
     fence_after_sync();
     const uint32_t tm = tmem_base_sh;
 
-    if (warp == kWarpTMAV) {
+    if (abort_flag) {
+        // the diagnostic stall ran out during set-up: nothing is issued
+    } else if (warp == kWarpTMAV) {
         // ================= TMA producer: v =================
         if (lane == 0) {
             uint32_t ph_vfree[2] = {0, 0};
@@ -397,8 +402,10 @@ __global__ void __maxnreg__(96)
                         __syncwarp();
                         if (lane == 0) mbar_arrive(&bars.p_free);
                     }
-                    reduce_2pi_if_needed(a);
-                    if (NS) reduce_2pi_if_needed(w);
+                    if (NS)
+                        reduce_2pi_if_needed(a, w);
+                    else
+                        reduce_2pi_if_needed(a);
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
                         float s0, c0, s1, c1;

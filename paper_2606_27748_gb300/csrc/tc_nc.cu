@@ -268,8 +268,10 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
             fence_before_sync();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars.p_free[pb]);
-            reduce_2pi_if_needed(a);
-            if (NS) reduce_2pi_if_needed(w);
+            if (NS)
+                reduce_2pi_if_needed(a, w);
+            else
+                reduce_2pi_if_needed(a);
             uint32_t pc[16], ps[16];
 #pragma unroll
             for (int e = 0; e < 16; ++e) {

@@ -48,37 +48,77 @@ __device__ __forceinline__ float reduce_2pi(float x)
     return fmaf(-n, k2PiLo, fmaf(-n, k2PiHi, x));
 }
 
-// Reduces every value of v when any lane of the warp holds one beyond [-pi, pi]; the test
-// costs one max per value, so inputs inside the range (the common case) skip the step.
-// Warp-collective: all 32 lanes call it together.
+// OR of the bit patterns of v, as a balanced tree (the compiler fuses pairs of ORs into
+// three-input logic ops: about n/2 instructions, depth log2 n).  Bit 30 of an fp32 value
+// is the top bit of its exponent field: set exactly when |x| >= 2 (or x is not finite).
 template <int n>
-__device__ __forceinline__ void reduce_2pi_if_needed(float (&v)[n])
+__device__ __forceinline__ uint32_t or_bits(const float (&v)[n])
 {
-    float m = 0.f;
+    uint32_t acc[n];
 #pragma unroll
-    for (int i = 0; i < n; ++i) m = fmaxf(m, fabsf(v[i]));
-    if (__any_sync(0xffffffffu, m > kPi)) {
+    for (int i = 0; i < n; ++i) acc[i] = __float_as_uint(v[i]);
 #pragma unroll
-        for (int i = 0; i < n; ++i) v[i] = reduce_2pi(v[i]);
+    for (int s = 1; s < n; s *= 2)
+#pragma unroll
+        for (int i = 0; i + s < n; i += 2 * s) acc[i] |= acc[i + s];
+    return acc[0];
+}
+constexpr uint32_t kAbsGE2 = 0x40000000u;
+
+template <int n>
+__device__ __forceinline__ void reduce_2pi_all(float (&v)[n])
+{
+#pragma unroll
+    for (int i = 0; i < n; ++i) v[i] = reduce_2pi(v[i]);
+}
+
+// Reduces every value of a (and of w) when any lane of the warp holds one with |x| >= 2:
+// inside [-2, 2] (a subset of [-pi, pi], where the hardware sin/cos keeps its 2^-21
+// bound) the step is skipped, for about half an instruction per value.  Warp-collective:
+// all 32 lanes call it together.
+template <int n>
+__device__ __forceinline__ void reduce_2pi_if_needed(float (&a)[n])
+{
+    if (__any_sync(0xffffffffu, or_bits(a) & kAbsGE2)) reduce_2pi_all(a);
+}
+template <int n>
+__device__ __forceinline__ void reduce_2pi_if_needed(float (&a)[n], float (&w)[n])
+{
+    if (__any_sync(0xffffffffu, (or_bits(a) | or_bits(w)) & kAbsGE2)) {
+        reduce_2pi_all(a);
+        reduce_2pi_all(w);
     }
 }
 
 // Bounded wait on one mbarrier phase.  On a time-out the CTA is told to stop (abort flag)
 // and the status word (if any) records FLEX_ETIMEOUT; every other wait then returns at once.
 __device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                         int* status)
+                                         int* status, long long limit = kWaitCycles)
 {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     while (true) {
         if (mbar_try_wait(bar, parity)) return true;
         if (*abort_flag) return false;
-        if (clock64() - t0 > kWaitCycles) {
+        if (clock64() - t0 > limit) {
             *abort_flag = 1;
             if (status) atomicExch(status, (int)FLEX_ETIMEOUT);
             return false;
         }
     }
+}
+
+// The diagnostic stall of flex_debug_stall: when the workspace header asks for it
+// (stall_cycles > 0), one thread of the CTA waits that many clocks at most on `bar`, an
+// mbarrier that nothing arrives on, so the wait runs out exactly as a wait for a lost
+// arrival would: the abort flag is set and the status word records FLEX_ETIMEOUT.  Called
+// during set-up, before anything is issued; the kernel then issues nothing and exits.
+__device__ __forceinline__ void diagnostic_stall(uint64_t* bar, volatile int* abort_flag,
+                                                 int* status)
+{
+    if (!status) return;
+    const int cycles = *reinterpret_cast<volatile int*>(status + kStallWord);
+    if (cycles > 0) bar_wait(bar, 0, abort_flag, status, cycles);
 }
 
 // bar_wait for a barrier that other CTAs of the cluster arrive on (acquire at cluster scope).

@@ -23,7 +23,8 @@ FLEX_OK, FLEX_EINVAL, FLEX_EUNSUPPORTED, FLEX_EWORKSPACE, FLEX_ECUDA, FLEX_ETIME
 EXPORTS = ("flex_strerror", "flex_workspace_bytes", "flex_featmap", "flex_linattn_fwd",
            "flex_linattn_bwd", "flex_decode_workspace_bytes", "flex_linattn_decode",
            "flex_awd_workspace_bytes", "flex_awd_loss", "flex_awd_bwd_workspace_bytes",
-           "flex_awd_loss_bwd", "flex_kernel_launches", "flex_check_status")
+           "flex_awd_loss_bwd", "flex_kernel_launches", "flex_check_status",
+           "flex_debug_stall")
 
 
 class FlexShape(ctypes.Structure):
@@ -73,11 +74,12 @@ def load(path: str = LIBRARY) -> ctypes.CDLL:
         lib.flex_awd_loss_bwd.argtypes = [shp, vp, vp, vp, vp, vp, ip, vp, vp, vp, vp, vp, vp,
                                           sz, vp]
         lib.flex_check_status.argtypes = [vp, vp]
+        lib.flex_debug_stall.argtypes = [vp, sz, ip, vp]
         lib.flex_kernel_launches.argtypes = []
         lib.flex_kernel_launches.restype = ctypes.c_ulonglong
         for fn in (lib.flex_featmap, lib.flex_linattn_fwd, lib.flex_linattn_bwd,
                    lib.flex_linattn_decode, lib.flex_awd_loss, lib.flex_awd_loss_bwd,
-                   lib.flex_check_status):
+                   lib.flex_check_status, lib.flex_debug_stall):
             fn.restype = ip
         _lib = lib
         return lib
@@ -283,3 +285,11 @@ def awd_loss_bwd(q, k, W1, W2=None, causal=False, tau=None, dloss=None, loss=Non
 def check_status(ws, stream=None):
     """Synchronise and raise if a kernel that used `ws` gave up on a bounded wait."""
     _check(load().flex_check_status(_ptr(ws), _stream(stream)), "flex_check_status")
+
+
+def debug_stall(ws, cycles: int, stream=None):
+    """Diagnostic of the bounded waits: while `cycles` > 0, the causal tensor-core forward
+    run with workspace `ws` gives up after a wait of at most `cycles` clocks that nothing
+    ends, before doing any work (FLEX_ETIMEOUT through check_status).  0 restores it."""
+    _check(load().flex_debug_stall(_ptr(ws), ws.numel(), int(cycles), _stream(stream)),
+           "flex_debug_stall")

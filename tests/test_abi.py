@@ -156,3 +156,12 @@ def test_awd_bwd_host_validation_without_gpu(lib):
              None) == FLEX_EWORKSPACE
     assert f(ctypes.byref(ok), p, p, p, None, None, 0, p, p, ctypes.c_void_p(4100), None, None,
              p, need, None) == FLEX_EINVAL                          # misaligned dW1
+
+
+def test_debug_stall_validation_without_gpu(lib):
+    from paper_2606_27748_gb300.flexattn import FLEX_EINVAL, FLEX_EWORKSPACE
+    p = ctypes.c_void_p(4096)  # 256-byte aligned, never dereferenced: validation fails first
+    assert lib.flex_debug_stall(None, 256, 1000, None) == FLEX_EINVAL
+    assert lib.flex_debug_stall(ctypes.c_void_p(4100), 256, 1000, None) == FLEX_EINVAL
+    assert lib.flex_debug_stall(p, 256, -1, None) == FLEX_EINVAL
+    assert lib.flex_debug_stall(p, 255, 1000, None) == FLEX_EWORKSPACE
