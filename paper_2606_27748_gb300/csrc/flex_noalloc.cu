@@ -3,8 +3,9 @@
 //
 // It always runs the fp32 CUDA-core (SIMT) backward, whose only scratch is the
 // per-sequence partial frequency gradients (B * H * (Mc * d + 1) floats, Mc = M or 2M)
-// before they are summed over the batch; the tensor-core backward's scratch (fp32 dq, dk,
-// dv accumulators) grows with N and does not fit a fixed array.  Here that scratch is a
+// before they are summed over the batch; the tensor-core backward's scratch (dW partials
+// of 128 rows per frequency group, pass and sequence, plus key weights growing with N) is
+// several times larger.  Here that scratch is a
 // fixed array in the library's own device memory instead, so nothing is allocated per
 // call: every GPU that loads the library holds the array (4 MiB) until the process exits.
 #include <cuda.h>

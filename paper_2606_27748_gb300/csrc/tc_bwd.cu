@@ -11,12 +11,15 @@
 // phi_non) by the chain rule: dx = da W, dW += da^T x.
 //
 // Every term splits over feature groups (64 frequencies = 128 features), and A enters dv
-// linearly, so one CTA handles one (sequence, group) pair and the group results are summed:
-// dq, dk, dv by fp32 adds onto zeroed accumulators (at most two groups, so the sum does not
-// depend on the order), dW through per-(pass, sequence, group) partials reduced over the
-// batch in a fixed order.  Pass F runs the chunks forward (dq and the q part of dW, state
-// S, z), pass R runs them backward (dk, dv and the k part of dW, state R, r); the two are
-// independent and run as the two halves of one grid.
+// linearly, so one CTA handles one (sequence, group) pair and the group results are summed.
+// With two groups (M = 128) the two CTAs of a (pass, sequence) form a cluster: each chunk,
+// CTA r finishes rows 64r..64r+63 of dq (pass F) or dk and dv (pass R): it sends its
+// fp32 partial rows of the other half to the partner (staged in its own shared memory, one
+// bulk copy into a region the partner has declared free), adds the partner's partial to its
+// own rows and stores bf16.  dW goes through per-(pass, sequence, group) partials reduced
+// over the batch in a fixed order.  Pass F runs the chunks forward (dq and the q part of
+// dW, state S, z), pass R runs them backward (dk, dv and the k part of dW, state R, r); the
+// two are independent and run as the two halves of one grid, pass R (the longer) first.
 //
 // Norm prefactor (Sec. 3.2, optional): with key weights w_j = exp(|k_j|^2 exp(-tau)) (kw,
 // one pass over k before this kernel), phi(k) is stored weighted, so S, z, A and dv come
@@ -28,6 +31,11 @@
 //
 // Phases are serialised: all 256 threads load, compute features and run the CUDA-core
 // epilogues; thread 0 issues the MMAs; one mbarrier tracks their completion (bounded waits).
+//
+// Exchange regions (per chunk; each freed by this CTA before it tells the partner "ready"):
+// pass F receives dq in DO (free once g is built) and stages in PQ (free after the
+// projection backward); pass R receives dv in DO and dk in O (bf16 A, free after the
+// gradient MMAs) and stages dv in Q and dk in DA2 (bf16 dA, free at the same point).
 //
 // Tensor memory (512 columns): [0,128) projection, [128,256) A / dA (bf16 in place) then
 // dx (0-63) and the chunk's dW (64-127), [256,384) dphi, [384,464) S|z or R|r.
@@ -43,6 +51,7 @@ using namespace tc;
 
 constexpr int kC = 128;
 constexpr int kThreadsB = 256;
+constexpr uint32_t kXBytes = 64 * 64 * 4;  // one exchanged half: 64 rows x 64 fp32
 enum { kPassF = 0, kPassR = 1 };
 
 template <bool NS>
@@ -64,20 +73,14 @@ struct BwCfg {
 };
 
 
-__device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d)
-{
-    asm volatile("red.global.add.v4.f32 [%0], {%1,%2,%3,%4};" ::"l"(addr), "f"(a), "f"(b),
-                 "f"(c), "f"(d)
-                 : "memory");
-}
-
 __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes)
 {
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
-// KW: key weights of the norm prefactor given (compile-time; the plain kernel is unchanged)
-template <bool NS, bool KW>
+// KW: key weights of the norm prefactor given (compile-time; the plain kernel is unchanged);
+// CS: CTAs per cluster = frequency groups (1 or 2)
+template <bool NS, bool KW, int CS>
 __global__ void __launch_bounds__(kThreadsB, 1)
     tc_bwd_kernel(const __grid_constant__ CUtensorMap tmap_q,
                   const __grid_constant__ CUtensorMap tmap_k,
@@ -88,21 +91,28 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                   const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __restrict__ v,
                   const float* __restrict__ W1, const float* __restrict__ W2,
                   const __nv_bfloat16* __restrict__ outp, const float* __restrict__ den,
-                  const __nv_bfloat16* __restrict__ dout, float* __restrict__ acc_q,
-                  float* __restrict__ acc_k, float* __restrict__ acc_v, float* __restrict__ dw_part,
+                  const __nv_bfloat16* __restrict__ dout, __nv_bfloat16* __restrict__ dq,
+                  __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv,
+                  float* __restrict__ dw_part,
                   const float* __restrict__ kw, const float* __restrict__ tau,
                   float* __restrict__ dtau_part, int units, int* status)
 {
     using L = BwCfg<NS>;
-    // blocks [0, units): pass F, [units, 2 units): pass R; unit = (sequence, group)
-    const int PASS = (int)blockIdx.x >= units ? kPassR : kPassF;
+    // blocks [0, units): pass R, [units, 2 units): pass F; unit = (sequence, group); partial
+    // slots are indexed by slot = pass * units + unit
+    const int PASS = (int)blockIdx.x < units ? kPassR : kPassF;
     const int unit = (int)blockIdx.x % units;
-    float* const acc_x = PASS == kPassF ? acc_q : acc_k;
+    const int slot = PASS * units + unit;
+    __nv_bfloat16* const dx_out = PASS == kPassF ? dq : dk;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const uint32_t sb = smem_u32(sm);
     __shared__ uint32_t tmem_base_sh;
     __shared__ __align__(8) uint64_t mbar, tma_bar;
+    // cluster exchange: xready: the partner's receive regions are free; xdone: the partner
+    // has read what this CTA sent (so the staging region may be rewritten); xfull[0]: dq (F)
+    // or dv (R) partial landed, xfull[1]: dk (R) (transaction counts)
+    __shared__ __align__(8) uint64_t xready, xdone, xfull[2];
     __shared__ volatile int abort_flag;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -138,11 +148,20 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         st_shared_v4(sb + L::C16 + idx * 16, fill, fill, fill, fill);
     }
     for (int idx = tid; idx < 128; idx += kThreadsB) zr[idx] = 0.f;
+    const int rank = CS > 1 ? (int)cluster_rank() : 0;  // = g
     if (tid == 0) {
         mbar_init(&mbar, 1);
         mbar_init(&tma_bar, 1);
+        mbar_init(&xready, 1);
+        mbar_init(&xdone, 1);
+        mbar_init(&xfull[0], 1);
+        mbar_init(&xfull[1], 1);
         abort_flag = 0;
         fence_mbar_init();
+        if (CS > 1) {  // the first chunk's exchanges
+            mbar_arrive_expect_tx(&xfull[0], kXBytes);
+            if (PASS == kPassR) mbar_arrive_expect_tx(&xfull[1], kXBytes);
+        }
     }
     if (warp == 0) {
         tmem_alloc(&tmem_base_sh, 512);
@@ -150,11 +169,15 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     }
     fence_proxy_async();
     fence_before_sync();
-    __syncthreads();
+    if (CS > 1)
+        cluster_sync();  // the partner's barriers exist before anything arrives on them
+    else
+        __syncthreads();
     fence_after_sync();
     const uint32_t tm = tmem_base_sh;
     const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
-    uint32_t phase = 0, tma_phase = 0;
+    uint32_t phase = 0, tma_phase = 0, ph_xready = 0, ph_xdone = 0, ph_xfull[2] = {0, 0};
+    const uint32_t partner = (uint32_t)rank ^ 1u;
 
     auto handoff = [&]() {
         fence_proxy_async();
@@ -352,8 +375,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             tmem_ld16(tm_row + T_DW + 16 * j, *reinterpret_cast<float(*)[16]>(&v_[16 * j]));
         tmem_wait_ld();
         if (t < L::P && wg == 1) {
-            float4* dst = reinterpret_cast<float4*>(dw_part + ((size_t)blockIdx.x * 128 + t) * 64);
-            // slot blockIdx.x = pass * units + unit
+            float4* dst = reinterpret_cast<float4*>(dw_part + ((size_t)slot * 128 + t) * 64);
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
                 float4 old = first ? make_float4(0.f, 0.f, 0.f, 0.f) : dst[j];
@@ -376,9 +398,33 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                          pack_bf16(s_[8 * j + 4], s_[8 * j + 5]), pack_bf16(s_[8 * j + 6], s_[8 * j + 7]));
         if (wg == 0) zr[t] = zz[0];
     };
-    // rows of a [128 x 64] TMEM block (T_A[0,64)) added into an fp32 [token][64] accumulator
-    // kcoef != 0: + kcoef * k_t (the prefactor's dk term; k row from the K tile)
-    auto add_rows = [&](float* acc, int t0, bool valid, float kcoef) {
+    // ---- cluster exchange of the dq / dk / dv partials (CS = 2) ----
+    // This CTA's receive regions for the chunk are free: tell the partner (all threads are
+    // past their last use of them).
+    auto signal_ready = [&]() {
+        if (CS > 1 && tid == 0) mbar_arrive_cluster(mapa(smem_u32(&xready), partner));
+    };
+    // Before the staging region is rewritten: the partner has read the previous chunk's data.
+    auto wait_done = [&](bool any_sent) -> bool {
+        bool ok = true;
+        if (CS > 1 && any_sent && tid == 0) {
+            ok = bar_wait_cluster(&xdone, ph_xdone, &abort_flag, status);
+            ph_xdone ^= 1;
+        }
+        ok = !__syncthreads_or(!ok);
+        return ok;
+    };
+    // Byte offset of 16-byte chunk j (0-7) of this thread's half row in a 64 x 64 fp32
+    // exchange block (256-byte rows, chunks swizzled by row: conflict-free float4 access).
+    auto xoff = [&](uint32_t rr, int j) {
+        return rr * 256u + ((((uint32_t)(8 * wg + j)) ^ (rr & 7u)) << 4);
+    };
+    // Rows of a [128 x 64] TMEM block (T_A[0,64)) -> bf16 rows of `out` for the chunk at t0.
+    // kcoef != 0: + kcoef * k_t (the prefactor's dk term; k row from the K tile).  With a
+    // partner: this CTA stores rows 64 rank .. + 63, adding the partner's partial (exchange
+    // xi: staged at `stage`, received at `recv`); the other rows are sent.
+    auto finish_rows = [&](__nv_bfloat16* out, int t0, bool valid, float kcoef, int xi,
+                           uint32_t stage, uint32_t recv, bool last_of_chunk) -> bool {
         float v_[32];
         tmem_ld16(tm_row + L::T_A + 32 * wg, *reinterpret_cast<float(*)[16]>(&v_[0]));
         tmem_ld16(tm_row + L::T_A + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&v_[16]));
@@ -396,12 +442,60 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 }
             }
         }
-        if (valid) {
-            float* dst = acc + base + (size_t)(t0 + t) * 64 + 32 * wg;
+        bool ok = true;
+        const uint32_t rr = (uint32_t)t & 63u;
+        const bool own = CS == 1 || (t >> 6) == rank;
+        if (CS > 1) {
+            if (!own) {
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
-                red_add_v4(dst + 4 * j, v_[4 * j], v_[4 * j + 1], v_[4 * j + 2], v_[4 * j + 3]);
+                for (int j = 0; j < 8; ++j)
+                    st_shared_v4(stage + xoff(rr, j), __float_as_uint(v_[4 * j]),
+                                 __float_as_uint(v_[4 * j + 1]), __float_as_uint(v_[4 * j + 2]),
+                                 __float_as_uint(v_[4 * j + 3]));
+            }
+            fence_proxy_async();  // the staged rows, visible to the bulk copy
+            __syncthreads();
+            if (tid == 0) {
+                if (xi == 0) {  // one "ready" per chunk covers its exchanges
+                    ok = bar_wait_cluster(&xready, ph_xready, &abort_flag, status);
+                    ph_xready ^= 1;
+                }
+                if (ok)
+                    bulk_copy_cluster(mapa(recv, partner), stage, kXBytes,
+                                      mapa(smem_u32(&xfull[xi]), partner));
+            }
+            if (own) {
+                ok = ok && bar_wait(&xfull[xi], ph_xfull[xi], &abort_flag, status);
+                if (ok) {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const float4 p4 = *reinterpret_cast<const float4*>(sm + (recv - sb) + xoff(rr, j));
+                        v_[4 * j] += p4.x;
+                        v_[4 * j + 1] += p4.y;
+                        v_[4 * j + 2] += p4.z;
+                        v_[4 * j + 3] += p4.w;
+                    }
+                }
+            }
+            ph_xfull[xi] ^= 1;
         }
+        if (own && valid && ok) {
+            uint4* dst = reinterpret_cast<uint4*>(out + base + (size_t)(t0 + t) * 64 + 32 * wg);
+#pragma unroll
+            for (int cc = 0; cc < 4; ++cc)
+                dst[cc] = make_uint4(pack_bf16(v_[8 * cc], v_[8 * cc + 1]),
+                                     pack_bf16(v_[8 * cc + 2], v_[8 * cc + 3]),
+                                     pack_bf16(v_[8 * cc + 4], v_[8 * cc + 5]),
+                                     pack_bf16(v_[8 * cc + 6], v_[8 * cc + 7]));
+        }
+        ok = !__syncthreads_or(!ok);
+        if (CS > 1 && ok && tid == 0) {
+            // the next chunk's exchange of this kind; after the last one of the chunk the
+            // partner may reuse its staging region
+            mbar_arrive_expect_tx(&xfull[xi], kXBytes);
+            if (last_of_chunk) mbar_arrive_cluster(mapa(smem_u32(&xdone), partner));
+        }
+        return ok;
     };
 
     const int nch = (N + kC - 1) / kC;
@@ -475,8 +569,11 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                     __float2bfloat16_rn(cval);
         }
         handoff();
+        if (PASS == kPassF) signal_ready();  // DO is free for the partner's dq partial
         // ---- features of q and k for this group ----
         if (!project_qk()) goto done;
+        // the partner has read the previous chunk's exchange data staged in PQ
+        if (CS > 1 && !wait_done(it > 0)) goto done;
         features(sb + L::PQ, L::T_P, valid, 1.f);
         features(sb + L::PK, L::T_A, valid, wk);
         handoff();
@@ -535,7 +632,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             feature_backward(sb + L::PQ, crow[t], valid, 1.f);
             handoff();
             if (!project_back(dPQ, dPQmn, dQmn, it == 0)) goto done;
-            add_rows(acc_x, t0, valid, 0.f);
+            if (!finish_rows(dx_out, t0, valid, 0.f, 0, sb + L::PQ, sb + L::DO, true)) goto done;
             if (NS) dw_accumulate(it == 0);
             snapshot();
             handoff();
@@ -612,7 +709,9 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 }
             }
             if (!commit_wait()) goto done;
-            add_rows(acc_v, t0, valid, 0.f);  // dv of this group
+            signal_ready();  // DO, O are free for the partner's dv, dk partials
+            // dv of this group
+            if (!finish_rows(dv, t0, valid, 0.f, 0, sb + L::PQ, sb + L::DO, false)) goto done;
             fence_before_sync();
             __syncthreads();
             if (NS && !project(dK)) goto done;  // u, w of k for the chain rule
@@ -625,7 +724,9 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             }
             handoff();
             if (!project_back(dPK, dPKmn, dKmn, it == 0)) goto done;
-            add_rows(acc_x, t0, valid, KW ? 2.f * itau * (spart[t] + spart[128 + t]) : 0.f);
+            if (!finish_rows(dx_out, t0, valid, KW ? 2.f * itau * (spart[t] + spart[128 + t]) : 0.f,
+                             1, sb + L::PQ + 16384, sb + L::O, true))
+                goto done;
             if (NS) dw_accumulate(it == 0);
             snapshot();
             handoff();
@@ -640,7 +741,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         if (tid == 0) {
             float sum = 0.f;
             for (int w8 = 0; w8 < kThreadsB / 32; ++w8) sum += spart[w8];
-            dtau_part[blockIdx.x] = sum;
+            dtau_part[slot] = sum;
         }
     }
 done:
@@ -648,6 +749,7 @@ done:
     __syncthreads();
     fence_after_sync();
     if (warp == 0) tmem_dealloc(tm, 512);
+    if (CS > 1) cluster_sync();  // no CTA leaves while its partner may still copy into it
 }
 
 // dW over the batch in a fixed order.  Partial slots [pass][bh * G + g][row][64]; s: rows
@@ -687,18 +789,6 @@ __global__ void tc_dw_reduce_kernel(int B, int H, int M, int G, int nonstat,
     }
 }
 
-__global__ void tc_to_bf16_kernel(size_t n, const float* __restrict__ a, const float* __restrict__ b,
-                                  const float* __restrict__ c, __nv_bfloat16* __restrict__ oa,
-                                  __nv_bfloat16* __restrict__ ob, __nv_bfloat16* __restrict__ oc)
-{
-    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
-         i += (size_t)gridDim.x * blockDim.x) {
-        oa[i] = __float2bfloat16_rn(a[i]);
-        ob[i] = __float2bfloat16_rn(b[i]);
-        oc[i] = __float2bfloat16_rn(c[i]);
-    }
-}
-
 template <bool NS>
 cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const void* v,
                        const float* W1, const float* W2, const float* tau, const void* out,
@@ -707,15 +797,10 @@ cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const voi
                        cudaStream_t s)
 {
     const int BH = p.B * p.H, G = p.M / 64;
-    const size_t n = (size_t)BH * p.N * 64;
-    float* acc_q = static_cast<float*>(scratch);
-    float* acc_k = acc_q + n;
-    float* acc_v = acc_k + n;
-    float* part = acc_v + n;
+    float* part = static_cast<float*>(scratch);
     float* kw = part + (size_t)2 * BH * G * 128 * 64;  // key weights [B*H*N] (prefactor)
     float* dtau_part = kw + (size_t)BH * p.N;           // [2 units]
-    cudaError_t e = cudaMemsetAsync(acc_q, 0, 3 * n * sizeof(float), s);
-    if (e != cudaSuccess) return e;
+    cudaError_t e = cudaSuccess;
     if (tau && (e = launch_key_weights(p, k, tau, kw, s)) != cudaSuccess) return e;
     const int smem = (int)BwCfg<NS>::BYTES + 1024;
     CUtensorMap mq, mk, mv, mdo, mo;
@@ -723,21 +808,31 @@ cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const voi
         !make_act_map(&mv, v, BH, p.N) || !make_act_map(&mdo, dout, BH, p.N) ||
         !make_act_map(&mo, out, BH, p.N))
         return cudaErrorInvalidValue;
-    auto kb = tau ? tc_bwd_kernel<NS, true> : tc_bwd_kernel<NS, false>;
+    auto kb = G == 2 ? (tau ? tc_bwd_kernel<NS, true, 2> : tc_bwd_kernel<NS, false, 2>)
+                     : (tau ? tc_bwd_kernel<NS, true, 1> : tc_bwd_kernel<NS, false, 1>);
     if ((e = cudaFuncSetAttribute(kb, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return e;
     typedef const __nv_bfloat16* CB;
+    typedef __nv_bfloat16* B16;
     const int units = BH * G;
-    kb<<<2 * units, kThreadsB, smem, s>>>(mq, mk, mv, mdo, mo, p.H, p.N, p.M, G, p.causal, (CB)q, (CB)k,
-                                          (CB)v, W1,
-                                          W2, (CB)out, den, (CB)dout, acc_q, acc_k, acc_v, part,
-                                          tau ? kw : nullptr, tau, dtau_part, units, status);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(2 * units));
+    cfg.blockDim = dim3(kThreadsB);
+    cfg.dynamicSmemBytes = (size_t)smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = G;  // the frequency groups of one (pass, sequence)
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, kb, mq, mk, mv, mdo, mo, p.H, p.N, p.M, G, p.causal, (CB)q,
+                           (CB)k, (CB)v, W1, W2, (CB)out, den, (CB)dout, (B16)dq, (B16)dk,
+                           (B16)dv, part, tau ? kw : nullptr, tau, dtau_part, units, status);
+    if (e != cudaSuccess) return e;
     const size_t work = (size_t)p.H * p.M * 64;
     tc_dw_reduce_kernel<<<(int)std::min<size_t>((work + 255) / 256, 152 * 8), 256, 0, s>>>(
         p.B, p.H, p.M, G, p.nonstat, part, dW1, dW2, dtau_part, tau ? dtau : nullptr);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    tc_to_bf16_kernel<<<152 * 8, 256, 0, s>>>(n, acc_q, acc_k, acc_v, (__nv_bfloat16*)dq,
-                                               (__nv_bfloat16*)dk, (__nv_bfloat16*)dv);
     return cudaGetLastError();
 }
 
@@ -750,12 +845,12 @@ bool tc_bwd_supported(const Problem& p)
     return p.bf16 && p.causal && p.d == 64 && (p.M == 64 || p.M == 128);
 }
 
-// fp32 dq/dk/dv accumulators, dW partials [2 passes][B*H*G][128][64], key weights
-// [B*H*N] and dtau partials [2 B*H*G] (norm prefactor).
+// dW partials [2 passes][B*H*G][128][64], key weights [B*H*N] and dtau partials
+// [2 B*H*G] (norm prefactor).
 size_t tc_bwd_ws_bytes(const Problem& p)
 {
     const size_t BH = (size_t)p.B * p.H, G = (size_t)p.M / 64;
-    return (3 * BH * p.N * 64 + 2 * BH * G * 128 * 64 + BH * p.N + 2 * BH * G) * sizeof(float);
+    return (2 * BH * G * 128 * 64 + BH * p.N + 2 * BH * G) * sizeof(float);
 }
 
 cudaError_t launch_tc_bwd(const Problem& p, const void* q, const void* k, const void* v,

@@ -249,6 +249,22 @@ __device__ __forceinline__ void tma_prefetch_3d(const void* tmap, int c0, int c1
                  : "memory");
 }
 
+// ---- register split between warpgroups ---------------------------------------------------
+
+// Every warp of a warpgroup executes these together; inc waits until the registers that
+// other warpgroups released (dec) are available.  The shares must add up to at most the
+// registers the CTA was launched with.
+template <uint32_t kRegs>
+__device__ __forceinline__ void setmaxnreg_inc()
+{
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegs));
+}
+template <uint32_t kRegs>
+__device__ __forceinline__ void setmaxnreg_dec()
+{
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegs));
+}
+
 // ---- thread-block clusters ---------------------------------------------------------------
 
 __device__ __forceinline__ uint32_t cluster_rank()

@@ -402,17 +402,27 @@ __global__ void __maxnreg__(96)
                         __syncwarp();
                         if (lane == 0) mbar_arrive(&bars.p_free);
                     }
-                    if (NS)
-                        reduce_2pi_if_needed(a, w);
-                    else
+                    if (NS) {
+                        // w <- cos(w): on the FMA pipe (polynomial) when every argument of
+                        // the warp is inside [-2, 2], else reduced + hardware cos
+                        if (__any_sync(0xffffffffu, (or_bits(a) | or_bits(w)) & kAbsGE2)) {
+                            reduce_2pi_all(a);
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) w[i] = __cosf(reduce_2pi(w[i]));
+                        } else {
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) cos_poly2(w[2 * i], w[2 * i + 1]);
+                        }
+                    } else {
                         reduce_2pi_if_needed(a);
+                    }
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
                         float s0, c0, s1, c1;
                         __sincosf(a[2 * i], &s0, &c0);
                         __sincosf(a[2 * i + 1], &s1, &c1);
                         if (NS) {
-                            const float cw0 = __cosf(w[2 * i]), cw1 = __cosf(w[2 * i + 1]);
+                            const float cw0 = w[2 * i], cw1 = w[2 * i + 1];
                             c0 *= cw0; s0 *= cw0; c1 *= cw1; s1 *= cw1;
                         }
                         if (KW && which == 1) { c0 *= wk; s0 *= wk; c1 *= wk; s1 *= wk; }

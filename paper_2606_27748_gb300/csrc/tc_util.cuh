@@ -90,6 +90,48 @@ __device__ __forceinline__ void reduce_2pi_if_needed(float (&a)[n], float (&w)[n
     }
 }
 
+// ---- packed f32x2 arithmetic (two fp32 lanes in one 64-bit register) --------------------
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi)
+{
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi)
+{
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b)
+{
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c)
+{
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+
+// cos(x) for |x| <= 2 on the FMA pipe: p(x^2) with p of degree 4, fitted here to
+// cos(sqrt(y)) on y in [0, 4] by least squares on 4000 Chebyshev nodes refined by Lawson's
+// iteratively reweighted least squares (an approximation to the minimax polynomial);
+// max error with fp32 evaluation 6.6e-7 over [-2, 2] (the hardware cos: 4e-7 on
+// [-pi, pi]).  Two values per call, one packed multiply and four packed fmas.
+__device__ __forceinline__ void cos_poly2(float& x0, float& x1)
+{
+    constexpr float C0 = 0.9999995231628418f, C1 = -0.4999936819076538f,
+                    C2 = 0.04165392369031906f, C3 = -0.0013798808213323355f,
+                    C4 = 2.2181484382599592e-05f;
+    const uint64_t x = f2_pack(x0, x1), y = f2_mul(x, x);
+    uint64_t p = f2_fma(f2_pack(C4, C4), y, f2_pack(C3, C3));
+    p = f2_fma(p, y, f2_pack(C2, C2));
+    p = f2_fma(p, y, f2_pack(C1, C1));
+    p = f2_fma(p, y, f2_pack(C0, C0));
+    f2_unpack(p, x0, x1);
+}
+
 // Bounded wait on one mbarrier phase.  On a time-out the CTA is told to stop (abort flag)
 // and the status word (if any) records FLEX_ETIMEOUT; every other wait then returns at once.
 __device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
