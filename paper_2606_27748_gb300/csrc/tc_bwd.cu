@@ -419,12 +419,15 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     auto xoff = [&](uint32_t rr, int j) {
         return rr * 256u + ((((uint32_t)(8 * wg + j)) ^ (rr & 7u)) << 4);
     };
-    // Rows of a [128 x 64] TMEM block (T_A[0,64)) -> bf16 rows of `out` for the chunk at t0.
-    // kcoef != 0: + kcoef * k_t (the prefactor's dk term; k row from the K tile).  With a
-    // partner: this CTA stores rows 64 rank .. + 63, adding the partner's partial (exchange
-    // xi: staged at `stage`, received at `recv`); the other rows are sent.
-    auto finish_rows = [&](__nv_bfloat16* out, int t0, bool valid, float kcoef, int xi,
-                           uint32_t stage, uint32_t recv, bool last_of_chunk) -> bool {
+    // Rows of a [128 x 64] TMEM block (T_A[0,64)) -> bf16 rows of `out` for the chunk at t0,
+    // in two steps so that the exchange's latency is hidden behind other work.
+    // send_rows: kcoef != 0 adds kcoef * k_t (the prefactor's dk term; k row from the K
+    // tile).  Without a partner every row is stored at once.  With one, the rows the partner
+    // finishes are staged at `stage` and bulk-copied to its `recv` (once it has signalled
+    // that the region is free); this CTA's own rows (64 rank .. + 63) stay in T_A (written
+    // back when the dk term was added) for finalize_rows.
+    auto send_rows = [&](__nv_bfloat16* out, int t0, bool valid, float kcoef, int xi,
+                         uint32_t stage, uint32_t recv) -> bool {
         float v_[32];
         tmem_ld16(tm_row + L::T_A + 32 * wg, *reinterpret_cast<float(*)[16]>(&v_[0]));
         tmem_ld16(tm_row + L::T_A + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&v_[16]));
@@ -443,17 +446,37 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             }
         }
         bool ok = true;
-        const uint32_t rr = (uint32_t)t & 63u;
-        const bool own = CS == 1 || (t >> 6) == rank;
-        if (CS > 1) {
+        const bool own = CS == 1 || (t >> 6) == rank;  // uniform over a warp
+        if (CS == 1) {
+            if (valid) {
+                uint4* dst = reinterpret_cast<uint4*>(out + base + (size_t)(t0 + t) * 64 + 32 * wg);
+#pragma unroll
+                for (int cc = 0; cc < 4; ++cc)
+                    dst[cc] = make_uint4(pack_bf16(v_[8 * cc], v_[8 * cc + 1]),
+                                         pack_bf16(v_[8 * cc + 2], v_[8 * cc + 3]),
+                                         pack_bf16(v_[8 * cc + 4], v_[8 * cc + 5]),
+                                         pack_bf16(v_[8 * cc + 6], v_[8 * cc + 7]));
+            }
+        } else {
+            const uint32_t rr = (uint32_t)t & 63u;
             if (!own) {
 #pragma unroll
                 for (int j = 0; j < 8; ++j)
                     st_shared_v4(stage + xoff(rr, j), __float_as_uint(v_[4 * j]),
                                  __float_as_uint(v_[4 * j + 1]), __float_as_uint(v_[4 * j + 2]),
                                  __float_as_uint(v_[4 * j + 3]));
+            } else if (KW && xi == 1) {  // own dk rows keep the dk term
+                uint32_t w_[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) w_[i] = __float_as_uint(v_[i]);
+                tmem_st16(tm_row + L::T_A + 32 * wg, w_);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) w_[i] = __float_as_uint(v_[16 + i]);
+                tmem_st16(tm_row + L::T_A + 32 * wg + 16, w_);
+                tmem_wait_st();
             }
             fence_proxy_async();  // the staged rows, visible to the bulk copy
+            fence_before_sync();
             __syncthreads();
             if (tid == 0) {
                 if (xi == 0) {  // one "ready" per chunk covers its exchanges
@@ -464,114 +487,155 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                     bulk_copy_cluster(mapa(recv, partner), stage, kXBytes,
                                       mapa(smem_u32(&xfull[xi]), partner));
             }
-            if (own) {
-                ok = ok && bar_wait(&xfull[xi], ph_xfull[xi], &abort_flag, status);
-                if (ok) {
+        }
+        fence_proxy_async();  // generic reads of the K tile before its next TMA load
+        ok = !__syncthreads_or(!ok);
+        fence_after_sync();
+        return ok;
+    };
+    // finalize_rows (with a partner): once the partner's partial of this CTA's own rows has
+    // landed at `recv`, adds it to the rows still in T_A and stores bf16 rows of the chunk at
+    // t0 (CL valid rows); re-arms exchange xi for the next chunk and, after the chunk's last
+    // exchange, tells the partner that its staging region may be rewritten.
+    auto finalize_rows = [&](__nv_bfloat16* out, int t0, int CL, int xi, uint32_t recv,
+                             bool last) -> bool {
+        if (CS == 1) return true;
+        bool ok = true;
+        if ((t >> 6) == rank) {  // uniform over a warp
+            const uint32_t rr = (uint32_t)t & 63u;
+            float v_[32];
+            tmem_ld16(tm_row + L::T_A + 32 * wg, *reinterpret_cast<float(*)[16]>(&v_[0]));
+            tmem_ld16(tm_row + L::T_A + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&v_[16]));
+            ok = bar_wait(&xfull[xi], ph_xfull[xi], &abort_flag, status);
+            tmem_wait_ld();
+            if (ok) {
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        const float4 p4 = *reinterpret_cast<const float4*>(sm + (recv - sb) + xoff(rr, j));
-                        v_[4 * j] += p4.x;
-                        v_[4 * j + 1] += p4.y;
-                        v_[4 * j + 2] += p4.z;
-                        v_[4 * j + 3] += p4.w;
-                    }
+                for (int j = 0; j < 8; ++j) {
+                    const float4 p4 = *reinterpret_cast<const float4*>(sm + (recv - sb) + xoff(rr, j));
+                    v_[4 * j] += p4.x;
+                    v_[4 * j + 1] += p4.y;
+                    v_[4 * j + 2] += p4.z;
+                    v_[4 * j + 3] += p4.w;
+                }
+                if (t < CL) {
+                    uint4* dst = reinterpret_cast<uint4*>(out + base + (size_t)(t0 + t) * 64 + 32 * wg);
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc)
+                        dst[cc] = make_uint4(pack_bf16(v_[8 * cc], v_[8 * cc + 1]),
+                                             pack_bf16(v_[8 * cc + 2], v_[8 * cc + 3]),
+                                             pack_bf16(v_[8 * cc + 4], v_[8 * cc + 5]),
+                                             pack_bf16(v_[8 * cc + 6], v_[8 * cc + 7]));
                 }
             }
-            ph_xfull[xi] ^= 1;
         }
-        if (own && valid && ok) {
-            uint4* dst = reinterpret_cast<uint4*>(out + base + (size_t)(t0 + t) * 64 + 32 * wg);
-#pragma unroll
-            for (int cc = 0; cc < 4; ++cc)
-                dst[cc] = make_uint4(pack_bf16(v_[8 * cc], v_[8 * cc + 1]),
-                                     pack_bf16(v_[8 * cc + 2], v_[8 * cc + 3]),
-                                     pack_bf16(v_[8 * cc + 4], v_[8 * cc + 5]),
-                                     pack_bf16(v_[8 * cc + 6], v_[8 * cc + 7]));
-        }
+        ph_xfull[xi] ^= 1;
+        fence_before_sync();
         ok = !__syncthreads_or(!ok);
-        if (CS > 1 && ok && tid == 0) {
-            // the next chunk's exchange of this kind; after the last one of the chunk the
-            // partner may reuse its staging region
+        fence_after_sync();
+        if (ok && tid == 0) {
             mbar_arrive_expect_tx(&xfull[xi], kXBytes);
-            if (last_of_chunk) mbar_arrive_cluster(mapa(smem_u32(&xdone), partner));
+            if (last) mbar_arrive_cluster(mapa(smem_u32(&xdone), partner));
         }
         return ok;
+    };
+    // TMA of one tile of chunk cn into shared memory (completes on tma_bar)
+    auto load_tile = [&](uint32_t dst, const CUtensorMap* map, int cn) {
+        tma_load_3d(sb + dst, map, 0, cn * kC, bh, &tma_bar);
     };
 
     const int nch = (N + kC - 1) / kC;
     const float dscale = 1.0f / (float)M;  // den' = M den
+    // Tiles of chunk c + 1 are loaded while chunk c is worked on, each as soon as its region
+    // is free: pass F: dout, out after g is built, k after the projections, v after the state
+    // update, q after the projection backward; pass R: q, v, dout, out after the gradient
+    // MMAs, k once the dk rows are sent.  All five complete on tma_bar.
+    if (tid == 0) {
+        const int c0 = PASS == kPassF ? 0 : nch - 1;
+        mbar_arrive_expect_tx(&tma_bar, 5 * kTileBytes);
+        load_tile(L::Q, &tmap_q, c0);
+        load_tile(L::K, &tmap_k, c0);
+        load_tile(L::V, &tmap_v, c0);
+        load_tile(L::DO, &tmap_do, c0);
+        load_tile(L::O, &tmap_o, c0);
+    }
+    int prev_t0 = 0, prev_CL = 0;  // the chunk whose dq (F) or dk (R) rows await the partner
+    bool tma_outstanding = true;   // tile loads issued and not yet waited for
     for (int it = 0; it < nch; ++it) {
         const int c = PASS == kPassF ? it : nch - 1 - it;
+        const int cn = PASS == kPassF ? c + 1 : c - 1;  // the next chunk, if it exists
+        const bool has_next = it + 1 < nch;
         const int t0 = c * kC, CL = min(kC, N - t0);
         const bool valid = t < CL;
         const float wk = (KW && valid) ? kw[(size_t)bh * N + t0 + t] : 1.f;
-        if (tid == 0) {  // the next chunk's tiles into L2 while this one is worked on
-            const int cn = PASS == kPassF ? c + 1 : c - 1;
-            if (cn >= 0 && cn < nch) {
-                const size_t off = base + (size_t)cn * kC * 64;
-                const uint32_t bytes = (uint32_t)min(kC, N - cn * kC) * 128;
-                prefetch_l2(q + off, bytes);
-                prefetch_l2(k + off, bytes);
-                prefetch_l2(v + off, bytes);
-                prefetch_l2(dout + off, bytes);
-                prefetch_l2(outp + off, bytes);
-            }
+        if (tid == 0 && it + 2 < nch) {  // the chunk after next into L2
+            const int c2 = PASS == kPassF ? c + 2 : c - 2;
+            const size_t off = base + (size_t)c2 * kC * 64;
+            const uint32_t bytes = (uint32_t)min(kC, N - c2 * kC) * 128;
+            prefetch_l2(q + off, bytes);
+            prefetch_l2(k + off, bytes);
+            prefetch_l2(v + off, bytes);
+            prefetch_l2(dout + off, bytes);
+            prefetch_l2(outp + off, bytes);
         }
-        // ---- loads: q, k, v, dout, out tiles (TMA; rows past N read as zero; dout and out
-        // go to [DO | O], free until pass R stores bf16(A) there later in the chunk); then
-        // the g tile and c_t from dout, out (shared memory) and den ----
-        if (tid == 0) {
-            mbar_arrive_expect_tx(&tma_bar, 5 * kTileBytes);
-            tma_load_3d(sb + L::Q, &tmap_q, 0, t0, bh, &tma_bar);
-            tma_load_3d(sb + L::K, &tmap_k, 0, t0, bh, &tma_bar);
-            tma_load_3d(sb + L::V, &tmap_v, 0, t0, bh, &tma_bar);
-            tma_load_3d(sb + L::DO, &tmap_do, 0, t0, bh, &tma_bar);
-            tma_load_3d(sb + L::O, &tmap_o, 0, t0, bh, &tma_bar);
-        }
-        const float den_t = (wg == 0 && valid) ? den[(size_t)bh * N + t0 + t] : 1.f;
+        // ---- this chunk's tiles (rows past N read as zero); then the g tile and c_t from
+        // dout, out (shared memory) and den, each thread taking half a row ----
+        const float den_t = valid ? den[(size_t)bh * N + t0 + t] : 1.f;
         if (!bar_wait(&tma_bar, tma_phase, &abort_flag, status)) goto done;
         tma_phase ^= 1;
-        if (wg == 0) {
-            float gsc = 0.f, cval = 0.f;
-            uint32_t gp[32];
-            if (valid) {
-                gsc = dscale / den_t;
-                float dot = 0.f;
+        tma_outstanding = false;
+        // pass R: the previous chunk's dk rows (received in GT, which g overwrites next)
+        if (PASS == kPassR && it > 0 &&
+            !finalize_rows(dx_out, prev_t0, prev_CL, 1, sb + L::GT, true))
+            goto done;
+        {
+            const float gsc = valid ? dscale / den_t : 0.f;
+            float dot = 0.f;
+            uint32_t gp[16];
 #pragma unroll
-                for (int cc = 0; cc < 8; ++cc) {
-                    const uint4 a4 = *reinterpret_cast<const uint4*>(sm + L::DO + swz128(t, cc * 8));
-                    const uint4 o4 = *reinterpret_cast<const uint4*>(sm + L::O + swz128(t, cc * 8));
-                    const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w}, ow[4] = {o4.x, o4.y, o4.z, o4.w};
+            for (int j = 0; j < 4; ++j) {
+                const int cc = 4 * wg + j;
+                const uint4 a4 = *reinterpret_cast<const uint4*>(sm + L::DO + swz128(t, cc * 8));
+                const uint4 o4 = *reinterpret_cast<const uint4*>(sm + L::O + swz128(t, cc * 8));
+                const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w}, ow[4] = {o4.x, o4.y, o4.z, o4.w};
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float a0 = __uint_as_float(aw[e] << 16), a1 = __uint_as_float(aw[e] & 0xFFFF0000u);
-                        const float b0 = __uint_as_float(ow[e] << 16), b1 = __uint_as_float(ow[e] & 0xFFFF0000u);
-                        // c uses the same bf16-rounded g as the MMAs, so g.v_j + c_i cancels
-                        // exactly where out_i = v_j (e.g. the first causal position)
-                        const uint32_t gw = pack_bf16(a0 * gsc, a1 * gsc);
-                        gp[cc * 4 + e] = gw;
-                        dot = fmaf(__uint_as_float(gw << 16), b0,
-                                   fmaf(__uint_as_float(gw & 0xFFFF0000u), b1, dot));
-                    }
+                for (int e = 0; e < 4; ++e) {
+                    const float a0 = __uint_as_float(aw[e] << 16), a1 = __uint_as_float(aw[e] & 0xFFFF0000u);
+                    const float b0 = __uint_as_float(ow[e] << 16), b1 = __uint_as_float(ow[e] & 0xFFFF0000u);
+                    // c uses the same bf16-rounded g as the MMAs, so g.v_j + c_i cancels
+                    // exactly where out_i = v_j (e.g. the first causal position)
+                    const uint32_t gw = pack_bf16(a0 * gsc, a1 * gsc);
+                    gp[j * 4 + e] = gw;
+                    dot = fmaf(__uint_as_float(gw << 16), b0,
+                               fmaf(__uint_as_float(gw & 0xFFFF0000u), b1, dot));
                 }
-                cval = -dot;
-            } else {
-#pragma unroll
-                for (int e = 0; e < 32; ++e) gp[e] = 0u;
             }
 #pragma unroll
-            for (int cc = 0; cc < 8; ++cc)
-                st_shared_v4(sb + L::GT + swz128(t, cc * 8), gp[4 * cc], gp[4 * cc + 1],
-                             gp[4 * cc + 2], gp[4 * cc + 3]);
+            for (int j = 0; j < 4; ++j)
+                st_shared_v4(sb + L::GT + swz128(t, (4 * wg + j) * 8), gp[4 * j], gp[4 * j + 1],
+                             gp[4 * j + 2], gp[4 * j + 3]);
+            spart[128 * wg + t] = dot;  // free until the feature backward
+        }
+        handoff();
+        if (wg == 0) {
+            const float cval = valid ? -(spart[t] + spart[128 + t]) : 0.f;
             crow[t] = cval;
             if (PASS == kPassR)  // row 0 of the K-major [16][tokens] c operand
                 *reinterpret_cast<__nv_bfloat16*>(sm + L::C16 + (t >> 6) * 2048 + swz128(0, t & 63)) =
                     __float2bfloat16_rn(cval);
         }
-        handoff();
-        if (PASS == kPassF) signal_ready();  // DO is free for the partner's dq partial
+        if (PASS == kPassF) {
+            if (tid == 0 && has_next) {  // DO, O are free: the next chunk's dout, out
+                mbar_arrive_expect_tx(&tma_bar, 5 * kTileBytes);
+                load_tile(L::DO, &tmap_do, cn);
+                load_tile(L::O, &tmap_o, cn);
+            }
+            tma_outstanding = has_next;
+            // the previous chunk's dq rows (received in PK, which the features overwrite)
+            if (it > 0 && !finalize_rows(dx_out, prev_t0, prev_CL, 0, sb + L::PK, true)) goto done;
+        }
         // ---- features of q and k for this group ----
         if (!project_qk()) goto done;
+        if (PASS == kPassF && tid == 0 && has_next) load_tile(L::K, &tmap_k, cn);  // K is free
         // the partner has read the previous chunk's exchange data staged in PQ
         if (CS > 1 && !wait_done(it > 0)) goto done;
         features(sb + L::PQ, L::T_P, valid, 1.f);
@@ -628,11 +692,16 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 }
             }
             if (!commit_wait()) goto done;
+            signal_ready();  // PK is free for the partner's dq partial
+            if (tid == 0 && has_next) load_tile(L::V, &tmap_v, cn);  // V is free
             // n: u, w of q for the chain rule are still in T_P
             feature_backward(sb + L::PQ, crow[t], valid, 1.f);
             handoff();
             if (!project_back(dPQ, dPQmn, dQmn, it == 0)) goto done;
-            if (!finish_rows(dx_out, t0, valid, 0.f, 0, sb + L::PQ, sb + L::DO, true)) goto done;
+            if (tid == 0 && has_next) load_tile(L::Q, &tmap_q, cn);  // Q is free
+            if (!send_rows(dx_out, t0, valid, 0.f, 0, sb + L::PQ, sb + L::PK)) goto done;
+            prev_t0 = t0;
+            prev_CL = CL;
             if (NS) dw_accumulate(it == 0);
             snapshot();
             handoff();
@@ -709,11 +778,17 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 }
             }
             if (!commit_wait()) goto done;
-            signal_ready();  // DO, O are free for the partner's dv, dk partials
-            // dv of this group
-            if (!finish_rows(dv, t0, valid, 0.f, 0, sb + L::PQ, sb + L::DO, false)) goto done;
-            fence_before_sync();
-            __syncthreads();
+            signal_ready();  // DA2, GT are free for the partner's dv, dk partials
+            if (tid == 0 && has_next) {  // Q, V, DO, O are free: the next chunk's tiles
+                mbar_arrive_expect_tx(&tma_bar, 5 * kTileBytes);
+                load_tile(L::Q, &tmap_q, cn);
+                load_tile(L::V, &tmap_v, cn);
+                load_tile(L::DO, &tmap_do, cn);
+                load_tile(L::O, &tmap_o, cn);
+            }
+            tma_outstanding = has_next;
+            // dv of this group: sent now, finished before the projection backward overwrites it
+            if (!send_rows(dv, t0, valid, 0.f, 0, sb + L::PQ, sb + L::DA2)) goto done;
             if (NS && !project(dK)) goto done;  // u, w of k for the chain rule
             {
                 const float sp = feature_backward(sb + L::PK, 1.0f, valid, wk);
@@ -723,15 +798,23 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 }
             }
             handoff();
+            if (!finalize_rows(dv, t0, CL, 0, sb + L::DA2, false)) goto done;
             if (!project_back(dPK, dPKmn, dKmn, it == 0)) goto done;
-            if (!finish_rows(dx_out, t0, valid, KW ? 2.f * itau * (spart[t] + spart[128 + t]) : 0.f,
-                             1, sb + L::PQ + 16384, sb + L::O, true))
+            if (!send_rows(dx_out, t0, valid, KW ? 2.f * itau * (spart[t] + spart[128 + t]) : 0.f,
+                           1, sb + L::PQ + 16384, sb + L::GT))
                 goto done;
+            if (tid == 0 && has_next) load_tile(L::K, &tmap_k, cn);  // K is free
+            prev_t0 = t0;
+            prev_CL = CL;
             if (NS) dw_accumulate(it == 0);
             snapshot();
             handoff();
         }
     }
+    // the last chunk's rows that await the partner: dq (F) or dk (R)
+    if (!finalize_rows(dx_out, prev_t0, prev_CL, PASS == kPassF ? 0 : 1,
+                       sb + (PASS == kPassF ? L::PK : L::GT), false))
+        goto done;
     if (!NS) dw_accumulate(true);  // s: the sum over all chunks, from T_P[64,128)
     if (KW) {  // this CTA's dtau (pass R; 0 in pass F): warps, then in order
         for (int o = 16; o > 0; o >>= 1) dtau_acc += __shfl_xor_sync(0xffffffffu, dtau_acc, o);
@@ -745,6 +828,13 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         }
     }
 done:
+    if (abort_flag && tid == 0) {  // gave up: let copies into this CTA's shared memory land
+        if (tma_outstanding) mbar_drain(&tma_bar, tma_phase, kDrainCycles);
+        if (CS > 1) {
+            mbar_drain(&xfull[0], ph_xfull[0], kDrainCycles);
+            if (PASS == kPassR) mbar_drain(&xfull[1], ph_xfull[1], kDrainCycles);
+        }
+    }
     fence_before_sync();
     __syncthreads();
     fence_after_sync();

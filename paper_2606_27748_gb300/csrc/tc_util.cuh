@@ -163,6 +163,17 @@ __device__ __forceinline__ void diagnostic_stall(uint64_t* bar, volatile int* ab
     if (cycles > 0) bar_wait(bar, 0, abort_flag, status, cycles);
 }
 
+// On the way out after an abort: waits at most `limit` clocks, regardless of the abort
+// flag, for a phase of an mbarrier that copies into this CTA's shared memory complete on,
+// so that none is still in flight when the CTA exits.
+constexpr long long kDrainCycles = 20000000LL;  // ~10 ms
+__device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, long long limit)
+{
+    const long long t0 = clock64();
+    while (!mbar_try_wait(bar, parity) && clock64() - t0 < limit) {
+    }
+}
+
 // bar_wait for a barrier that other CTAs of the cluster arrive on (acquire at cluster scope).
 __device__ __forceinline__ bool bar_wait_cluster(uint64_t* bar, uint32_t parity,
                                                  volatile int* abort_flag, int* status)
