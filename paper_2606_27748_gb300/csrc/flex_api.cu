@@ -165,7 +165,7 @@ int flex_linattn_bwd(const flex_shape* shape, const void* q, const void* k, cons
     cudaStream_t s = (cudaStream_t)stream;
     void* scratch = (char*)ws + header_bytes();
     if (flex::tc_bwd_supported(p))  // with tau: one more launch, the key weights
-        return count(tau ? 3 : 2,
+        return count(flex::tc_bwd_launches(p, tau != nullptr),
                      flex::launch_tc_bwd(p, q, k, v, W1, W2, tau, out, den, dout, dq, dk, dv,
                                          dW1, dW2, dtau, scratch, &((flex::WsHeader*)ws)->status,
                                          s));

@@ -89,6 +89,7 @@ cudaError_t launch_tc_nc(const Problem& p, const void* q, const void* k, const v
 
 bool tc_bwd_supported(const Problem& p);
 size_t tc_bwd_ws_bytes(const Problem& p);
+int tc_bwd_launches(const Problem& p, bool tau);  // kernels enqueued by launch_tc_bwd
 cudaError_t launch_tc_bwd(const Problem& p, const void* q, const void* k, const void* v,
                           const float* W1, const float* W2, const float* tau, const void* out,
                           const float* den, const void* dout, void* dq, void* dk, void* dv,

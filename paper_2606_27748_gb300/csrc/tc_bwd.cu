@@ -53,6 +53,11 @@ constexpr int kC = 128;
 constexpr int kThreadsB = 256;
 constexpr uint32_t kXBytes = 64 * 64 * 4;  // one exchanged half: 64 rows x 64 fp32
 enum { kPassF = 0, kPassR = 1 };
+// kCausal: the chunked scans of the causal gradient.  Non-causal (every key for every query):
+// kState sums partial states over a range of chunks (pass F: [S | z] = sum phi(k) [v | 1],
+// pass R: [R | r] = sum phi(q) [g | c]); kGrad starts from their totals and needs no scan:
+// pass F dphi(q) = S g + c z, pass R dphi(k) = R v + r and dv = R^T phi(k).
+enum { kCausal = 0, kState = 1, kGrad = 2 };
 
 template <bool NS>
 struct BwCfg {
@@ -79,8 +84,9 @@ __device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes)
 }
 
 // KW: key weights of the norm prefactor given (compile-time; the plain kernel is unchanged);
-// CS: CTAs per cluster = frequency groups (1 or 2)
-template <bool NS, bool KW, int CS>
+// CS: CTAs per cluster = frequency groups (1 or 2; 1 for kState, which exchanges nothing);
+// MODE: kCausal, kState or kGrad
+template <bool NS, bool KW, int CS, int MODE>
 __global__ void __launch_bounds__(kThreadsB, 1)
     tc_bwd_kernel(const __grid_constant__ CUtensorMap tmap_q,
                   const __grid_constant__ CUtensorMap tmap_k,
@@ -95,14 +101,21 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                   __nv_bfloat16* __restrict__ dk, __nv_bfloat16* __restrict__ dv,
                   float* __restrict__ dw_part,
                   const float* __restrict__ kw, const float* __restrict__ tau,
-                  float* __restrict__ dtau_part, int units, int* status)
+                  float* __restrict__ dtau_part, int units, int nsplit,
+                  float* __restrict__ state_part, const float* __restrict__ state_total,
+                  int* status)
 {
     using L = BwCfg<NS>;
-    // blocks [0, units): pass R, [units, 2 units): pass F; unit = (sequence, group); partial
-    // slots are indexed by slot = pass * units + unit
-    const int PASS = (int)blockIdx.x < units ? kPassR : kPassF;
-    const int unit = (int)blockIdx.x % units;
-    const int slot = PASS * units + unit;
+    // blocks [0, half): pass R, [half, 2 half): pass F, half = units * nsplit; within a pass
+    // idx = (sequence * nsplit + split) * G + group (the groups of a cluster adjacent); the
+    // chunks are split into nsplit ranges (non-causal modes; 1 for the causal scans).
+    // Partial slots are indexed by slot = pass * half + idx.
+    const int half_grid = units * nsplit;
+    const int PASS = (int)blockIdx.x < half_grid ? kPassR : kPassF;
+    const int idx = (int)blockIdx.x % half_grid;
+    const int split = (idx / G) % nsplit;
+    const int unit = (idx / G / nsplit) * G + idx % G;
+    const int slot = PASS * half_grid + idx;
     __nv_bfloat16* const dx_out = PASS == kPassF ? dq : dk;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -244,7 +257,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         }
         tmem_wait_ld();
         if (NS)
-            reduce_2pi_if_needed(a, w);
+            cos_w_args(a, w);  // w <- cos(w)
         else
             reduce_2pi_if_needed(a);
         uint32_t pc[16], ps[16];
@@ -254,7 +267,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             __sincosf(a[2 * i], &s0, &c0);
             __sincosf(a[2 * i + 1], &s1, &c1);
             if (NS) {
-                const float cw0 = __cosf(w[2 * i]), cw1 = __cosf(w[2 * i + 1]);
+                const float cw0 = w[2 * i], cw1 = w[2 * i + 1];
                 c0 *= cw0; s0 *= cw0; c1 *= cw1; s1 *= cw1;
             }
             if (KW) { c0 *= wsc; s0 *= wsc; c1 *= wsc; s1 *= wsc; }
@@ -322,7 +335,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                     const float pc = __uint_as_float(e ? cpair[i] & 0xFFFF0000u : cpair[i] << 16);
                     const float psn = __uint_as_float(e ? spair[i] & 0xFFFF0000u : spair[i] << 16);
                     r1[e] = -psn * dphic + pc * dphis;
-                    r2[e] = 0.f;
+                    r2[e] = 0.f;  // (the low bf16 part of da, set below)
                     if (wt) sdot = fmaf(pc, dphic, fmaf(psn, dphis, sdot));
                 } else {
                     float su, cu, sw, cw;
@@ -339,6 +352,13 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 if (!valid) r1[e] = r2[e] = 0.f;
             }
             o1[i] = pack_bf16(r1[0], r1[1]);
+            if (!NS) {
+                // s: the sin half of the tile (unused by dx = da W) carries da - bf16(da), so
+                // the dW MMA (all 128 rows) gets da to ~2^-17: rows 64-127 of dW are added
+                // to rows 0-63 in the reduction
+                r2[0] = r1[0] - __uint_as_float(o1[i] << 16);
+                r2[1] = r1[1] - __uint_as_float(o1[i] & 0xFFFF0000u);
+            }
             o2[i] = pack_bf16(r2[0], r2[1]);
         }
 #pragma unroll
@@ -374,7 +394,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         for (int j = 0; j < 4; ++j)
             tmem_ld16(tm_row + T_DW + 16 * j, *reinterpret_cast<float(*)[16]>(&v_[16 * j]));
         tmem_wait_ld();
-        if (t < L::P && wg == 1) {
+        if (wg == 1) {  // all 128 rows (s: rows 64-127 hold the low part's contribution)
             float4* dst = reinterpret_cast<float4*>(dw_part + ((size_t)slot * 128 + t) * 64);
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
@@ -538,57 +558,13 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         }
         return ok;
     };
-    // TMA of one tile of chunk cn into shared memory (completes on tma_bar)
-    auto load_tile = [&](uint32_t dst, const CUtensorMap* map, int cn) {
-        tma_load_3d(sb + dst, map, 0, cn * kC, bh, &tma_bar);
-    };
-
-    const int nch = (N + kC - 1) / kC;
     const float dscale = 1.0f / (float)M;  // den' = M den
-    // Tiles of chunk c + 1 are loaded while chunk c is worked on, each as soon as its region
-    // is free: pass F: dout, out after g is built, k after the projections, v after the state
-    // update, q after the projection backward; pass R: q, v, dout, out after the gradient
-    // MMAs, k once the dk rows are sent.  All five complete on tma_bar.
-    if (tid == 0) {
-        const int c0 = PASS == kPassF ? 0 : nch - 1;
-        mbar_arrive_expect_tx(&tma_bar, 5 * kTileBytes);
-        load_tile(L::Q, &tmap_q, c0);
-        load_tile(L::K, &tmap_k, c0);
-        load_tile(L::V, &tmap_v, c0);
-        load_tile(L::DO, &tmap_do, c0);
-        load_tile(L::O, &tmap_o, c0);
-    }
-    int prev_t0 = 0, prev_CL = 0;  // the chunk whose dq (F) or dk (R) rows await the partner
-    bool tma_outstanding = true;   // tile loads issued and not yet waited for
-    for (int it = 0; it < nch; ++it) {
-        const int c = PASS == kPassF ? it : nch - 1 - it;
-        const int cn = PASS == kPassF ? c + 1 : c - 1;  // the next chunk, if it exists
-        const bool has_next = it + 1 < nch;
-        const int t0 = c * kC, CL = min(kC, N - t0);
-        const bool valid = t < CL;
-        const float wk = (KW && valid) ? kw[(size_t)bh * N + t0 + t] : 1.f;
-        if (tid == 0 && it + 2 < nch) {  // the chunk after next into L2
-            const int c2 = PASS == kPassF ? c + 2 : c - 2;
-            const size_t off = base + (size_t)c2 * kC * 64;
-            const uint32_t bytes = (uint32_t)min(kC, N - c2 * kC) * 128;
-            prefetch_l2(q + off, bytes);
-            prefetch_l2(k + off, bytes);
-            prefetch_l2(v + off, bytes);
-            prefetch_l2(dout + off, bytes);
-            prefetch_l2(outp + off, bytes);
-        }
-        // ---- this chunk's tiles (rows past N read as zero); then the g tile and c_t from
-        // dout, out (shared memory) and den, each thread taking half a row ----
-        const float den_t = valid ? den[(size_t)bh * N + t0 + t] : 1.f;
-        if (!bar_wait(&tma_bar, tma_phase, &abort_flag, status)) goto done;
-        tma_phase ^= 1;
-        tma_outstanding = false;
-        // pass R: the previous chunk's dk rows (received in GT, which g overwrites next)
-        if (PASS == kPassR && it > 0 &&
-            !finalize_rows(dx_out, prev_t0, prev_CL, 1, sb + L::GT, true))
-            goto done;
+    // g = dout / den' (bf16, the tile GT) and c_t = -(g . out) (crow; with c_row also row 0
+    // of the c operand C16, and with c_lo row 1 = c - bf16(c)) from the dout and out tiles;
+    // each thread takes half a row.
+    auto build_g = [&](bool valid_, float den_t, bool c_row, bool c_lo) {
         {
-            const float gsc = valid ? dscale / den_t : 0.f;
+            const float gsc = valid_ ? dscale / den_t : 0.f;
             float dot = 0.f;
             uint32_t gp[16];
 #pragma unroll
@@ -617,12 +593,68 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         }
         handoff();
         if (wg == 0) {
-            const float cval = valid ? -(spart[t] + spart[128 + t]) : 0.f;
+            const float cval = valid_ ? -(spart[t] + spart[128 + t]) : 0.f;
             crow[t] = cval;
-            if (PASS == kPassR)  // row 0 of the K-major [16][tokens] c operand
-                *reinterpret_cast<__nv_bfloat16*>(sm + L::C16 + (t >> 6) * 2048 + swz128(0, t & 63)) =
-                    __float2bfloat16_rn(cval);
+            if (c_row) {  // row 0 of the K-major [16][tokens] c operand
+                const __nv_bfloat16 chi = __float2bfloat16_rn(cval);
+                *reinterpret_cast<__nv_bfloat16*>(sm + L::C16 + (t >> 6) * 2048 + swz128(0, t & 63)) = chi;
+                if (c_lo)
+                    *reinterpret_cast<__nv_bfloat16*>(sm + L::C16 + (t >> 6) * 2048 + swz128(1, t & 63)) =
+                        __float2bfloat16_rn(cval - __bfloat162float(chi));
+            }
         }
+    };
+    // TMA of one tile of chunk cn into shared memory (completes on tma_bar)
+    auto load_tile = [&](uint32_t dst, const CUtensorMap* map, int cn) {
+        tma_load_3d(sb + dst, map, 0, cn * kC, bh, &tma_bar);
+    };
+
+    const int nch = (N + kC - 1) / kC;
+    int prev_t0 = 0, prev_CL = 0;  // the chunk whose dq (F) or dk (R) rows await the partner
+    bool tma_outstanding = false;  // tile loads issued and not yet waited for
+    if constexpr (MODE == kCausal) {
+    // Tiles of chunk c + 1 are loaded while chunk c is worked on, each as soon as its region
+    // is free: pass F: dout, out after g is built, k after the projections, v after the state
+    // update, q after the projection backward; pass R: q, v, dout, out after the gradient
+    // MMAs, k once the dk rows are sent.  All five complete on tma_bar.
+    if (tid == 0) {
+        const int c0 = PASS == kPassF ? 0 : nch - 1;
+        mbar_arrive_expect_tx(&tma_bar, 5 * kTileBytes);
+        load_tile(L::Q, &tmap_q, c0);
+        load_tile(L::K, &tmap_k, c0);
+        load_tile(L::V, &tmap_v, c0);
+        load_tile(L::DO, &tmap_do, c0);
+        load_tile(L::O, &tmap_o, c0);
+    }
+    tma_outstanding = true;
+    for (int it = 0; it < nch; ++it) {
+        const int c = PASS == kPassF ? it : nch - 1 - it;
+        const int cn = PASS == kPassF ? c + 1 : c - 1;  // the next chunk, if it exists
+        const bool has_next = it + 1 < nch;
+        const int t0 = c * kC, CL = min(kC, N - t0);
+        const bool valid = t < CL;
+        const float wk = (KW && valid) ? kw[(size_t)bh * N + t0 + t] : 1.f;
+        if (tid == 0 && it + 2 < nch) {  // the chunk after next into L2
+            const int c2 = PASS == kPassF ? c + 2 : c - 2;
+            const size_t off = base + (size_t)c2 * kC * 64;
+            const uint32_t bytes = (uint32_t)min(kC, N - c2 * kC) * 128;
+            prefetch_l2(q + off, bytes);
+            prefetch_l2(k + off, bytes);
+            prefetch_l2(v + off, bytes);
+            prefetch_l2(dout + off, bytes);
+            prefetch_l2(outp + off, bytes);
+        }
+        // ---- this chunk's tiles (rows past N read as zero); then the g tile and c_t from
+        // dout, out (shared memory) and den, each thread taking half a row ----
+        const float den_t = valid ? den[(size_t)bh * N + t0 + t] : 1.f;
+        if (!bar_wait(&tma_bar, tma_phase, &abort_flag, status)) goto done;
+        tma_phase ^= 1;
+        tma_outstanding = false;
+        // pass R: the previous chunk's dk rows (received in GT, which g overwrites next)
+        if (PASS == kPassR && it > 0 &&
+            !finalize_rows(dx_out, prev_t0, prev_CL, 1, sb + L::GT, true))
+            goto done;
+        build_g(valid, den_t, PASS == kPassR, false);
         if (PASS == kPassF) {
             if (tid == 0 && has_next) {  // DO, O are free: the next chunk's dout, out
                 mbar_arrive_expect_tx(&tma_bar, 5 * kTileBytes);
@@ -815,8 +847,200 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     if (!finalize_rows(dx_out, prev_t0, prev_CL, PASS == kPassF ? 0 : 1,
                        sb + (PASS == kPassF ? L::PK : L::GT), false))
         goto done;
-    if (!NS) dw_accumulate(true);  // s: the sum over all chunks, from T_P[64,128)
-    if (KW) {  // this CTA's dtau (pass R; 0 in pass F): warps, then in order
+    } else {
+        // ---- non-causal: the chunks [cbeg, cend) of this split, in order ----
+        const int cps = (nch + nsplit - 1) / nsplit;
+        const int cbeg = split * cps, cend = min(nch, cbeg + cps);
+        // this CTA reads q, dout, out (kState R, kGrad F) or k, v (kState F, kGrad R)
+        const bool fq = (MODE == kState) == (PASS == kPassR);
+        // kGrad: the low part of the state snapshot, in a region the pass does not use
+        const uint32_t sl = sb + (PASS == kPassF ? L::V : L::PQ);
+        const uint64_t dSL = sdesc(sl, 16, 1024), dSLmn = sdesc(sl, 16384, 1024);
+        if (MODE == kGrad) {
+            // the totals ([S | z] for pass F, [R | r] for pass R) as the state snapshot, split
+            // into bf16 high (SN) and low (SL) parts [feature][64] so that the two MMAs carry
+            // the fp32 totals to ~2^-17: the terms S g and c z (R v and r) cancel exactly
+            // where the result is 0 (e.g. dq at N = 1); column 64 in zr (fp32)
+            const float* st = state_total + ((size_t)PASS * units + unit) * 128 * 80 + (size_t)t * 80;
+            float s_[32];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const float4 f4 = reinterpret_cast<const float4*>(st + 32 * wg)[j];
+                s_[4 * j] = f4.x; s_[4 * j + 1] = f4.y; s_[4 * j + 2] = f4.z; s_[4 * j + 3] = f4.w;
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                uint32_t hi[4], lo[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float x0 = s_[8 * j + 2 * e], x1 = s_[8 * j + 2 * e + 1];
+                    hi[e] = pack_bf16(x0, x1);
+                    lo[e] = pack_bf16(x0 - __uint_as_float(hi[e] << 16),
+                                      x1 - __uint_as_float(hi[e] & 0xFFFF0000u));
+                }
+                const uint32_t off = swz128(t, (4 * wg + j) * 8);
+                st_shared_v4(sb + L::SN + off, hi[0], hi[1], hi[2], hi[3]);
+                st_shared_v4(sl + off, lo[0], lo[1], lo[2], lo[3]);
+            }
+            if (wg == 0) zr[t] = st[64];
+            signal_ready();  // this CTA's receive regions are free for the first exchange
+        }
+        for (int c = cbeg; c < cend; ++c) {
+            const int it = c - cbeg;
+            const int t0 = c * kC, CL = min(kC, N - t0);
+            const bool valid = t < CL;
+            const float wk = (KW && !fq && valid) ? kw[(size_t)bh * N + t0 + t] : 1.f;
+            const float den_t = (fq && valid) ? den[(size_t)bh * N + t0 + t] : 1.f;
+            // ---- this chunk's tiles (rows past N read as zero); the next into L2 ----
+            if (tid == 0) {
+                if (c + 1 < cend) {
+                    const size_t off = base + (size_t)(c + 1) * kC * 64;
+                    const uint32_t bytes = (uint32_t)min(kC, N - (c + 1) * kC) * 128;
+                    if (fq) {
+                        prefetch_l2(q + off, bytes);
+                        prefetch_l2(dout + off, bytes);
+                        prefetch_l2(outp + off, bytes);
+                    } else {
+                        prefetch_l2(k + off, bytes);
+                        prefetch_l2(v + off, bytes);
+                    }
+                }
+                mbar_arrive_expect_tx(&tma_bar, (fq ? 3 : 2) * kTileBytes);
+                if (fq) {
+                    load_tile(L::Q, &tmap_q, c);
+                    load_tile(L::DO, &tmap_do, c);
+                    load_tile(L::O, &tmap_o, c);
+                } else {
+                    load_tile(L::K, &tmap_k, c);
+                    load_tile(L::V, &tmap_v, c);
+                }
+            }
+            tma_outstanding = true;
+            if (!bar_wait(&tma_bar, tma_phase, &abort_flag, status)) goto done;
+            tma_phase ^= 1;
+            tma_outstanding = false;
+            // g, c (and for the state [R | r] the c rows of C16: high and low bf16 parts, so r
+            // carries c to ~2^-17 like the exact-cancelling term g . v)
+            if (fq) build_g(valid, den_t, PASS == kPassR, MODE == kState);
+            // ---- features of the tile's rows (q or k) for this group ----
+            if (!project(fq ? dQ : dK)) goto done;
+            features(fq ? sb + L::PQ : sb + L::PK, L::T_P, valid, fq ? 1.f : wk);
+            handoff();
+            if (MODE == kState) {
+                // [S | z] += phi(K)^T [V | 1]  or  [R | r] += phi(Q)^T [G | c]
+                if (tid == 0) {
+                    fence_after_sync();
+                    const uint64_t dphi = fq ? dPQmn : dPKmn, dval = fq ? dGmn : dVmn;
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks) {
+                        const uint32_t acc = (it > 0 || ks > 0) ? 1u : 0u;
+                        mma_bf16(tm + L::T_S, adv(dphi, ks * 2048), adv(dval, ks * 2048), I_MM64, acc);
+                        mma_bf16(tm + L::T_S + 64, adv(dphi, ks * 2048),
+                                 adv(dC16, (ks >> 2) * 2048 + (ks & 3) * 32), I_M16, acc);
+                    }
+                }
+                if (!commit_wait()) goto done;
+                continue;
+            }
+            if (PASS == kPassF) {
+                // dphi(q) = g S^T (+ c z in the feature backward)
+                if (tid == 0) {
+                    fence_after_sync();
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_bf16(tm + L::T_D, adv(dG, ks * 32), adv(dSN, ks * 32), I_KK128, ks > 0);
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_bf16(tm + L::T_D, adv(dG, ks * 32), adv(dSL, ks * 32), I_KK128, 1u);
+                }
+                if (!commit_wait()) goto done;
+                // n: u, w of q for the chain rule are still in T_P
+                feature_backward(sb + L::PQ, crow[t], valid, 1.f);
+                handoff();
+                // the previous chunk's dq rows (received in PK), before the projection
+                // backward overwrites them; PK is then free for this chunk's exchange
+                if (it > 0) {
+                    if (!finalize_rows(dx_out, prev_t0, prev_CL, 0, sb + L::PK, true)) goto done;
+                    signal_ready();
+                }
+                if (!project_back(dPQ, dPQmn, dQmn, it == 0)) goto done;
+                // the partner has read the previous chunk's rows staged in K
+                if (CS > 1 && !wait_done(it > 0)) goto done;
+                if (!send_rows(dx_out, t0, valid, 0.f, 0, sb + L::K, sb + L::PK)) goto done;
+                prev_t0 = t0;
+                prev_CL = CL;
+                if (NS) dw_accumulate(it == 0);
+                handoff();
+            } else {
+                // the previous chunk's dk rows (received in O), before T_A is overwritten;
+                // DO, O are then free for this chunk's exchanges
+                if (it > 0) {
+                    if (!finalize_rows(dx_out, prev_t0, prev_CL, 1, sb + L::O, true)) goto done;
+                    signal_ready();
+                }
+                // dphi(k) = v R^T (+ r in the feature backward);  dv = phi(K) R
+                if (tid == 0) {
+                    fence_after_sync();
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_bf16(tm + L::T_D, adv(dV, ks * 32), adv(dSN, ks * 32), I_KK128, ks > 0);
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_bf16(tm + L::T_D, adv(dV, ks * 32), adv(dSL, ks * 32), I_KK128, 1u);
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_bf16(tm + L::T_A, adv(dPK, (ks >> 2) * 16384 + (ks & 3) * 32),
+                                 adv(dSNmn, ks * 2048), I_KM64, ks > 0);
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_bf16(tm + L::T_A, adv(dPK, (ks >> 2) * 16384 + (ks & 3) * 32),
+                                 adv(dSLmn, ks * 2048), I_KM64, 1u);
+                }
+                if (!commit_wait()) goto done;
+                // the partner has read the previous chunk's rows staged in Q and DA2
+                if (CS > 1 && !wait_done(it > 0)) goto done;
+                if (!send_rows(dv, t0, valid, 0.f, 0, sb + L::Q, sb + L::DO)) goto done;
+                {  // n: u, w of k for the chain rule are still in T_P
+                    const float sp = feature_backward(sb + L::PK, 1.0f, valid, wk);
+                    if (KW) {
+                        spart[128 * wg + t] = sp;
+                        dtau_acc = fmaf(-logf(wk), sp, dtau_acc);  // ln w = |k|^2 exp(-tau)
+                    }
+                }
+                handoff();
+                if (!finalize_rows(dv, t0, CL, 0, sb + L::DO, false)) goto done;
+                if (!project_back(dPK, dPKmn, dKmn, it == 0)) goto done;
+                if (!send_rows(dx_out, t0, valid, KW ? 2.f * itau * (spart[t] + spart[128 + t]) : 0.f,
+                               1, sb + L::DA2, sb + L::O))
+                    goto done;
+                prev_t0 = t0;
+                prev_CL = CL;
+                if (NS) dw_accumulate(it == 0);
+                handoff();
+            }
+        }
+        if (MODE == kState) {
+            // this CTA's partial state [128 features][80] fp32: S (or R) in columns 0-63,
+            // z (or r) in column 64
+            float s_[32], zz[16];
+            tmem_ld16(tm_row + L::T_S + 32 * wg, *reinterpret_cast<float(*)[16]>(&s_[0]));
+            tmem_ld16(tm_row + L::T_S + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&s_[16]));
+            tmem_ld16(tm_row + L::T_S + 64, zz);
+            tmem_wait_ld();
+            float* dst = state_part + ((size_t)slot * 128 + t) * 80;
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                reinterpret_cast<float4*>(dst + 32 * wg)[j] =
+                    make_float4(s_[4 * j], s_[4 * j + 1], s_[4 * j + 2], s_[4 * j + 3]);
+            // r = column 64 (c high) + column 65 (c low); z: column 64 (every C16 row is 1)
+            if (wg == 0) dst[64] = PASS == kPassR ? zz[0] + zz[1] : zz[0];
+        } else if (!finalize_rows(dx_out, prev_t0, prev_CL, PASS == kPassF ? 0 : 1,
+                                  sb + (PASS == kPassF ? L::PK : L::O), false)) {
+            goto done;  // the last chunk's dq (F) or dk (R) rows
+        }
+    }
+    if (MODE != kState && !NS) dw_accumulate(true);  // s: the sum over the chunks, T_P[64,128)
+    if (KW && MODE != kState) {  // this CTA's dtau (pass R; 0 in pass F): warps, then in order
         for (int o = 16; o > 0; o >>= 1) dtau_acc += __shfl_xor_sync(0xffffffffu, dtau_acc, o);
         __syncthreads();
         if (lane == 0) spart[warp] = dtau_acc;
@@ -842,19 +1066,23 @@ done:
     if (CS > 1) cluster_sync();  // no CTA leaves while its partner may still copy into it
 }
 
-// dW over the batch in a fixed order.  Partial slots [pass][bh * G + g][row][64]; s: rows
-// < 64 are frequencies 64g + row; n: rows < 64 are dU, rows >= 64 are dV of frequency
-// 64g + row%64.
-__global__ void tc_dw_reduce_kernel(int B, int H, int M, int G, int nonstat,
+// dW over the batch (and the chunk splits) in a fixed order.  Partial slots
+// [pass][((b * H + h) * nsplit + s) * G + g][row][64]; s: rows < 64 are frequencies
+// 64g + row (from the high bf16 part of da), rows >= 64 the same frequencies (from its low
+// part); n: rows < 64 are dU, rows >= 64 are dV of frequency 64g + row%64.
+__global__ void tc_dw_reduce_kernel(int B, int H, int M, int G, int nsplit, int nonstat,
                                     const float* __restrict__ part, float* __restrict__ dW1,
                                     float* __restrict__ dW2, const float* __restrict__ dtau_part,
                                     float* __restrict__ dtau)
 {
+    const size_t half = (size_t)B * H * nsplit * G;  // slots per pass
     if (dtau && blockIdx.x == 0)  // dtau[h]: the pass R slots of head h, in order
         for (int h = threadIdx.x; h < H; h += blockDim.x) {
             float a = 0.f;
             for (int b = 0; b < B; ++b)
-                for (int g = 0; g < G; ++g) a += dtau_part[(size_t)B * H * G + (b * H + h) * G + g];
+                for (int sp = 0; sp < nsplit; ++sp)
+                    for (int g = 0; g < G; ++g)
+                        a += dtau_part[half + ((size_t)(b * H + h) * nsplit + sp) * G + g];
             dtau[h] = a;
         }
     const size_t total = (size_t)H * M * 64;
@@ -864,14 +1092,16 @@ __global__ void tc_dw_reduce_kernel(int B, int H, int M, int G, int nonstat,
         const int f = (int)((idx / 64) % M), e = (int)(idx % 64);
         const int g = f / 64, r = f % 64;
         float a = 0.f, b2 = 0.f;
-        const size_t pass_stride = (size_t)B * H * G * 128 * 64;  // pass R slots follow pass F's
-        for (int b = 0; b < B; ++b) {
-            const float* p = part + ((size_t)((b * H + h) * G + g) * 128) * 64;
-            a += p[(size_t)r * 64 + e] + p[pass_stride + (size_t)r * 64 + e];
-            if (nonstat) b2 += p[(size_t)(64 + r) * 64 + e] + p[pass_stride + (size_t)(64 + r) * 64 + e];
-        }
+        const size_t pass_stride = half * 128 * 64;  // pass F slots follow pass R's
+        for (int b = 0; b < B; ++b)
+            for (int sp = 0; sp < nsplit; ++sp) {
+                const float* p = part + ((((size_t)(b * H + h) * nsplit + sp) * G + g) * 128) * 64;
+                a += p[(size_t)r * 64 + e] + p[pass_stride + (size_t)r * 64 + e];
+                // n: dV rows; s: the dW rows of the low part of da
+                b2 += p[(size_t)(64 + r) * 64 + e] + p[pass_stride + (size_t)(64 + r) * 64 + e];
+            }
         if (!nonstat) {
-            dW1[idx] = a;
+            dW1[idx] = a + b2;
         } else {
             dW1[idx] = 0.5f * (a + b2);
             dW2[idx] = 0.5f * (a - b2);
@@ -879,7 +1109,96 @@ __global__ void tc_dw_reduce_kernel(int B, int H, int M, int G, int nonstat,
     }
 }
 
-template <bool NS>
+// Non-causal totals: total[pass][unit][row][0..64] = sum over the splits, in order, of the
+// partial states [pass][(bh * nsplit + s) * G + g][row][0..64] (unit = bh * G + g).
+__global__ void nc_state_reduce_kernel(int units, int G, int nsplit,
+                                       const float* __restrict__ part, float* __restrict__ total)
+{
+    const size_t n = (size_t)2 * units * 128 * 65;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (size_t)gridDim.x * blockDim.x) {
+        const int col = (int)(i % 65), row = (int)((i / 65) % 128);
+        const int u = (int)((i / (65 * 128)) % units), pass = (int)(i / ((size_t)65 * 128 * units));
+        const int bh = u / G, g = u % G;
+        float a = 0.f;
+        for (int sp = 0; sp < nsplit; ++sp)
+            a += part[(((size_t)pass * units * nsplit + ((size_t)bh * nsplit + sp) * G + g) * 128 +
+                       row) * 80 + col];
+        total[(((size_t)pass * units + u) * 128 + row) * 80 + col] = a;
+    }
+}
+
+// Chunk splits per (pass, sequence, group) for the non-causal modes: enough CTAs for a few
+// waves of ~152 SMs, every split non-empty (depends on the shape only, so the workspace size
+// is known before the call).
+int nc_splits(const Problem& p)
+{
+    const int units = p.B * p.H * (p.M / 64), nch = (p.N + kC - 1) / kC;
+    const int target = std::max(1, std::min(nch, (4 * 152 + 2 * units - 1) / (2 * units)));
+    const int cps = (nch + target - 1) / target;
+    return (nch + cps - 1) / cps;
+}
+
+// Scratch layout (every region 256-byte aligned): dW partials [2 half][128][64], key
+// weights [B*H*N] (prefactor), dtau partials [2 half]; non-causal also partial states
+// [2 half][128][80] and totals [2 units][128][80] (half = B*H*G*nsplit, units = B*H*G).
+struct BwdWs {
+    size_t part, kw, dtau, state_part, state_total, total;
+};
+BwdWs bwd_ws(const Problem& p)
+{
+    const size_t units = (size_t)p.B * p.H * (p.M / 64);
+    const size_t half = units * (p.causal ? 1 : nc_splits(p));
+    auto a64 = [](size_t n) { return align_up(n, 64); };  // floats
+    BwdWs w;
+    w.part = 0;
+    w.kw = a64(w.part + 2 * half * 128 * 64);
+    w.dtau = a64(w.kw + (size_t)p.B * p.H * p.N);
+    w.state_part = a64(w.dtau + 2 * half);
+    w.state_total = a64(w.state_part + (p.causal ? 0 : 2 * half * 128 * 80));
+    w.total = a64(w.state_total + (p.causal ? 0 : 2 * units * 128 * 80));
+    return w;  // in floats
+}
+
+struct BwdArgs {
+    CUtensorMap mq, mk, mv, mdo, mo;
+};
+
+// One launch of tc_bwd_kernel<NS, KW, CS, MODE>: 2 * units * nsplit CTAs, clusters of CS.
+template <bool NS, bool KW, int CS, int MODE>
+cudaError_t launch_mode(const Problem& p, const BwdArgs& m, const void* q, const void* k,
+                        const void* v, const float* W1, const float* W2, const float* tau,
+                        const void* out, const float* den, const void* dout, void* dq, void* dk,
+                        void* dv, float* f, const BwdWs& w, int nsplit, int* status,
+                        cudaStream_t s)
+{
+    const int smem = (int)BwCfg<NS>::BYTES + 1024;
+    auto kb = tc_bwd_kernel<NS, KW, CS, MODE>;
+    cudaError_t e = cudaFuncSetAttribute(kb, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    typedef const __nv_bfloat16* CB;
+    typedef __nv_bfloat16* B16;
+    const int units = p.B * p.H * (p.M / 64);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(2 * units * nsplit));
+    cfg.blockDim = dim3(kThreadsB);
+    cfg.dynamicSmemBytes = (size_t)smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CS;  // the frequency groups of one (pass, sequence, split)
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kb, m.mq, m.mk, m.mv, m.mdo, m.mo, p.H, p.N, p.M, p.M / 64,
+                              p.causal, (CB)q, (CB)k, (CB)v, W1, W2, (CB)out, den, (CB)dout,
+                              (B16)dq, (B16)dk, (B16)dv, f + w.part, KW ? f + w.kw : nullptr, tau,
+                              f + w.dtau, units, nsplit, f + w.state_part,
+                              (const float*)(f + w.state_total), status);
+}
+
+template <bool NS, bool KW>
 cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const void* v,
                        const float* W1, const float* W2, const float* tau, const void* out,
                        const float* den, const void* dout, void* dq, void* dk, void* dv,
@@ -887,61 +1206,59 @@ cudaError_t launch_bwd(const Problem& p, const void* q, const void* k, const voi
                        cudaStream_t s)
 {
     const int BH = p.B * p.H, G = p.M / 64;
-    float* part = static_cast<float*>(scratch);
-    float* kw = part + (size_t)2 * BH * G * 128 * 64;  // key weights [B*H*N] (prefactor)
-    float* dtau_part = kw + (size_t)BH * p.N;           // [2 units]
+    float* f = static_cast<float*>(scratch);
+    const BwdWs w = bwd_ws(p);
     cudaError_t e = cudaSuccess;
-    if (tau && (e = launch_key_weights(p, k, tau, kw, s)) != cudaSuccess) return e;
-    const int smem = (int)BwCfg<NS>::BYTES + 1024;
-    CUtensorMap mq, mk, mv, mdo, mo;
-    if (!make_act_map(&mq, q, BH, p.N) || !make_act_map(&mk, k, BH, p.N) ||
-        !make_act_map(&mv, v, BH, p.N) || !make_act_map(&mdo, dout, BH, p.N) ||
-        !make_act_map(&mo, out, BH, p.N))
+    if (KW && (e = launch_key_weights(p, k, tau, f + w.kw, s)) != cudaSuccess) return e;
+    BwdArgs m;
+    if (!make_act_map(&m.mq, q, BH, p.N) || !make_act_map(&m.mk, k, BH, p.N) ||
+        !make_act_map(&m.mv, v, BH, p.N) || !make_act_map(&m.mdo, dout, BH, p.N) ||
+        !make_act_map(&m.mo, out, BH, p.N))
         return cudaErrorInvalidValue;
-    auto kb = G == 2 ? (tau ? tc_bwd_kernel<NS, true, 2> : tc_bwd_kernel<NS, false, 2>)
-                     : (tau ? tc_bwd_kernel<NS, true, 1> : tc_bwd_kernel<NS, false, 1>);
-    if ((e = cudaFuncSetAttribute(kb, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return e;
-    typedef const __nv_bfloat16* CB;
-    typedef __nv_bfloat16* B16;
-    const int units = BH * G;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(2 * units));
-    cfg.blockDim = dim3(kThreadsB);
-    cfg.dynamicSmemBytes = (size_t)smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = G;  // the frequency groups of one (pass, sequence)
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, kb, mq, mk, mv, mdo, mo, p.H, p.N, p.M, G, p.causal, (CB)q,
-                           (CB)k, (CB)v, W1, W2, (CB)out, den, (CB)dout, (B16)dq, (B16)dk,
-                           (B16)dv, part, tau ? kw : nullptr, tau, dtau_part, units, status);
-    if (e != cudaSuccess) return e;
+    int nsplit = 1;
+    if (p.causal) {
+        e = G == 2 ? launch_mode<NS, KW, 2, kCausal>(p, m, q, k, v, W1, W2, tau, out, den, dout, dq,
+                                                     dk, dv, f, w, 1, status, s)
+                   : launch_mode<NS, KW, 1, kCausal>(p, m, q, k, v, W1, W2, tau, out, den, dout, dq,
+                                                     dk, dv, f, w, 1, status, s);
+        if (e != cudaSuccess) return e;
+    } else {
+        nsplit = nc_splits(p);
+        e = launch_mode<NS, KW, 1, kState>(p, m, q, k, v, W1, W2, tau, out, den, dout, dq, dk, dv,
+                                           f, w, nsplit, status, s);
+        if (e != cudaSuccess) return e;
+        const int units = BH * G;
+        nc_state_reduce_kernel<<<152 * 4, 256, 0, s>>>(units, G, nsplit, f + w.state_part,
+                                                       f + w.state_total);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        e = G == 2 ? launch_mode<NS, KW, 2, kGrad>(p, m, q, k, v, W1, W2, tau, out, den, dout, dq,
+                                                   dk, dv, f, w, nsplit, status, s)
+                   : launch_mode<NS, KW, 1, kGrad>(p, m, q, k, v, W1, W2, tau, out, den, dout, dq,
+                                                   dk, dv, f, w, nsplit, status, s);
+        if (e != cudaSuccess) return e;
+    }
     const size_t work = (size_t)p.H * p.M * 64;
     tc_dw_reduce_kernel<<<(int)std::min<size_t>((work + 255) / 256, 152 * 8), 256, 0, s>>>(
-        p.B, p.H, p.M, G, p.nonstat, part, dW1, dW2, dtau_part, tau ? dtau : nullptr);
+        p.B, p.H, p.M, G, nsplit, p.nonstat, f + w.part, dW1, dW2, f + w.dtau,
+        KW ? dtau : nullptr);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-// Causal only: the running prefix (pass F) and suffix (pass R) states are exactly the
-// inter-chunk terms of the causal gradient.
+// bf16, d = 64, M in {64, 128}: causal (two scans) and non-causal (totals, then every
+// chunk independently).
 bool tc_bwd_supported(const Problem& p)
 {
-    return p.bf16 && p.causal && p.d == 64 && (p.M == 64 || p.M == 128);
+    return p.bf16 && p.d == 64 && (p.M == 64 || p.M == 128);
 }
 
-// dW partials [2 passes][B*H*G][128][64], key weights [B*H*N] and dtau partials
-// [2 B*H*G] (norm prefactor).
-size_t tc_bwd_ws_bytes(const Problem& p)
+int tc_bwd_launches(const Problem& p, bool tau)
 {
-    const size_t BH = (size_t)p.B * p.H, G = (size_t)p.M / 64;
-    return (2 * BH * G * 128 * 64 + BH * p.N + 2 * BH * G) * sizeof(float);
+    return (p.causal ? 2 : 4) + (tau ? 1 : 0);
 }
+
+size_t tc_bwd_ws_bytes(const Problem& p) { return bwd_ws(p).total * sizeof(float); }
 
 cudaError_t launch_tc_bwd(const Problem& p, const void* q, const void* k, const void* v,
                           const float* W1, const float* W2, const float* tau, const void* out,
@@ -949,11 +1266,11 @@ cudaError_t launch_tc_bwd(const Problem& p, const void* q, const void* k, const 
                           float* dW1, float* dW2, float* dtau, void* scratch, int* status,
                           cudaStream_t s)
 {
+#define FLEX_BWD_ARGS p, q, k, v, W1, W2, tau, out, den, dout, dq, dk, dv, dW1, dW2, dtau, scratch, status, s
     if (p.nonstat)
-        return launch_bwd<true>(p, q, k, v, W1, W2, tau, out, den, dout, dq, dk, dv, dW1, dW2,
-                                dtau, scratch, status, s);
-    return launch_bwd<false>(p, q, k, v, W1, W2, tau, out, den, dout, dq, dk, dv, dW1, dW2,
-                             dtau, scratch, status, s);
+        return tau ? launch_bwd<true, true>(FLEX_BWD_ARGS) : launch_bwd<true, false>(FLEX_BWD_ARGS);
+    return tau ? launch_bwd<false, true>(FLEX_BWD_ARGS) : launch_bwd<false, false>(FLEX_BWD_ARGS);
+#undef FLEX_BWD_ARGS
 }
 
 }  // namespace flex

@@ -121,7 +121,7 @@ __global__ void __launch_bounds__(kThreadsF)
             }
             tmem_wait_ld();
             if (NS)
-                reduce_2pi_if_needed(a, w);
+                cos_w_args(a, w);  // w <- cos(w)
             else
                 reduce_2pi_if_needed(a);
             uint32_t pc[16], ps[16];
@@ -132,8 +132,8 @@ __global__ void __launch_bounds__(kThreadsF)
                 __sincosf(a[2 * i + 1], &s1, &c1);
                 float k0 = sc, k1 = sc;
                 if (NS) {
-                    k0 *= __cosf(w[2 * i]);
-                    k1 *= __cosf(w[2 * i + 1]);
+                    k0 *= w[2 * i];
+                    k1 *= w[2 * i + 1];
                 }
                 pc[i] = pack_bf16(c0 * k0, c1 * k1);
                 ps[i] = pack_bf16(s0 * k0, s1 * k1);

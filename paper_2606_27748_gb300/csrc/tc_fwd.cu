@@ -402,20 +402,10 @@ __global__ void __maxnreg__(96)
                         __syncwarp();
                         if (lane == 0) mbar_arrive(&bars.p_free);
                     }
-                    if (NS) {
-                        // w <- cos(w): on the FMA pipe (polynomial) when every argument of
-                        // the warp is inside [-2, 2], else reduced + hardware cos
-                        if (__any_sync(0xffffffffu, (or_bits(a) | or_bits(w)) & kAbsGE2)) {
-                            reduce_2pi_all(a);
-#pragma unroll
-                            for (int i = 0; i < 16; ++i) w[i] = __cosf(reduce_2pi(w[i]));
-                        } else {
-#pragma unroll
-                            for (int i = 0; i < 8; ++i) cos_poly2(w[2 * i], w[2 * i + 1]);
-                        }
-                    } else {
+                    if (NS)
+                        cos_w_args(a, w);  // w <- cos(w)
+                    else
                         reduce_2pi_if_needed(a);
-                    }
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
                         float s0, c0, s1, c1;

@@ -132,6 +132,24 @@ __device__ __forceinline__ void cos_poly2(float& x0, float& x1)
     f2_unpack(p, x0, x1);
 }
 
+// Nonstationary feature arguments u (a) and w: reduces them when any lane of the warp holds
+// one with |x| >= 2 and then replaces w by the hardware cos(w); otherwise (every argument
+// inside [-2, 2]) replaces w by cos(w) from the FMA-pipe polynomial.  Either way w holds
+// cos(w) afterwards and a is ready for the hardware sin/cos.  Warp-collective.
+template <int n>
+__device__ __forceinline__ void cos_w_args(float (&a)[n], float (&w)[n])
+{
+    static_assert(n % 2 == 0, "pairs");
+    if (__any_sync(0xffffffffu, (or_bits(a) | or_bits(w)) & kAbsGE2)) {
+        reduce_2pi_all(a);
+#pragma unroll
+        for (int i = 0; i < n; ++i) w[i] = __cosf(reduce_2pi(w[i]));
+    } else {
+#pragma unroll
+        for (int i = 0; i < n / 2; ++i) cos_poly2(w[2 * i], w[2 * i + 1]);
+    }
+}
+
 // Bounded wait on one mbarrier phase.  On a time-out the CTA is told to stop (abort flag)
 // and the status word (if any) records FLEX_ETIMEOUT; every other wait then returns at once.
 __device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,

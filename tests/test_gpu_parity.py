@@ -151,6 +151,20 @@ def test_backward_full_size_head0():
     _compare_grads(w, g0, r)
 
 
+def test_backward_full_size_noncausal_head0():
+    """The non-causal backward on the long-sequence classification shape (8 x 8 x 65536,
+    many chunk splits per sequence), sequences of head 0 against the oracle (dW of head 0
+    sums the whole batch, so it is exact)."""
+    w = WL[3].replace(backward=True)
+    ins = workloads.make_inputs(w)
+    g = _gpu_bwd(w, ins, w.causal)
+    del ins
+    sub = workloads.make_inputs(w, hs=[0])
+    r = oracle.bwd(sub["q"], sub["k"], sub["v"], sub["W1"], sub["W2"], w.causal, sub["dO"])
+    g0 = [t[:, 0:1] for t in g[:3]] + [g[3][0:1], g[4][0:1]]
+    _compare_grads(w, g0, r)
+
+
 @pytest.mark.parametrize("N", [700, 1800, 2000, 4097])
 @pytest.mark.parametrize("w", [WL[1], WL[2]], ids=["stationary", "nonstationary"])
 def test_forward_sequence_splits(w, N):
@@ -167,9 +181,9 @@ def test_forward_sequence_splits(w, N):
 @pytest.mark.parametrize("w", [WL[1], WL[2]], ids=["stationary", "nonstationary"])
 def test_dispatch_launch_counts_and_determinism(w):
     """The tensor-core entry points run (launch counts per call: causal forward 1, non-causal
-    forward 3, causal backward 2), and the backward is bit-for-bit repeatable (dq, dk, dv
-    are sums of at most two groups, each added by the CTA that owns the row, dW is reduced
-    in a fixed order)."""
+    forward 3, causal backward 2, non-causal backward 4), and both backwards are bit-for-bit
+    repeatable (dq, dk, dv are sums of at most two groups, each added by the CTA that owns
+    the row; the non-causal totals and dW are reduced in a fixed order)."""
     ws_ = w.replace(B=2, H=2, N=700, backward=True)
     ins = workloads.make_inputs(ws_)
     n0 = flexattn.kernel_launches()
@@ -182,7 +196,11 @@ def test_dispatch_launch_counts_and_determinism(w):
     g1 = _gpu_bwd(ws_, ins, True)
     assert flexattn.kernel_launches() - n0 == 1 + 2  # the forward it runs first + backward
     g2 = _gpu_bwd(ws_, ins, True)
-    for a, b in zip(g1, g2):
+    n0 = flexattn.kernel_launches()
+    h1 = _gpu_bwd(ws_, ins, False)
+    assert flexattn.kernel_launches() - n0 == 3 + 4  # the non-causal forward + backward
+    h2 = _gpu_bwd(ws_, ins, False)
+    for a, b in list(zip(g1, g2)) + list(zip(h1, h2)):
         if a is None:
             assert b is None
         else:

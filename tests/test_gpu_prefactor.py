@@ -128,26 +128,28 @@ def test_tensor_core_forward_takes_the_prefactor(causal, launches):
     assert_close(to_host(out), ro, "bf16", "out")
 
 
+@pytest.mark.parametrize("causal,launches", [(True, 3), (False, 5)], ids=["causal", "non-causal"])
 @pytest.mark.parametrize("w,M", [(WL[2], 128), (WL[1], 64)], ids=["n-M128", "s-M64"])
-def test_tensor_core_backward_takes_the_prefactor(w, M):
-    """Causal bf16 d = 64 keeps the tensor-core backward with tau: the key-weight pass, the
-    two-pass kernel (bf16 dq, dk, dv written directly) and the dW/dtau reduction (3
-    launches); the result matches the oracle and repeats bit for bit."""
-    _, ins = _setup(w, True, 64, M, "bf16", N=520)
+def test_tensor_core_backward_takes_the_prefactor(w, M, causal, launches):
+    """bf16 d = 64 keeps the tensor-core backward with tau: the key-weight pass, then causal:
+    the two-scan kernel (bf16 dq, dk, dv written directly) and the dW/dtau reduction;
+    non-causal: the partial states, their totals, the gradient kernel and the reduction.
+    The result matches the oracle and repeats bit for bit."""
+    _, ins = _setup(w, causal, 64, M, "bf16", N=520)
     q, k, v, dO, W1, W2, tau = _dev(ins, "bf16")
-    out, den = flexattn.linattn_fwd(q, k, v, W1, W2, True, tau=tau)
+    out, den = flexattn.linattn_fwd(q, k, v, W1, W2, causal, tau=tau)
     shape = flexattn.shape_of(q, W1)
-    ws = flexattn.workspace(shape, True, True)
+    ws = flexattn.workspace(shape, causal, True)
     runs = []
     for _ in range(2):
         n0 = flexattn.kernel_launches()
-        g = flexattn.linattn_bwd(q, k, v, W1, W2, True, out, den, dO, ws=ws, tau=tau)
+        g = flexattn.linattn_bwd(q, k, v, W1, W2, causal, out, den, dO, ws=ws, tau=tau)
         flexattn.check_status(ws)
-        assert flexattn.kernel_launches() - n0 == 3
+        assert flexattn.kernel_launches() - n0 == launches
         runs.append([None if x is None else x.clone() for x in g])
     for a, b in zip(*runs):
         assert (a is None and b is None) or torch.equal(a, b), "not bit-exact repeatable"
-    r = oracle.bwd(ins["q"], ins["k"], ins["v"], ins["W1"], ins["W2"], True, ins["dO"],
+    r = oracle.bwd(ins["q"], ins["k"], ins["v"], ins["W1"], ins["W2"], causal, ins["dO"],
                    tau=ins["tau"])
     g = runs[0]
     for name, x, ref in zip(("dq", "dk", "dv", "dW1", "dW2"), g, r):
