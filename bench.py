@@ -227,7 +227,8 @@ def cpu_cores():
 
 
 def oracle_sample(w, nseq, cores, prefactor=False):
-    """Time the oracle forward over the first `nseq` whole sequences of `w`."""
+    """Time the oracle over the first `nseq` whole sequences of `w`: the forward, and for a
+    training workload (w.backward) the backward after it."""
     import oracle
     nb = -(-nseq // w.H)
     ins = workloads.make_inputs(w, bs=range(nb))
@@ -238,8 +239,11 @@ def oracle_sample(w, nseq, cores, prefactor=False):
     W1 = ins["W1"][heads]
     W2 = None if ins["W2"] is None else ins["W2"][heads]
     tau = workloads.draw_tau(w)[heads] if prefactor else None
+    dO = ins["dO"].reshape(nb * w.H, w.N, w.d)[None, :nseq] if w.backward else None
     t0 = time.perf_counter()
     oracle.fwd(q, k, v, W1, W2, w.causal, nthreads=cores, tau=tau)
+    if w.backward:
+        oracle.bwd(q, k, v, W1, W2, w.causal, dO, nthreads=cores, tau=tau)
     return time.perf_counter() - t0
 
 
@@ -308,7 +312,8 @@ def run_reference(args, w):
     step = sum(times) / len(times)
     value = nseq * w.N / w.H / step
     line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+        "metric": METRIC_TRAIN if w.backward else METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": step * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "impl": "reference",

@@ -376,6 +376,14 @@ __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
     float *A = sm + L.A, *dA = sm + L.dA, *dAct = sm + L.dAct, *Kc = sm + L.Kc;
     const float itau = tau ? expf(-tau[h]) : 0.f;
     float dtau_acc = 0.f;
+    // |k_0|^2 of the sequence: dtau = -exp(-tau) sum_j (|k_j|^2 - |k_0|^2) s_j (the s_j of a
+    // sequence sum to zero, as every output row is invariant to a common key-weight scale)
+    float n20 = 0.f;
+    if (tau)
+        for (int e = 0; e < d; ++e) {
+            const float x = load_act(k, base + e);
+            n20 = fmaf(x, x, n20);
+        }
 
     float dw_acc[kMaxDwPerThread];
 #pragma unroll
@@ -512,7 +520,7 @@ __global__ void __launch_bounds__(kThreads) simt_bwd_kernel(
                 for (int f = 0; f < D; ++f) sj = fmaf(Pk[j * (D + 1) + f], dP[j * (D + 1) + f], sj);
                 for (int e = 0; e < d; ++e) n2 = fmaf(Xk[j * d + e], Xk[j * d + e], n2);
                 Kc[j] = 2.f * itau * sj;
-                dtau_acc = fmaf(-itau * n2, sj, dtau_acc);
+                dtau_acc = fmaf(-itau * (n2 - n20), sj, dtau_acc);
             }
         if (p.causal) state_update(Pq, Gx, CL, D, d, R);
         feature_backward(p, Xk, Pk, dP, CL, W, dAct);

@@ -524,13 +524,14 @@ __global__ void __launch_bounds__(kThreadsG, 1)
             float dc[16], ds[16], u[16], w[16];
             tmem_ld16(tm_row + L::T_D + 64 * g + 16 * qd, dc);
             tmem_ld16(tm_row + L::T_D + M + 64 * g + 16 * qd, ds);
-            tmem_ld16(tm_row + L::T_S + 16 * qd, u);
-            if (NS) tmem_ld16(tm_row + L::T_S + 64 + 16 * qd, w);
+            float mu, mw = 0.f;  // max |x| per load
+            tmem_ld16_maxabs(tm_row + L::T_S + 16 * qd, u, mu);
+            if (NS) tmem_ld16_maxabs(tm_row + L::T_S + 64 + 16 * qd, w, mw);
             tmem_wait_ld();
             if (NS)
-                reduce_2pi_if_needed(u, w);
+                reduce_2pi_if_needed(u, w, fmaxf(mu, mw));
             else
-                reduce_2pi_if_needed(u);
+                reduce_2pi_if_needed(u, mu);
             uint32_t o1[8], o2[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) {

@@ -136,6 +136,12 @@ __global__ void __launch_bounds__(kThreadsB, 1)
     float* crow = reinterpret_cast<float*>(sm + L::CROW);
     float* spart = reinterpret_cast<float*>(sm + L::SPART);
     const float itau = KW ? expf(-tau[h]) : 0.f;
+    // dtau = -sum_j ln(w_j) s_j with s_j = phi~(k_j) . dphi~(k_j) = dL / d ln(w_j).  Scaling
+    // every key weight of a sequence by one factor leaves every output row unchanged, so the
+    // s_j of a sequence sum to zero and any per-sequence constant may be subtracted from
+    // ln(w_j); the log weight of the sequence's first key removes the common part, whose
+    // terms would otherwise cancel only to the rounding of the s_j.
+    const float lw0 = KW ? logf(kw[(size_t)bh * N]) : 0.f;
     float dtau_acc = 0.f;
 
     // ---- set-up: this group's projection rows, zero state, C16 ----
@@ -248,18 +254,20 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         return commit_wait();
     };
     auto features = [&](uint32_t dst, uint32_t tcol, bool valid, float wsc) {
-        float a[32], w[32];
-        tmem_ld16(tm_row + tcol + 32 * wg, *reinterpret_cast<float(*)[16]>(&a[0]));
-        tmem_ld16(tm_row + tcol + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+        float a[32], w[32], m0, m1, m2 = 0.f, m3 = 0.f;  // m: max |x| per load
+        tmem_ld16_maxabs(tm_row + tcol + 32 * wg, *reinterpret_cast<float(*)[16]>(&a[0]), m0);
+        tmem_ld16_maxabs(tm_row + tcol + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&a[16]), m1);
         if (NS) {
-            tmem_ld16(tm_row + tcol + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]));
-            tmem_ld16(tm_row + tcol + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
+            tmem_ld16_maxabs(tm_row + tcol + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]), m2);
+            tmem_ld16_maxabs(tm_row + tcol + 64 + 32 * wg + 16,
+                             *reinterpret_cast<float(*)[16]>(&w[16]), m3);
         }
         tmem_wait_ld();
+        const float mabs = fmaxf(fmaxf(m0, m1), fmaxf(m2, m3));
         if (NS)
-            cos_w_args(a, w);  // w <- cos(w)
+            cos_w_args(a, w, mabs);  // w <- cos(w)
         else
-            reduce_2pi_if_needed(a);
+            reduce_2pi_if_needed(a, mabs);
         uint32_t pc[16], ps[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
@@ -293,15 +301,18 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         tmem_ld16(tm_row + L::T_D + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&dc[16]));
         tmem_ld16(tm_row + L::T_D + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&ds[0]));
         tmem_ld16(tm_row + L::T_D + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&ds[16]));
-        float a[32], w[32];
+        float a[32], w[32], m0 = 0.f, m1 = 0.f, m2 = 0.f, m3 = 0.f;  // m: max |x| per load
         if (NS) {  // u, w recomputed by a fresh projection in T_P
-            tmem_ld16(tm_row + L::T_P + 32 * wg, *reinterpret_cast<float(*)[16]>(&a[0]));
-            tmem_ld16(tm_row + L::T_P + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
-            tmem_ld16(tm_row + L::T_P + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]));
-            tmem_ld16(tm_row + L::T_P + 64 + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
+            tmem_ld16_maxabs(tm_row + L::T_P + 32 * wg, *reinterpret_cast<float(*)[16]>(&a[0]), m0);
+            tmem_ld16_maxabs(tm_row + L::T_P + 32 * wg + 16, *reinterpret_cast<float(*)[16]>(&a[16]),
+                             m1);
+            tmem_ld16_maxabs(tm_row + L::T_P + 64 + 32 * wg, *reinterpret_cast<float(*)[16]>(&w[0]),
+                             m2);
+            tmem_ld16_maxabs(tm_row + L::T_P + 64 + 32 * wg + 16,
+                             *reinterpret_cast<float(*)[16]>(&w[16]), m3);
         }
         tmem_wait_ld();
-        if (NS) reduce_2pi_if_needed(a, w);
+        if (NS) reduce_2pi_if_needed(a, w, fmaxf(fmaxf(m0, m1), fmaxf(m2, m3)));
         uint32_t cpair[16], spair[16];  // s: this thread's cos / sin features, bf16 pairs
         if (!NS) {
 #pragma unroll
@@ -826,7 +837,9 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 const float sp = feature_backward(sb + L::PK, 1.0f, valid, wk);
                 if (KW) {
                     spart[128 * wg + t] = sp;
-                    dtau_acc = fmaf(-logf(wk), sp, dtau_acc);  // ln w = |k|^2 exp(-tau)
+                    // ln w = |k|^2 exp(-tau), centred on the sequence's first key (the s_j of
+                    // a sequence sum to zero): the cancelling part drops out exactly
+                    dtau_acc = fmaf(lw0 - logf(wk), sp, dtau_acc);
                 }
             }
             handoff();
@@ -1004,7 +1017,9 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                     const float sp = feature_backward(sb + L::PK, 1.0f, valid, wk);
                     if (KW) {
                         spart[128 * wg + t] = sp;
-                        dtau_acc = fmaf(-logf(wk), sp, dtau_acc);  // ln w = |k|^2 exp(-tau)
+                        // ln w = |k|^2 exp(-tau), centred on the sequence's first key (the s_j of
+                    // a sequence sum to zero): the cancelling part drops out exactly
+                    dtau_acc = fmaf(lw0 - logf(wk), sp, dtau_acc);
                     }
                 }
                 handoff();

@@ -149,6 +149,23 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16])
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// tmem_ld16 that also returns, per thread, the maximum |x| over its 16 values (the load's
+// own reduction, .red.max.abs; checked on GB300 against the stored values).
+__device__ __forceinline__ void tmem_ld16_maxabs(uint32_t taddr, float (&v)[16], float& mabs)
+{
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.red.sync.aligned.32x32b.x16.max.abs.f32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,"
+        "%11,%12,%13,%14,%15}, %16, [%17];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=f"(mabs)
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 // 32 lanes x 32 bits, one column.
 __device__ __forceinline__ float tmem_ld1(uint32_t taddr)
 {

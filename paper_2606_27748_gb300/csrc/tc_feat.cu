@@ -111,19 +111,20 @@ __global__ void __launch_bounds__(kThreadsF)
         const float sc = scale * ((rowscale && valid) ? rowscale[(size_t)bh * N + row] : 1.f);
         __nv_bfloat16* out = phi + ((size_t)bh * N + (valid ? row : 0)) * 2 * M;
         for (int g = 0; g < G; ++g) {
-            float a[32], w[32];
+            float a[32], w[32], m0, m1, m2 = 0.f, m3 = 0.f;  // m: max |x| per load
             const uint32_t col = tm_row + g * P + 32 * wg;
-            tmem_ld16(col, *reinterpret_cast<float(*)[16]>(&a[0]));
-            tmem_ld16(col + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+            tmem_ld16_maxabs(col, *reinterpret_cast<float(*)[16]>(&a[0]), m0);
+            tmem_ld16_maxabs(col + 16, *reinterpret_cast<float(*)[16]>(&a[16]), m1);
             if (NS) {
-                tmem_ld16(col + 64, *reinterpret_cast<float(*)[16]>(&w[0]));
-                tmem_ld16(col + 80, *reinterpret_cast<float(*)[16]>(&w[16]));
+                tmem_ld16_maxabs(col + 64, *reinterpret_cast<float(*)[16]>(&w[0]), m2);
+                tmem_ld16_maxabs(col + 80, *reinterpret_cast<float(*)[16]>(&w[16]), m3);
             }
             tmem_wait_ld();
+            const float mabs = fmaxf(fmaxf(m0, m1), fmaxf(m2, m3));
             if (NS)
-                cos_w_args(a, w);  // w <- cos(w)
+                cos_w_args(a, w, mabs);  // w <- cos(w)
             else
-                reduce_2pi_if_needed(a);
+                reduce_2pi_if_needed(a, mabs);
             uint32_t pc[16], ps[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i) {

@@ -394,8 +394,9 @@ __global__ void __maxnreg__(96)
                         fence_after_sync();
                     }
                     float a[16], w[16];
-                    tmem_ld16(tm_row + L::T_P + (NS ? 0u : 32u * r) + 16 * half, a);
-                    if (NS) tmem_ld16(tm_row + L::T_P + 32 + 16 * half, w);
+                    float ma, mw = 0.f;  // max |x| of this thread's arguments
+                    tmem_ld16_maxabs(tm_row + L::T_P + (NS ? 0u : 32u * r) + 16 * half, a, ma);
+                    if (NS) tmem_ld16_maxabs(tm_row + L::T_P + 32 + 16 * half, w, mw);
                     tmem_wait_ld();
                     if (NS || r == 1) {
                         fence_before_sync();
@@ -403,9 +404,9 @@ __global__ void __maxnreg__(96)
                         if (lane == 0) mbar_arrive(&bars.p_free);
                     }
                     if (NS)
-                        cos_w_args(a, w);  // w <- cos(w)
+                        cos_w_args(a, w, fmaxf(ma, mw));  // w <- cos(w)
                     else
-                        reduce_2pi_if_needed(a);
+                        reduce_2pi_if_needed(a, ma);
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
                         float s0, c0, s1, c1;

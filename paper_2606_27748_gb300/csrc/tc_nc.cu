@@ -257,21 +257,22 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
             if (!bar_wait(&bars.p_full[pb], (j >> 1) & 1, &abort_flag, status)) break;
             fence_after_sync();
             const uint32_t tp = tm_row + (pb ? L::T_P1 : L::T_P0);
-            float a[32], w[32];
-            tmem_ld16(tp + 32 * half, *reinterpret_cast<float(*)[16]>(&a[0]));
-            tmem_ld16(tp + 32 * half + 16, *reinterpret_cast<float(*)[16]>(&a[16]));
+            float a[32], w[32], m0, m1, m2 = 0.f, m3 = 0.f;  // m: max |x| per load
+            tmem_ld16_maxabs(tp + 32 * half, *reinterpret_cast<float(*)[16]>(&a[0]), m0);
+            tmem_ld16_maxabs(tp + 32 * half + 16, *reinterpret_cast<float(*)[16]>(&a[16]), m1);
             if (NS) {
-                tmem_ld16(tp + 64 + 32 * half, *reinterpret_cast<float(*)[16]>(&w[0]));
-                tmem_ld16(tp + 64 + 32 * half + 16, *reinterpret_cast<float(*)[16]>(&w[16]));
+                tmem_ld16_maxabs(tp + 64 + 32 * half, *reinterpret_cast<float(*)[16]>(&w[0]), m2);
+                tmem_ld16_maxabs(tp + 64 + 32 * half + 16, *reinterpret_cast<float(*)[16]>(&w[16]), m3);
             }
             tmem_wait_ld();
+            const float mabs = fmaxf(fmaxf(m0, m1), fmaxf(m2, m3));
             fence_before_sync();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars.p_free[pb]);
             if (NS)
-                reduce_2pi_if_needed(a, w);
+                reduce_2pi_if_needed(a, w, mabs);
             else
-                reduce_2pi_if_needed(a);
+                reduce_2pi_if_needed(a, mabs);
             uint32_t pc[16], ps[16];
 #pragma unroll
             for (int e = 0; e < 16; ++e) {

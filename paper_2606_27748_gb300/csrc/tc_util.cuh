@@ -48,23 +48,6 @@ __device__ __forceinline__ float reduce_2pi(float x)
     return fmaf(-n, k2PiLo, fmaf(-n, k2PiHi, x));
 }
 
-// OR of the bit patterns of v, as a balanced tree (the compiler fuses pairs of ORs into
-// three-input logic ops: about n/2 instructions, depth log2 n).  Bit 30 of an fp32 value
-// is the top bit of its exponent field: set exactly when |x| >= 2 (or x is not finite).
-template <int n>
-__device__ __forceinline__ uint32_t or_bits(const float (&v)[n])
-{
-    uint32_t acc[n];
-#pragma unroll
-    for (int i = 0; i < n; ++i) acc[i] = __float_as_uint(v[i]);
-#pragma unroll
-    for (int s = 1; s < n; s *= 2)
-#pragma unroll
-        for (int i = 0; i + s < n; i += 2 * s) acc[i] |= acc[i + s];
-    return acc[0];
-}
-constexpr uint32_t kAbsGE2 = 0x40000000u;
-
 template <int n>
 __device__ __forceinline__ void reduce_2pi_all(float (&v)[n])
 {
@@ -72,19 +55,20 @@ __device__ __forceinline__ void reduce_2pi_all(float (&v)[n])
     for (int i = 0; i < n; ++i) v[i] = reduce_2pi(v[i]);
 }
 
-// Reduces every value of a (and of w) when any lane of the warp holds one with |x| >= 2:
-// inside [-2, 2] (a subset of [-pi, pi], where the hardware sin/cos keeps its 2^-21
-// bound) the step is skipped, for about half an instruction per value.  Warp-collective:
-// all 32 lanes call it together.
+// The range test: `mabs` is this thread's max |x| over its arguments, as the tensor-memory
+// load returns it (tmem_ld16_maxabs).  Reduces every value of a (and of w) when any lane of
+// the warp holds one with |x| >= 2 (or not finite); inside [-2, 2] (a subset of [-pi, pi],
+// where the hardware sin/cos keeps its 2^-21 bound) the step is skipped for one compare and
+// one vote.  Warp-collective: all 32 lanes call it together.
 template <int n>
-__device__ __forceinline__ void reduce_2pi_if_needed(float (&a)[n])
+__device__ __forceinline__ void reduce_2pi_if_needed(float (&a)[n], float mabs)
 {
-    if (__any_sync(0xffffffffu, or_bits(a) & kAbsGE2)) reduce_2pi_all(a);
+    if (__any_sync(0xffffffffu, !(mabs < 2.f))) reduce_2pi_all(a);
 }
 template <int n>
-__device__ __forceinline__ void reduce_2pi_if_needed(float (&a)[n], float (&w)[n])
+__device__ __forceinline__ void reduce_2pi_if_needed(float (&a)[n], float (&w)[n], float mabs)
 {
-    if (__any_sync(0xffffffffu, (or_bits(a) | or_bits(w)) & kAbsGE2)) {
+    if (__any_sync(0xffffffffu, !(mabs < 2.f))) {
         reduce_2pi_all(a);
         reduce_2pi_all(w);
     }
@@ -132,15 +116,15 @@ __device__ __forceinline__ void cos_poly2(float& x0, float& x1)
     f2_unpack(p, x0, x1);
 }
 
-// Nonstationary feature arguments u (a) and w: reduces them when any lane of the warp holds
-// one with |x| >= 2 and then replaces w by the hardware cos(w); otherwise (every argument
-// inside [-2, 2]) replaces w by cos(w) from the FMA-pipe polynomial.  Either way w holds
-// cos(w) afterwards and a is ready for the hardware sin/cos.  Warp-collective.
+// Nonstationary feature arguments u (a) and w, with mabs the max |x| over both: when any
+// lane holds one with |x| >= 2 (or not finite), both are reduced and w is replaced by the
+// hardware cos(w); otherwise w is replaced by cos(w) from the FMA-pipe polynomial.  Either
+// way w holds cos(w) afterwards and a is ready for the hardware sin/cos.  Warp-collective.
 template <int n>
-__device__ __forceinline__ void cos_w_args(float (&a)[n], float (&w)[n])
+__device__ __forceinline__ void cos_w_args(float (&a)[n], float (&w)[n], float mabs)
 {
     static_assert(n % 2 == 0, "pairs");
-    if (__any_sync(0xffffffffu, (or_bits(a) | or_bits(w)) & kAbsGE2)) {
+    if (__any_sync(0xffffffffu, !(mabs < 2.f))) {
         reduce_2pi_all(a);
 #pragma unroll
         for (int i = 0; i < n; ++i) w[i] = __cosf(reduce_2pi(w[i]));

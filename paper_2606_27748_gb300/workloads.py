@@ -86,6 +86,11 @@ WORKLOADS[DECODE.name] = DECODE
 AWD = Workload("n_awd_bf16_B32H8N512_d64M64", "n", False, "bf16", 32, 8, 512, 64, 64,
                64 ** -0.25, "normal", 7, awd=True)
 WORKLOADS[AWD.name] = AWD
+# A training step (forward + backward) on the long-sequence classification shape: the
+# non-causal backward.
+NONCAUSAL_TRAIN = ORDERED[3].replace(name="n_noncausal_train_bf16_B8H8N65536_d64M64",
+                                     backward=True)
+WORKLOADS[NONCAUSAL_TRAIN.name] = NONCAUSAL_TRAIN
 # One distillation training step on the same batch: the loss and its gradient with respect
 # to the kernel's parameters (W1, W2; tau with the prefactor).
 AWD_TRAIN = AWD.replace(name="n_awd_train_bf16_B32H8N512_d64M64", backward=True)

@@ -8,7 +8,7 @@ import torch
 
 import oracle
 from paper_2606_27748_gb300 import flexattn, workloads
-from parity import F32_REL_L2, assert_close, rel_l2, to_dev, to_host
+from parity import BF16_REL_L2, F32_REL_L2, assert_close, rel_l2, to_dev, to_host
 
 pytestmark = pytest.mark.gpu
 
@@ -75,11 +75,11 @@ def test_backward_with_prefactor(w, causal, d, M, dtype):
             continue
         scale = 1.0 if name in ("dq", "dk", "dv") else float(np.sqrt(np.mean(ref * ref)))
         assert_close(to_host(x), ref, dtype, name, max_abs_scale=scale)
-    # dtau is ill-conditioned: keys of equal norm give dtau = 0 exactly, so it is the small
-    # remainder of a sum over every key whose terms carry the bf16 rounding of the stored
-    # out that the backward reads.  fp32 storage: the usual 1e-4; bf16: rel L2 <= 5e-2.
+    # dtau is the remainder of a sum over every key that cancels exactly when the key norms
+    # are equal; the kernels subtract that common part exactly (the s_j of a sequence sum to
+    # zero), so dtau keeps the stated tolerances.
     err = rel_l2(to_host(g[5]), r[5])
-    assert err <= (F32_REL_L2 if dtype == "f32" else 5e-2), f"dtau: rel L2 {err:.3e}"
+    assert err <= (F32_REL_L2 if dtype == "f32" else BF16_REL_L2), f"dtau: rel L2 {err:.3e}"
 
 
 @pytest.mark.parametrize("w,causal,d,M,dtype", [c for c in _cases() if c[1]],
@@ -158,4 +158,4 @@ def test_tensor_core_backward_takes_the_prefactor(w, M, causal, launches):
         scale = 1.0 if name in ("dq", "dk", "dv") else float(np.sqrt(np.mean(ref * ref)))
         assert_close(to_host(x), ref, "bf16", name, max_abs_scale=scale)
     err = rel_l2(to_host(g[5]), r[5])
-    assert err <= 5e-2, f"dtau: rel L2 {err:.3e}"
+    assert err <= BF16_REL_L2, f"dtau: rel L2 {err:.3e}"
