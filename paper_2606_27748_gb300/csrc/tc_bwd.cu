@@ -382,8 +382,10 @@ __global__ void __launch_bounds__(kThreadsB, 1)
         return NS ? sdot * wkey : sdot;  // n: phi~ = w cos u cos w, w sin u cos w
     };
     // dx = da W (T_A[0,64)) and dW = da^T x: n: this chunk's in T_A[64,128); s: summed
-    // over the chunks in the projection's unused half, T_P[64,128)
-    constexpr uint32_t T_DW = NS ? L::T_A + 64 : L::T_P + 64;
+    // over the chunks in the projection's unused half, T_P[64,128); n in kGrad: summed in
+    // T_S, which holds no state without a scan
+    constexpr bool kDwPerChunk = NS && MODE != kGrad;
+    constexpr uint32_t T_DW = kDwPerChunk ? L::T_A + 64 : (NS ? L::T_S : L::T_P + 64);
     auto project_back = [&](uint64_t d_da, uint64_t d_da_mn, uint64_t d_x_mn, bool first) {
         if (tid == 0) {
             fence_after_sync();
@@ -394,7 +396,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
 #pragma unroll
             for (int ks = 0; ks < 8; ++ks)
                 mma_bf16(tm + T_DW, adv(d_da_mn, ks * 2048), adv(d_x_mn, ks * 2048), I_MM64,
-                         (NS ? ks > 0 : (!first || ks > 0)) ? 1u : 0u);
+                         (kDwPerChunk ? ks > 0 : (!first || ks > 0)) ? 1u : 0u);
         }
         return commit_wait();
     };
@@ -898,45 +900,66 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             if (wg == 0) zr[t] = st[64];
             signal_ready();  // this CTA's receive regions are free for the first exchange
         }
+        // The tiles of chunk c + 1 are loaded while chunk c is worked on, each as soon as its
+        // region is free: dout, out once g is built, q after its last MMA (the projection,
+        // or in kGrad the projection backward); k after its projection (kState) or once the
+        // dk rows are sent (kGrad), v after the MMA that reads it.
+        const uint32_t nc_bytes = (fq ? 3 : 2) * kTileBytes;
+        if (tid == 0 && cbeg < cend) {
+            mbar_arrive_expect_tx(&tma_bar, nc_bytes);
+            if (fq) {
+                load_tile(L::Q, &tmap_q, cbeg);
+                load_tile(L::DO, &tmap_do, cbeg);
+                load_tile(L::O, &tmap_o, cbeg);
+            } else {
+                load_tile(L::K, &tmap_k, cbeg);
+                load_tile(L::V, &tmap_v, cbeg);
+            }
+        }
+        tma_outstanding = cbeg < cend;
         for (int c = cbeg; c < cend; ++c) {
             const int it = c - cbeg;
+            const bool has_next = c + 1 < cend;
             const int t0 = c * kC, CL = min(kC, N - t0);
             const bool valid = t < CL;
             const float wk = (KW && !fq && valid) ? kw[(size_t)bh * N + t0 + t] : 1.f;
             const float den_t = (fq && valid) ? den[(size_t)bh * N + t0 + t] : 1.f;
-            // ---- this chunk's tiles (rows past N read as zero); the next into L2 ----
-            if (tid == 0) {
-                if (c + 1 < cend) {
-                    const size_t off = base + (size_t)(c + 1) * kC * 64;
-                    const uint32_t bytes = (uint32_t)min(kC, N - (c + 1) * kC) * 128;
-                    if (fq) {
-                        prefetch_l2(q + off, bytes);
-                        prefetch_l2(dout + off, bytes);
-                        prefetch_l2(outp + off, bytes);
-                    } else {
-                        prefetch_l2(k + off, bytes);
-                        prefetch_l2(v + off, bytes);
-                    }
-                }
-                mbar_arrive_expect_tx(&tma_bar, (fq ? 3 : 2) * kTileBytes);
+            if (tid == 0 && c + 2 < cend) {  // the chunk after next into L2
+                const size_t off = base + (size_t)(c + 2) * kC * 64;
+                const uint32_t bytes = (uint32_t)min(kC, N - (c + 2) * kC) * 128;
                 if (fq) {
-                    load_tile(L::Q, &tmap_q, c);
-                    load_tile(L::DO, &tmap_do, c);
-                    load_tile(L::O, &tmap_o, c);
+                    prefetch_l2(q + off, bytes);
+                    prefetch_l2(dout + off, bytes);
+                    prefetch_l2(outp + off, bytes);
                 } else {
-                    load_tile(L::K, &tmap_k, c);
-                    load_tile(L::V, &tmap_v, c);
+                    prefetch_l2(k + off, bytes);
+                    prefetch_l2(v + off, bytes);
                 }
             }
-            tma_outstanding = true;
+            // arms the next chunk's loads at its first issue point
+            auto arm_next = [&]() {
+                if (tid == 0 && has_next) mbar_arrive_expect_tx(&tma_bar, nc_bytes);
+                tma_outstanding = has_next;
+            };
             if (!bar_wait(&tma_bar, tma_phase, &abort_flag, status)) goto done;
             tma_phase ^= 1;
             tma_outstanding = false;
             // g, c (and for the state [R | r] the c rows of C16: high and low bf16 parts, so r
             // carries c to ~2^-17 like the exact-cancelling term g . v)
-            if (fq) build_g(valid, den_t, PASS == kPassR, MODE == kState);
+            if (fq) {
+                build_g(valid, den_t, PASS == kPassR, MODE == kState);
+                arm_next();
+                if (tid == 0 && has_next) {  // DO, O are free
+                    load_tile(L::DO, &tmap_do, c + 1);
+                    load_tile(L::O, &tmap_o, c + 1);
+                }
+            }
             // ---- features of the tile's rows (q or k) for this group ----
             if (!project(fq ? dQ : dK)) goto done;
+            if (MODE == kState) {  // the projection was the tile's last use
+                if (!fq) arm_next();
+                if (tid == 0 && has_next) load_tile(fq ? L::Q : L::K, fq ? &tmap_q : &tmap_k, c + 1);
+            }
             features(fq ? sb + L::PQ : sb + L::PK, L::T_P, valid, fq ? 1.f : wk);
             handoff();
             if (MODE == kState) {
@@ -953,6 +976,7 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                     }
                 }
                 if (!commit_wait()) goto done;
+                if (!fq && tid == 0 && has_next) load_tile(L::V, &tmap_v, c + 1);  // V is free
                 continue;
             }
             if (PASS == kPassF) {
@@ -977,12 +1001,13 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                     signal_ready();
                 }
                 if (!project_back(dPQ, dPQmn, dQmn, it == 0)) goto done;
+                if (tid == 0 && has_next) load_tile(L::Q, &tmap_q, c + 1);  // Q is free
                 // the partner has read the previous chunk's rows staged in K
                 if (CS > 1 && !wait_done(it > 0)) goto done;
                 if (!send_rows(dx_out, t0, valid, 0.f, 0, sb + L::K, sb + L::PK)) goto done;
                 prev_t0 = t0;
                 prev_CL = CL;
-                if (NS) dw_accumulate(it == 0);
+                if (kDwPerChunk) dw_accumulate(it == 0);
                 handoff();
             } else {
                 // the previous chunk's dk rows (received in O), before T_A is overwritten;
@@ -1010,6 +1035,8 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                                  adv(dSLmn, ks * 2048), I_KM64, 1u);
                 }
                 if (!commit_wait()) goto done;
+                arm_next();
+                if (tid == 0 && has_next) load_tile(L::V, &tmap_v, c + 1);  // V is free
                 // the partner has read the previous chunk's rows staged in Q and DA2
                 if (CS > 1 && !wait_done(it > 0)) goto done;
                 if (!send_rows(dv, t0, valid, 0.f, 0, sb + L::Q, sb + L::DO)) goto done;
@@ -1028,9 +1055,10 @@ __global__ void __launch_bounds__(kThreadsB, 1)
                 if (!send_rows(dx_out, t0, valid, KW ? 2.f * itau * (spart[t] + spart[128 + t]) : 0.f,
                                1, sb + L::DA2, sb + L::O))
                     goto done;
+                if (tid == 0 && has_next) load_tile(L::K, &tmap_k, c + 1);  // K is free
                 prev_t0 = t0;
                 prev_CL = CL;
-                if (NS) dw_accumulate(it == 0);
+                if (kDwPerChunk) dw_accumulate(it == 0);
                 handoff();
             }
         }
@@ -1054,7 +1082,8 @@ __global__ void __launch_bounds__(kThreadsB, 1)
             goto done;  // the last chunk's dq (F) or dk (R) rows
         }
     }
-    if (MODE != kState && !NS) dw_accumulate(true);  // s: the sum over the chunks, T_P[64,128)
+    // s (and n in kGrad): the sum over the chunks, held in tensor memory
+    if (MODE != kState && !kDwPerChunk) dw_accumulate(true);
     if (KW && MODE != kState) {  // this CTA's dtau (pass R; 0 in pass F): warps, then in order
         for (int o = 16; o > 0; o >>= 1) dtau_acc += __shfl_xor_sync(0xffffffffu, dtau_acc, o);
         __syncthreads();
