@@ -29,13 +29,16 @@
 // adds 2 exp(-tau) s_j k_j to dk_j (folded into the same row adds) and -ln(w_j) s_j to
 // dtau (per-CTA slots, reduced with dW in a fixed order).
 //
-// Phases are serialised: all 256 threads load, compute features and run the CUDA-core
-// epilogues; thread 0 issues the MMAs; one mbarrier tracks their completion (bounded waits).
+// Phases run in order inside a CTA: all 256 threads load, compute features and run the
+// CUDA-core epilogues; thread 0 issues the MMAs; one mbarrier tracks their completion
+// (bounded waits).  The next chunk's q / k / v / dout / out tiles are loaded as soon as
+// the region each one occupies is free, and each exchange is sent at once and finished
+// later (dq and dk rows at the start of the next chunk, dv before the projection
+// backward), so the copies and the partner's progress overlap this CTA's work.
 //
-// Exchange regions (per chunk; each freed by this CTA before it tells the partner "ready"):
-// pass F receives dq in DO (free once g is built) and stages in PQ (free after the
-// projection backward); pass R receives dv in DO and dk in O (bf16 A, free after the
-// gradient MMAs) and stages dv in Q and dk in DA2 (bf16 dA, free at the same point).
+// Exchange regions (staging -> the partner's receive region; each free when it is used):
+//   causal   pass F  dq: PQ -> PK        pass R  dv: PQ -> DA2, dk: PQ+16K -> GT
+//   kGrad    pass F  dq: K  -> PK        pass R  dv: Q  -> DO,  dk: DA2 -> O
 //
 // Tensor memory (512 columns): [0,128) projection, [128,256) A / dA (bf16 in place) then
 // dx (0-63) and the chunk's dW (64-127), [256,384) dphi, [384,464) S|z or R|r.
