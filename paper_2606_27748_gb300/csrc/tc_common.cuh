@@ -202,6 +202,14 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t* r)
                  : "memory");
 }
 
+// 32 lanes x 32 bits, 4 consecutive columns, from registers into tensor memory.
+__device__ __forceinline__ void tmem_st4(uint32_t taddr, const uint32_t* r)
+{
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};" ::"r"(taddr),
+                 "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3])
+                 : "memory");
+}
+
 __device__ __forceinline__ void tmem_wait_st()
 {
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
@@ -233,6 +241,20 @@ __device__ __forceinline__ uint32_t mbar_try_wait(void* mbar, uint32_t parity)
     return ok;
 }
 
+// Non-blocking test of one phase (returns at once, whether or not it has completed).
+__device__ __forceinline__ uint32_t mbar_test_wait(void* mbar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(mbar)), "r"(parity)
+        : "memory");
+    return ok;
+}
+
 __device__ __forceinline__ void mbar_arrive(void* mbar)
 {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(mbar)) : "memory");
@@ -255,6 +277,54 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const void* tmap, int 
         "{%2, %3, %4}], [%5];" ::"r"(dst),
         "l"((uint64_t)tmap), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(mbar))
         : "memory");
+}
+
+// TMA: store a 3-D tile from shared memory (same tensor-map layout as the load), tracked by
+// the issuing thread's bulk groups.  Rows outside the tensor are not written.
+__device__ __forceinline__ void tma_store_3d(const void* tmap, uint32_t src, int c0, int c1, int c2)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.3d.global.shared::cta.tile.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+            (uint64_t)tmap),
+        "r"(src), "r"(c0), "r"(c1), "r"(c2)
+        : "memory");
+}
+__device__ __forceinline__ void bulk_commit_group()
+{
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// Until at most N of this thread's bulk groups are still reading their shared source.
+template <int N>
+__device__ __forceinline__ void bulk_wait_group_read()
+{
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// Until at most N of this thread's bulk groups are incomplete.
+template <int N>
+__device__ __forceinline__ void bulk_wait_group()
+{
+    asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Named barrier `id` over `nthreads` threads (a multiple of 32) that also returns the AND of
+// every thread's `pred`: threads that must take the same branch agree on it here.  The
+// non-aligned form: the threads of a warp need not arrive together.
+__device__ __forceinline__ bool bar_and(int id, int nthreads, bool pred)
+{
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "barrier.cta.red.and.pred q, %2, %3, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}\n"
+        : "=r"(r)
+        : "r"((uint32_t)pred), "r"(id), "r"(nthreads)
+        : "memory");
+    return r != 0;
+}
+__device__ __forceinline__ void bar_named(int id, int nthreads)
+{
+    asm volatile("barrier.cta.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
 // TMA: prefetch a 3-D tile into L2 (no shared memory, no completion tracking).

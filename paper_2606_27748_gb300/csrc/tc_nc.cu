@@ -16,10 +16,13 @@
 // K-major [S | z] snapshot, so the denominator comes out as column 64 of the output.
 // Features are unscaled (the M^{-1/2} of Eq. phi_n / phi_non cancels); den = den' / M.
 //
-// Warp roles (448 threads): warp 0 TMA, warp 1 MMA issue, warps 2-9 features (warps 2-5
-// frequencies 0-31 of a group, 6-9 frequencies 32-63), warps 10-13 epilogue.  Projection
-// buffers (TMEM) and feature tiles (shared memory) are double-buffered, so the feature
-// warps compute job j+1 while the tensor core consumes job j.
+// Warp roles (736 threads): warp 0 TMA of the q or k tiles, warp 1 issues the projection
+// MMAs, warp 22 the state (or output) MMAs, warps 2-17 features (four per lane quadrant,
+// warp 2 + 4 fq + r' taking frequencies 16 fq .. 16 fq + 15 of a group), warps 18-21
+// epilogue (state mode: warp 21 first issues the v tiles' TMA; output mode: rows staged in
+// shared memory and written by TMA stores).  Projection buffers (TMEM) and feature tiles
+// (shared memory) are double-buffered, so the feature warps compute job j+1 while the
+// tensor core consumes job j.
 #include <cuda.h>
 
 #include <algorithm>
@@ -33,8 +36,9 @@ namespace {
 using namespace tc;
 
 constexpr int kC = 128;
-constexpr int kThreadsNC = 448;
-constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kWarpEW = 10;
+constexpr int kThreadsNC = 736;  // 23 warps
+constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kNumFW = 16, kWarpEW = 18, kWarpCons = 22;
+constexpr int kAhead = 4;  // chunks prefetched into L2 ahead of their tile load
 constexpr int kSMs = 152;
 constexpr int kTargetUnits = 8 * kSMs;  // most work units per launch
 constexpr int kSetupChunks = 5;         // fixed cost of a unit, in chunk times
@@ -87,7 +91,6 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
     const int nch = (N + kC - 1) / kC;
     const int c0 = (int)((long long)sp * nch / splits), c1 = (int)((long long)(sp + 1) * nch / splits);
     const int nc = c1 - c0;  // chunks of this unit (>= 1: splits <= nch)
-    const size_t base = (size_t)bh * N * 64;
 
     // ---- set-up: frequencies, [V | 1] ones block, [S | z] snapshot (output phase) ----
     for (int idx = tid; idx < G * L::P * 8; idx += kThreadsNC) {
@@ -132,8 +135,8 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
             mbar_init(&bars.v_full[i], 1);
             mbar_init(&bars.v_free[i], 1);
             mbar_init(&bars.p_full[i], 1);
-            mbar_init(&bars.p_free[i], 8);
-            mbar_init(&bars.phi_full[i], 8);
+            mbar_init(&bars.p_free[i], kNumFW);
+            mbar_init(&bars.phi_full[i], kNumFW);
             mbar_init(&bars.phi_free[i], 1);
             mbar_init(&bars.o_full[i], 1);
             mbar_init(&bars.o_free[i], 4);
@@ -154,31 +157,22 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
     const int njobs = nc * G;
 
     if (warp == kWarpTMA) {
+        // q or k tiles (v has its own thread: a v buffer frees late, after the state MMA two
+        // chunks back, and must not hold up the next projection's tile)
         if (lane == 0) {
-            uint32_t ph_x[2] = {0, 0}, ph_v[2] = {0, 0};
+            uint32_t ph_x[2] = {0, 0};
             for (int i = 0; i < nc; ++i) {
                 const int b = i & 1, t0 = (c0 + i) * kC;
-                if (i + 2 < nc) {  // two chunks ahead into L2
-                    tma_prefetch_3d(&tmap_x, 0, t0 + 2 * kC, bh);
-                    if (MODE == kState) tma_prefetch_3d(&tmap_v, 0, t0 + 2 * kC, bh);
-                }
+                if (i + kAhead < nc) tma_prefetch_3d(&tmap_x, 0, t0 + kAhead * kC, bh);  // into L2
                 if (i >= 2) {
                     if (!bar_wait(&bars.x_free[b], ph_x[b], &abort_flag, status)) break;
                     ph_x[b] ^= 1;
                 }
                 mbar_arrive_expect_tx(&bars.x_full[b], kTileBytes);
                 tma_load_3d(sb + (b ? L::X1 : L::X0), &tmap_x, 0, t0, bh, &bars.x_full[b]);
-                if (MODE == kState) {
-                    if (i >= 2) {
-                        if (!bar_wait(&bars.v_free[b], ph_v[b], &abort_flag, status)) break;
-                        ph_v[b] ^= 1;
-                    }
-                    mbar_arrive_expect_tx(&bars.v_full[b], kTileBytes);
-                    tma_load_3d(sb + (b ? L::V1 : L::V0), &tmap_v, 0, t0, bh, &bars.v_full[b]);
-                }
             }
         }
-    } else if (warp == kWarpMMA) {
+    } else if (warp == kWarpMMA || warp == kWarpCons) {
         if (lane == 0) {
             constexpr uint32_t I_PROJ = idesc_bf16(128, L::P, 0, 0);
             constexpr uint32_t I_KV = idesc_bf16(128, 80, 1, 1);
@@ -226,7 +220,10 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
                     if (g == G - 1) mma_commit(&bars.o_full[ib]);
                 }
             };
-            for (int j = 0; j < njobs && ok; ++j) {
+            // Projections and the state / output MMAs come from two threads, so a late v
+            // tile (the state MMA of job j waits for it) never holds up the projection of
+            // job j + 2 that the feature warps will want next.
+            for (int j = 0; j < njobs && ok && warp == kWarpMMA; ++j) {
                 const int i = j / G, g = j % G, pb = j & 1, ib = i & 1;
                 if (g == 0) wait(&bars.x_full[ib], (i >> 1) & 1);
                 if (j >= 2) wait(&bars.p_free[pb], ((j - 2) >> 1) & 1);
@@ -239,14 +236,20 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
                              I_PROJ, ks > 0);
                 mma_commit(&bars.p_full[pb]);
                 if (g == G - 1) mma_commit(&bars.x_free[ib]);
-                if (j >= 1) consume(j - 1);
             }
-            if (ok) consume(njobs - 1);
-            if (ok && MODE == kState) mma_commit(&bars.state_done);
+            if (warp == kWarpCons) {
+                for (int j = 0; j < njobs && ok; ++j) consume(j);
+                if (ok && MODE == kState) mma_commit(&bars.state_done);
+            }
         }
     } else if (warp < kWarpEW) {
         // ================= features =================
-        const int half = (warp - kWarpFW) >> 2, quad = warp & 3, t = 32 * quad + lane;
+        // Four warps per lane quadrant, each on 16 frequencies of the job's group: with four
+        // warps per scheduler one warp's tensor-memory read or sin/cos latency is covered by
+        // the others.  Frequencies 16 fq + 2e, + 1 -> pair e of 16-byte chunks 2 fq, 2 fq + 1
+        // of the cos and sin blocks.  n: cos(w) by the FMA-pipe polynomial when every argument
+        // of the warp is inside [-2, 2].
+        const int fq = (warp - kWarpFW) >> 2, quad = warp & 3, t = 32 * quad + lane;
         const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
         for (int j = 0; j < njobs; ++j) {
             const int i = j / G, pb = j & 1;
@@ -256,31 +259,26 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
                                  ? kw[(size_t)bh * N + (size_t)(c0 + i) * kC + t] : 1.f;
             if (!bar_wait(&bars.p_full[pb], (j >> 1) & 1, &abort_flag, status)) break;
             fence_after_sync();
-            const uint32_t tp = tm_row + (pb ? L::T_P1 : L::T_P0);
-            float a[32], w[32], m0, m1, m2 = 0.f, m3 = 0.f;  // m: max |x| per load
-            tmem_ld16_maxabs(tp + 32 * half, *reinterpret_cast<float(*)[16]>(&a[0]), m0);
-            tmem_ld16_maxabs(tp + 32 * half + 16, *reinterpret_cast<float(*)[16]>(&a[16]), m1);
-            if (NS) {
-                tmem_ld16_maxabs(tp + 64 + 32 * half, *reinterpret_cast<float(*)[16]>(&w[0]), m2);
-                tmem_ld16_maxabs(tp + 64 + 32 * half + 16, *reinterpret_cast<float(*)[16]>(&w[16]), m3);
-            }
+            const uint32_t tp = tm_row + (pb ? L::T_P1 : L::T_P0) + 16 * fq;
+            float a[16], w[16], ma, mw = 0.f;  // max |x| of each load
+            tmem_ld16_maxabs(tp, a, ma);
+            if (NS) tmem_ld16_maxabs(tp + 64, w, mw);
             tmem_wait_ld();
-            const float mabs = fmaxf(fmaxf(m0, m1), fmaxf(m2, m3));
             fence_before_sync();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars.p_free[pb]);
             if (NS)
-                reduce_2pi_if_needed(a, w, mabs);
+                cos_w_args(a, w, fmaxf(ma, mw));  // w <- cos(w)
             else
-                reduce_2pi_if_needed(a, mabs);
-            uint32_t pc[16], ps[16];
+                reduce_2pi_if_needed(a, ma);
+            uint32_t pc[8], ps[8];
 #pragma unroll
-            for (int e = 0; e < 16; ++e) {
+            for (int e = 0; e < 8; ++e) {
                 float s0, cc0, s1, cc1;
                 __sincosf(a[2 * e], &s0, &cc0);
                 __sincosf(a[2 * e + 1], &s1, &cc1);
                 if (NS) {
-                    const float cw0 = __cosf(w[2 * e]), cw1 = __cosf(w[2 * e + 1]);
+                    const float cw0 = w[2 * e], cw1 = w[2 * e + 1];
                     cc0 *= cw0; s0 *= cw0; cc1 *= cw1; s1 *= cw1;
                 }
                 if (MODE == kState && KW) { cc0 *= wk; s0 *= wk; cc1 *= wk; s1 *= wk; }
@@ -292,8 +290,8 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
                 break;
             const uint32_t dst = sb + (pb ? L::PB1 : L::PB0);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint32_t off = swz128(t, (4 * half + q) * 8);
+            for (int q = 0; q < 2; ++q) {
+                const uint32_t off = swz128(t, (2 * fq + q) * 8);
                 st_shared_v4(dst + off, pc[4 * q], pc[4 * q + 1], pc[4 * q + 2], pc[4 * q + 3]);
                 st_shared_v4(dst + 16384 + off, ps[4 * q], ps[4 * q + 1], ps[4 * q + 2],
                              ps[4 * q + 3]);
@@ -307,50 +305,92 @@ __global__ void __launch_bounds__(kThreadsNC, 1)
         const int quad = warp & 3, t = 32 * quad + lane;
         const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
         if (MODE == kState) {
+            if (warp == kWarpEW + 3) {
+                // v tiles (tmap_v), issued by this warp's lane 0 before it joins the epilogue
+                if (lane == 0) {
+                    uint32_t ph_v[2] = {0, 0};
+                    for (int i = 0; i < nc; ++i) {
+                        const int b = i & 1, t0 = (c0 + i) * kC;
+                        if (i + kAhead < nc) tma_prefetch_3d(&tmap_v, 0, t0 + kAhead * kC, bh);
+                        if (i >= 2) {
+                            if (!bar_wait(&bars.v_free[b], ph_v[b], &abort_flag, status)) break;
+                            ph_v[b] ^= 1;
+                        }
+                        mbar_arrive_expect_tx(&bars.v_full[b], kTileBytes);
+                        tma_load_3d(sb + (b ? L::V1 : L::V0), &tmap_v, 0, t0, bh, &bars.v_full[b]);
+                    }
+                }
+                __syncwarp();
+            }
             if (bar_wait(&bars.state_done, 0, &abort_flag, status)) {
                 fence_after_sync();
                 float* dst = part + ((size_t)blockIdx.x * G * 128 + t) * kRow;
-#pragma unroll
                 for (int g = 0; g < G; ++g) {
-                    float s_[80];
-#pragma unroll
-                    for (int j = 0; j < 5; ++j)
-                        tmem_ld16(tm_row + L::T_S + 80 * g + 16 * j,
-                                  *reinterpret_cast<float(*)[16]>(&s_[16 * j]));
-                    tmem_wait_ld();
                     float4* d4 = reinterpret_cast<float4*>(dst + (size_t)g * 128 * kRow);
 #pragma unroll
-                    for (int j = 0; j < 20; ++j)
-                        d4[j] = make_float4(s_[4 * j], s_[4 * j + 1], s_[4 * j + 2], s_[4 * j + 3]);
+                    for (int j = 0; j < 5; ++j) {  // 16 columns at a time (register budget)
+                        float s_[16];
+                        tmem_ld16(tm_row + L::T_S + 80 * g + 16 * j, s_);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            d4[4 * j + e] = make_float4(s_[4 * e], s_[4 * e + 1], s_[4 * e + 2],
+                                                        s_[4 * e + 3]);
+                    }
                 }
             }
         } else {
+            // Output rows are staged as bf16 (128-byte swizzle) in the v tiles, unused in this
+            // mode, and written by one TMA store per chunk (tmap_v maps out here): a row per
+            // thread straight to global memory puts 32 cache lines in every warp store, and
+            // the queue they wait in also holds the feature warps' shared-memory stores.
+            // Named barrier 1 joins the 4 epilogue warps; its AND keeps their control flow
+            // the same when a wait gives up.
+            const bool issuer = warp == kWarpEW && lane == 0;
             for (int i = 0; i < nc; ++i) {
                 const int ib = i & 1, t0 = (c0 + i) * kC;
-                if (!bar_wait(&bars.o_full[ib], (i >> 1) & 1, &abort_flag, status)) break;
-                fence_after_sync();
-                float o[64], dn[16];
-                const uint32_t to = tm_row + (ib ? L::T_O1 : L::T_O0);
-#pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    tmem_ld16(to + 16 * j, *reinterpret_cast<float(*)[16]>(&o[16 * j]));
-                tmem_ld16(to + 64, dn);
-                tmem_wait_ld();
-                fence_before_sync();
+                const bool got = bar_wait(&bars.o_full[ib], (i >> 1) & 1, &abort_flag, status);
+                // (the issuer reaches this barrier only after the store that last read
+                // staging buffer ib, two chunks back, has read it)
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&bars.o_free[ib]);
-                if (t < min(kC, N - t0)) {
-                    const float inv = 1.f / dn[0];
-                    uint4* dst = reinterpret_cast<uint4*>(out + base + (size_t)(t0 + t) * 64);
+                if (!bar_and(1, 128, got)) break;
+                fence_after_sync();
+                const uint32_t to = tm_row + (ib ? L::T_O1 : L::T_O0);
+                const uint32_t stg = sb + (ib ? L::V1 : L::V0);
+                float dn = 0.f, inv = 0.f;
 #pragma unroll
-                    for (int cc = 0; cc < 8; ++cc)
-                        dst[cc] = make_uint4(pack_bf16(o[8 * cc] * inv, o[8 * cc + 1] * inv),
-                                             pack_bf16(o[8 * cc + 2] * inv, o[8 * cc + 3] * inv),
-                                             pack_bf16(o[8 * cc + 4] * inv, o[8 * cc + 5] * inv),
-                                             pack_bf16(o[8 * cc + 6] * inv, o[8 * cc + 7] * inv));
-                    if (den) den[(size_t)bh * N + t0 + t] = dn[0] / (float)M;
+                for (int hh = 0; hh < 2; ++hh) {  // 32 output columns at a time
+                    float o[32];
+                    tmem_ld16(to + 32 * hh, *reinterpret_cast<float(*)[16]>(&o[0]));
+                    tmem_ld16(to + 32 * hh + 16, *reinterpret_cast<float(*)[16]>(&o[16]));
+                    if (hh == 0) dn = tmem_ld1(to + 64);
+                    tmem_wait_ld();
+                    if (hh == 1) {
+                        fence_before_sync();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&bars.o_free[ib]);
+                    } else {
+                        inv = 1.f / dn;
+                    }
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc)
+                        st_shared_v4(stg + swz128(t, (4 * hh + cc) * 8),
+                                     pack_bf16(o[8 * cc] * inv, o[8 * cc + 1] * inv),
+                                     pack_bf16(o[8 * cc + 2] * inv, o[8 * cc + 3] * inv),
+                                     pack_bf16(o[8 * cc + 4] * inv, o[8 * cc + 5] * inv),
+                                     pack_bf16(o[8 * cc + 6] * inv, o[8 * cc + 7] * inv));
+                }
+                if (den && t < min(kC, N - t0)) den[(size_t)bh * N + t0 + t] = dn / (float)M;
+                fence_proxy_async();
+                __syncwarp();
+                bar_named(1, 128);
+                if (issuer) {
+                    tma_store_3d(&tmap_v, stg, 0, t0, bh);  // rows past N are not written
+                    bulk_commit_group();
+                    bulk_wait_group_read<1>();
                 }
             }
+            if (issuer) bulk_wait_group<0>();
         }
     }
 
@@ -381,9 +421,9 @@ cudaError_t launch_nc(const Problem& p, const void* q, const void* k, const void
                       void* scratch, int* status, cudaStream_t s)
 {
     const int BH = p.B * p.H, splits = tc_nc_splits(p);
-    CUtensorMap mq, mk, mv;
+    CUtensorMap mq, mk, mv, mo;
     if (!make_act_map(&mq, q, BH, p.N) || !make_act_map(&mk, k, BH, p.N) ||
-        !make_act_map(&mv, v, BH, p.N))
+        !make_act_map(&mv, v, BH, p.N) || !make_act_map(&mo, out, BH, p.N))
         return cudaErrorInvalidValue;
     float* part = static_cast<float*>(scratch);
     float* total = part + (size_t)BH * splits * G * 128 * kRow;
@@ -401,7 +441,7 @@ cudaError_t launch_nc(const Problem& p, const void* q, const void* k, const void
     nc_reduce_kernel<<<(int)std::min<size_t>((n + 255) / 256, 152 * 8), 256, 0, s>>>(BH, splits, G,
                                                                                     part, total);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    k_out<<<BH * splits, kThreadsNC, smem, s>>>(mq, mv, p.H, p.N, p.M, splits, W1, W2, nullptr,
+    k_out<<<BH * splits, kThreadsNC, smem, s>>>(mq, mo, p.H, p.N, p.M, splits, W1, W2, nullptr,
                                                nullptr, total, (__nv_bfloat16*)out, den, status);
     return cudaGetLastError();
 }
