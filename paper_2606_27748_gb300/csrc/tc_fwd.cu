@@ -17,20 +17,23 @@
 // ([cos, sin] instead of M^{-1/2}[cos, sin]): the factor cancels in the output, and only
 // the stored denominator is rescaled (den = den' / M).
 //
-// Warp roles (640 threads), handshakes on mbarriers:
+// Warp roles, handshakes on mbarriers (n: 896 threads, FW = 16 feature warps; s: 640
+// threads, FW = 8):
 //   warp 0      TMA: q and k chunk tiles (128B swizzle) into shared memory
-//   warp 19     TMA: v chunk tiles (a buffer frees late, after A V, and must not hold up
-//               the q and k loads)
 //   warp 1      one thread issues the attention MMAs (numerator, QK, state, A V); owns the
 //               tensor-memory allocation
-//   warp 18     one thread issues the projection MMAs, so they never queue behind an
-//               attention step that has not been issued yet
-//   warps 2-9   features: projection (TMEM) -> cos/sin -> phi(Q) into TMEM (bf16 pairs),
-//               phi(K) into shared memory; per half group of 32 frequencies, warps 2-5
-//               take the first 16, warps 6-9 the last 16
-//   warps 10-17 epilogue, two halves of 4 warps: causal mask + bf16 of A (written back
+//   warps 2 ..  features: projection (TMEM) -> cos/sin -> phi(Q) into TMEM (bf16 pairs),
+//   1 + FW      phi(K) into shared memory; FW / 4 warps per lane quadrant (warp 2 + 4 fq +
+//               r'), warp fq on 64 / (FW / 4) frequencies of the group per feature tile (n,
+//               per half group of 32: 8 fq .. 8 fq + 7 of the half); with four warps per
+//               scheduler the sin/cos unit stays busy while a warp waits on its loads
+//   next 8      epilogue, two halves of 4 warps: causal mask + bf16 of A (written back
 //               into TMEM as the A operand of A V), bf16 snapshot of [S | z] for the next
 //               chunk, partial output rows (own rows, or the partner's rows staged for it)
+//   next        one thread issues the projection MMAs, so they never queue behind an
+//               attention step that has not been issued yet
+//   last        TMA: v chunk tiles (a buffer frees late, after A V, and must not hold up
+//               the q and k loads)
 //
 // Per chunk c the attention issuer runs phi(Q) [S | z] as soon as phi(Q) and the snapshot
 // of the state before c are ready, then phi(Q) phi(K)^T and the state update once phi(K)
@@ -53,7 +56,8 @@
 // is the denominator, built from exactly the bf16 values that build the numerator.
 //
 // Tensor memory (512 columns x 128 lanes, 32-bit):
-//   [0,64)     projection (s: a of the 64 frequencies; n: u, w of 32 frequencies)
+//   [0,64)     projection (s: a of the 64 frequencies; n: u, w of 32 frequencies, as 4
+//              blocks of [u of 8 | w of 8], one per feature warp of a quadrant)
 //   [64,192)   A = phi(Q) phi(K)^T (row = query, col = key); after the epilogue, columns
 //              [0,32) and [64,96) hold bf16(masked A) of keys 0-63 and 64-127, two per column
 //   [192,352)  two buffers of phi(Q) [S | z] + A [V | 1]: numerator 0-63, denominator 64
@@ -70,19 +74,25 @@ namespace {
 using namespace tc;
 
 constexpr int kC = 128;            // tokens per chunk = MMA M
-constexpr int kThreadsTC = 640;    // 20 warps
-constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kWarpEW = 10, kEpiWarps = 8;
-constexpr int kWarpProj = 18, kWarpTMAV = 19;
+constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kEpiWarps = 8;
 
 template <bool NS>
 struct Cfg {
     static constexpr int NH = NS ? 2 : 1;  // projections per feature tile (64 columns each)
+    // Feature warps: n 16 (four per lane quadrant, 72 registers a thread), s 8 (two per
+    // quadrant, 96 registers): the s features are cheap enough that the attention and
+    // epilogue chain sets the chunk period, and it runs faster with the larger budget.
+    static constexpr int FW = NS ? 16 : 8;
+    static constexpr int EW = kWarpFW + FW;        // first epilogue warp
+    static constexpr int PROJ = EW + kEpiWarps;    // projection MMA issuer
+    static constexpr int TMAV = PROJ + 1;          // v tiles
+    static constexpr int THREADS = 32 * (TMAV + 1);
     // shared memory offsets (bytes, 1024-aligned); X0/X1 hold q/k tiles.  VONE is the
     // second 64-column block of [V | 1] (column 0 = 1, the rest 0), reached from either V
     // buffer through the descriptor's leading byte offset.
     static constexpr uint32_t X0 = 0, X1 = 16384, V0 = 32768, V1 = 49152, VONE = 65536;
     // frequencies, bf16 K-major, 64 rows per projection: s: W rows 0-63; n: half h = rows
-    // U(32h..32h+31), V(32h..32h+31)
+    // [U | V] of frequencies 32h + 8fq .. + 7 for fq = 0..3
     static constexpr uint32_t W = 81920;
     static constexpr uint32_t PK = W + 16384;  // phi(K): cos block, sin block (64 features)
     // [S | z] snapshot, MN-major (row = feature): block 0 holds S[f][0..63], block 1 holds
@@ -121,7 +131,7 @@ __device__ __forceinline__ int segment_bound(int nch, int splits, int j)
 // NS: nonstationary features; CS: CTAs per cluster = frequency groups (M / 64); KW: key
 // weights of the norm prefactor given (a compile-time switch: the plain kernel is unchanged).
 template <bool NS, int CS, bool KW>
-__global__ void __maxnreg__(96)
+__global__ void __launch_bounds__(Cfg<NS>::THREADS, 1)
     tc_fwd_causal_kernel(const __grid_constant__ CUtensorMap tmap_q,
                          const __grid_constant__ CUtensorMap tmap_k,
                          const __grid_constant__ CUtensorMap tmap_v, int H, int N, int M,
@@ -147,11 +157,13 @@ __global__ void __maxnreg__(96)
     const size_t base = (size_t)bh * N * 64;
 
     // ---- set-up: frequencies of the group (bf16, K-major rows), ones, zero snapshot ----
-    for (int idx = tid; idx < 128 * 8; idx += kThreadsTC) {
+    for (int idx = tid; idx < 128 * 8; idx += L::THREADS) {
         const int r = idx >> 3, c = idx & 7;
         if (!NS && r >= 64) break;
-        // n: row r of half r/64: U (r%64 < 32) or V of frequency 32 (r/64) + r%32
-        const int f = 64 * rank + (NS ? 32 * (r >> 6) + (r & 31) : r);
+        // n: row r of half h = r/64 belongs to feature warp fq = (r%64)/16: U (r%16 < 8) or
+        // V (r%16 >= 8) of frequency 32 h + 8 fq + r%8, so that warp's u and w are the
+        // adjacent projection columns 16 fq .. 16 fq + 15
+        const int f = 64 * rank + (NS ? 32 * (r >> 6) + 8 * ((r >> 4) & 3) + (r & 7) : r);
         const float* w1 = W1 + ((size_t)h * M + f) * 64 + c * 8;
         float x[8];
         if (!NS) {
@@ -159,19 +171,19 @@ __global__ void __maxnreg__(96)
             for (int e = 0; e < 8; ++e) x[e] = w1[e];
         } else {
             const float* w2 = W2 + ((size_t)h * M + f) * 64 + c * 8;
-            const float sgn = (r & 32) ? -1.f : 1.f;  // U = (W1+W2)/2, V = (W1-W2)/2
+            const float sgn = (r & 8) ? -1.f : 1.f;  // U = (W1+W2)/2, V = (W1-W2)/2
 #pragma unroll
             for (int e = 0; e < 8; ++e) x[e] = 0.5f * (w1[e] + sgn * w2[e]);
         }
         st_shared_v4(sb + L::W + swz128(r, c * 8), pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]),
                      pack_bf16(x[4], x[5]), pack_bf16(x[6], x[7]));
     }
-    for (int idx = tid; idx < 16384 / 16; idx += kThreadsTC)  // [1, 0, ..., 0] rows
+    for (int idx = tid; idx < 16384 / 16; idx += L::THREADS)  // [1, 0, ..., 0] rows
         st_shared_v4(sb + L::VONE + idx * 16, 0, 0, 0, 0);
-    for (int idx = tid; idx < 32768 / 16; idx += kThreadsTC)
+    for (int idx = tid; idx < 32768 / 16; idx += L::THREADS)
         st_shared_v4(sb + L::SX + idx * 16, 0, 0, 0, 0);
     __syncthreads();
-    for (int r = tid; r < kC; r += kThreadsTC)
+    for (int r = tid; r < kC; r += L::THREADS)
         *reinterpret_cast<uint16_t*>(sm + L::VONE + swz128(r, 0)) = 0x3F80u;  // bf16 1.0
     if (tid == 0) {
         for (int i = 0; i < 2; ++i) {
@@ -182,9 +194,9 @@ __global__ void __maxnreg__(96)
             mbar_init(&bars.epi_done[i], kEpiWarps);
         }
         mbar_init(&bars.p_full, 1);
-        mbar_init(&bars.p_free, 8);
-        mbar_init(&bars.phiq_full, 8);
-        mbar_init(&bars.phik_full, 8);
+        mbar_init(&bars.p_free, L::FW);
+        mbar_init(&bars.phiq_full, L::FW);
+        mbar_init(&bars.phik_full, L::FW);
         mbar_init(&bars.phiq_free, 1);
         mbar_init(&bars.phik_free, 1);
         mbar_init(&bars.attn_done, 1);
@@ -218,7 +230,7 @@ __global__ void __maxnreg__(96)
 
     if (abort_flag) {
         // the diagnostic stall ran out during set-up: nothing is issued
-    } else if (warp == kWarpTMAV) {
+    } else if (warp == L::TMAV) {
         // ================= TMA producer: v =================
         if (lane == 0) {
             uint32_t ph_vfree[2] = {0, 0};
@@ -263,7 +275,7 @@ __global__ void __maxnreg__(96)
                 }
             }
         }
-    } else if (warp == kWarpMMA || warp == kWarpProj) {
+    } else if (warp == kWarpMMA || warp == L::PROJ) {
         // ================= MMA issue (one thread per role) =================
         if (lane == 0) {
             constexpr uint32_t I_PROJ = idesc_bf16(128, 64, 0, 0);
@@ -280,7 +292,7 @@ __global__ void __maxnreg__(96)
             // Descriptors are built once; an operand K step adds its byte offset / 16 to
             // the start-address field (addresses stay below 256 KB: no carry out).
             auto adv = [](uint64_t d, uint32_t bytes) { return d + (bytes >> 4); };
-            if (warp == kWarpProj) {
+            if (warp == L::PROJ) {
                 // projections: per chunk q (main chunks) then k, each in NH parts
                 const uint64_t d_x[2] = {sdesc(sb + L::X0, 16, 1024), sdesc(sb + L::X1, 16, 1024)};
                 const uint64_t d_w = sdesc(sb + L::W, 16, 1024);
@@ -370,12 +382,18 @@ __global__ void __maxnreg__(96)
                 }
             }
         }
-    } else if (warp < kWarpEW) {
+    } else if (warp < L::EW) {
         // ================= features =================
-        // Per feature tile two rounds of 16 frequencies: round r covers frequencies
-        // 32r + 16 half .. + 15 (n: the projection of half r holds u in columns 0-31 and w in
-        // 32-63; s: the one projection holds a of all 64 frequencies).
-        const int half = (warp - kWarpFW) >> 2, quad = warp & 3, t = 32 * quad + lane;
+        // FW / 4 warps per lane quadrant; warp fq of a quadrant covers FQ = 64 / (FW / 4)
+        // frequencies of the group per feature tile.  n (FW = 16): per half r (one projection
+        // of 32 frequencies) it reads columns 16 fq .. + 15 = u then w of frequencies
+        // 32 r + 8 fq .. + 7; s: the one projection's columns FQ fq .. + FQ - 1 = a of those
+        // frequencies.  Each 16-column load returns its max |x| for the range test.
+        static_assert(!NS || L::FW == 16, "n: the W rows are ordered for four warps per quadrant");
+        constexpr int FQ = 256 / L::FW;  // frequencies per warp per tile (16 or 32)
+        constexpr int NL = NS ? 1 : FQ / 16;  // 16-column loads per projection
+        constexpr int NPR = NS ? 4 : 8 * NL;  // bf16 pairs per projection
+        const int fq = (warp - kWarpFW) >> 2, quad = warp & 3, t = 32 * quad + lane;
         const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
         uint32_t ph_pfull = 0;
         int n = 0, nq = 0;  // k and q feature tiles produced so far
@@ -385,53 +403,65 @@ __global__ void __maxnreg__(96)
             // key weight of the norm prefactor (phi(k) scaled by it), loaded early
             const float wk = (KW && valid) ? kw[(size_t)bh * N + (size_t)c * kC + t] : 1.f;
             for (int which = main ? 0 : 1; which < 2; ++which) {  // 0: q, 1: k
-                uint32_t pc[16], ps[16];  // [8 r + i]: frequencies 32r + 16 half + 2i, +1
+                // bf16 pairs: pair p = frequencies 2p, 2p + 1 of the warp's FQ (n: pairs
+                // 4r .. 4r + 3 from half r)
+                uint32_t pc[FQ / 2], ps[FQ / 2];
 #pragma unroll
-                for (int r = 0; r < 2; ++r) {
-                    if (NS || r == 0) {
-                        if (!bar_wait(&bars.p_full, ph_pfull, &abort_flag, status)) goto fw_out;
-                        ph_pfull ^= 1;
-                        fence_after_sync();
-                    }
-                    float a[16], w[16];
-                    float ma, mw = 0.f;  // max |x| of this thread's arguments
-                    tmem_ld16_maxabs(tm_row + L::T_P + (NS ? 0u : 32u * r) + 16 * half, a, ma);
-                    if (NS) tmem_ld16_maxabs(tm_row + L::T_P + 32 + 16 * half, w, mw);
+                for (int r = 0; r < L::NH; ++r) {
+                    if (!bar_wait(&bars.p_full, ph_pfull, &abort_flag, status)) goto fw_out;
+                    ph_pfull ^= 1;
+                    fence_after_sync();
+                    float x[NL][16], mabs[NL];
+#pragma unroll
+                    for (int l = 0; l < NL; ++l)
+                        tmem_ld16_maxabs(tm_row + L::T_P + 16 * (NL * fq + l), x[l], mabs[l]);
                     tmem_wait_ld();
-                    if (NS || r == 1) {
-                        fence_before_sync();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&bars.p_free);
-                    }
-                    if (NS)
-                        cos_w_args(a, w, fmaxf(ma, mw));  // w <- cos(w)
-                    else
-                        reduce_2pi_if_needed(a, ma);
+                    fence_before_sync();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&bars.p_free);
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) {
+                    for (int l = 0; l < NL; ++l) {
+                        if (NS)  // x[l][8 ..] <- cos(w)
+                            cos_w_args(*reinterpret_cast<float(*)[8]>(&x[l][0]),
+                                       *reinterpret_cast<float(*)[8]>(&x[l][8]), mabs[l]);
+                        else
+                            reduce_2pi_if_needed(x[l], mabs[l]);
+                    }
+#pragma unroll
+                    for (int i = 0; i < NPR; ++i) {
+                        const float* xl = x[NS ? 0 : i / 8];
+                        const int e = NS ? 2 * i : 2 * (i % 8);
                         float s0, c0, s1, c1;
-                        __sincosf(a[2 * i], &s0, &c0);
-                        __sincosf(a[2 * i + 1], &s1, &c1);
+                        __sincosf(xl[e], &s0, &c0);
+                        __sincosf(xl[e + 1], &s1, &c1);
                         if (NS) {
-                            const float cw0 = w[2 * i], cw1 = w[2 * i + 1];
+                            const float cw0 = xl[8 + e], cw1 = xl[8 + e + 1];
                             c0 *= cw0; s0 *= cw0; c1 *= cw1; s1 *= cw1;
                         }
                         if (KW && which == 1) { c0 *= wk; s0 *= wk; c1 *= wk; s1 *= wk; }
                         if (!valid) { c0 = s0 = c1 = s1 = 0.f; }
-                        pc[8 * r + i] = pack_bf16(c0, c1);
-                        ps[8 * r + i] = pack_bf16(s0, s1);
+                        pc[NPR * r + i] = pack_bf16(c0, c1);
+                        ps[NPR * r + i] = pack_bf16(s0, s1);
                     }
                 }
                 if (which == 0) {
                     // phi(Q) -> tensor memory once the previous chunk's MMAs that read it
-                    // are done; frequencies 32r + 16 half + 2i, +1 -> column 16r + 8 half + i
+                    // are done; column = frequency / 2 (cos), 32 + frequency / 2 (sin)
                     if (nq > 0 && !bar_wait(&bars.phiq_free, (nq - 1) & 1, &abort_flag, status))
                         goto fw_out;
                     fence_after_sync();
+                    if (NS) {
 #pragma unroll
-                    for (int r = 0; r < 2; ++r) {
-                        tmem_st8(tm_row + L::T_Q + 16 * r + 8 * half, &pc[8 * r]);
-                        tmem_st8(tm_row + L::T_Q + 32 + 16 * r + 8 * half, &ps[8 * r]);
+                        for (int r = 0; r < 2; ++r) {
+                            tmem_st4(tm_row + L::T_Q + 16 * r + 4 * fq, &pc[4 * r]);
+                            tmem_st4(tm_row + L::T_Q + 32 + 16 * r + 4 * fq, &ps[4 * r]);
+                        }
+                    } else {
+#pragma unroll
+                        for (int l = 0; l < NL; ++l) {
+                            tmem_st8(tm_row + L::T_Q + FQ / 2 * fq + 8 * l, &pc[8 * l]);
+                            tmem_st8(tm_row + L::T_Q + 32 + FQ / 2 * fq + 8 * l, &ps[8 * l]);
+                        }
                     }
                     tmem_wait_st();
                     fence_before_sync();
@@ -441,18 +471,16 @@ __global__ void __maxnreg__(96)
                 } else {
                     if (n > 0 && !bar_wait(&bars.phik_free, (n - 1) & 1, &abort_flag, status))
                         goto fw_out;
-                    // frequencies 32r + 16 half .. + 15: 16-byte chunks 4r + 2 half, + 1 of the
-                    // cos and sin blocks
+                    // 16-byte chunk m = frequencies 8 m .. 8 m + 7: n: m = 4 j + fq (j = half),
+                    // s: m = FQ / 8 fq + j
 #pragma unroll
-                    for (int r = 0; r < 2; ++r)
-#pragma unroll
-                        for (int j = 0; j < 2; ++j) {
-                            const uint32_t off = swz128(t, (4 * r + 2 * half + j) * 8);
-                            const int b = 8 * r + 4 * j;
-                            st_shared_v4(sb + L::PK + off, pc[b], pc[b + 1], pc[b + 2], pc[b + 3]);
-                            st_shared_v4(sb + L::PK + 16384 + off, ps[b], ps[b + 1], ps[b + 2],
-                                         ps[b + 3]);
-                        }
+                    for (int j = 0; j < FQ / 8; ++j) {
+                        const uint32_t off = swz128(t, (NS ? 4 * j + fq : FQ / 8 * fq + j) * 8);
+                        st_shared_v4(sb + L::PK + off, pc[4 * j], pc[4 * j + 1], pc[4 * j + 2],
+                                     pc[4 * j + 3]);
+                        st_shared_v4(sb + L::PK + 16384 + off, ps[4 * j], ps[4 * j + 1],
+                                     ps[4 * j + 2], ps[4 * j + 3]);
+                    }
                     fence_proxy_async();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(&bars.phik_full);
@@ -468,7 +496,7 @@ __global__ void __maxnreg__(96)
         // [32eh, 32eh+32) (+ z for eh = 0).  With a partner CTA, a warp on the partner's
         // rows stages its partial block and bulk-copies it into the partner's XCH; a warp on
         // the own rows adds the partner's block once it has landed.
-        const int eh = (warp - kWarpEW) >> 2, quad = warp & 3, t = 32 * quad + lane;
+        const int eh = (warp - L::EW) >> 2, quad = warp & 3, t = 32 * quad + lane;
         const uint32_t tm_row = tm + ((uint32_t)(32 * quad) << 16);
         const int partner = rank ^ 1;
         const bool own_rows = CS == 1 || (quad >> 1) == rank;
@@ -512,11 +540,38 @@ __global__ void __maxnreg__(96)
             if (!bar_wait(&bars.attn_done, ph_attn, &abort_flag, status)) goto ew_out;
             ph_attn ^= 1;
             fence_after_sync();
-            // Causal mask + bf16.  32-key block kb of this half (keys 32kb..32kb+31, kb =
-            // 2eh + b) lies above the diagonal block of this warp's rows (kb > quad: zero),
-            // on it (kb = quad: j <= i) or below it (kb < quad: copied); its bf16 pairs go to
-            // columns 64eh + 16b .., which this thread has already read.
-            {
+            // Causal mask + bf16 of the two 32-key blocks kb = 2 eh + b of this half: a block
+            // above the diagonal block of this warp's rows (kb > quad) is zeros (nothing
+            // loaded), the diagonal block (kb = quad) keeps j <= i, a block below it
+            // (kb < quad) is copied.  Block b's bf16 pairs go to columns 64 eh + 16 b .. + 15,
+            // which this thread read with block 0.
+            if constexpr (NS) {
+                // one block at a time (72-register budget)
+#pragma unroll 1
+                for (int b = 0; b < 2; ++b) {
+                    const int kb = 2 * eh + b;
+                    uint32_t pk[16];
+                    if (kb <= quad) {
+                        float a[32];
+                        tmem_ld16(tm_row + L::T_A + 32 * kb, *reinterpret_cast<float(*)[16]>(&a[0]));
+                        tmem_ld16(tm_row + L::T_A + 32 * kb + 16,
+                                  *reinterpret_cast<float(*)[16]>(&a[16]));
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const int j0 = 32 * kb + 2 * i;
+                            pk[i] = kb < quad ? pack_bf16(a[2 * i], a[2 * i + 1])
+                                              : pack_bf16(j0 <= t ? a[2 * i] : 0.f,
+                                                          j0 + 1 <= t ? a[2 * i + 1] : 0.f);
+                        }
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) pk[i] = 0u;
+                    }
+                    tmem_st16(tm_row + L::T_A + 64 * eh + 16 * b, pk);
+                }
+            } else {
+                // block 1 is loaded while block 0 is stored
                 auto convert = [&](const float (&a)[32], int kb, uint32_t (&pk2)[16]) {
 #pragma unroll
                     for (int i = 0; i < 16; ++i) {
@@ -655,7 +710,7 @@ cudaError_t launch_one(const Problem& p, const void* q, const void* k, const voi
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(BH * splits * CS));
-    cfg.blockDim = dim3(kThreadsTC);
+    cfg.blockDim = dim3(Cfg<NS>::THREADS);
     cfg.dynamicSmemBytes = (size_t)smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
