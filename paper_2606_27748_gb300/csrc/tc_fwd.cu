@@ -134,7 +134,8 @@ template <bool NS, int CS, bool KW>
 __global__ void __launch_bounds__(Cfg<NS>::THREADS, 1)
     tc_fwd_causal_kernel(const __grid_constant__ CUtensorMap tmap_q,
                          const __grid_constant__ CUtensorMap tmap_k,
-                         const __grid_constant__ CUtensorMap tmap_v, int H, int N, int M,
+                         const __grid_constant__ CUtensorMap tmap_v,
+                         const __grid_constant__ CUtensorMap tmap_o, int H, int N, int M,
                          int splits, const float* __restrict__ W1,
                          const float* __restrict__ W2, const float* __restrict__ kw,
                          __nv_bfloat16* __restrict__ out, float* __restrict__ den, int* status)
@@ -669,7 +670,31 @@ __global__ void __launch_bounds__(Cfg<NS>::THREADS, 1)
                     if (lane == 0 && (quad & 1) == 0 && eh == 0 && c + 2 < ce)
                         mbar_arrive_expect_tx(&bars.xch_full[xb], L::XBUF);
                 }
-                if (valid) {
+                if constexpr (CS == 1) {
+                    // This warp's 32 x 32 block of out goes through its own staging tile in
+                    // the (here unused) exchange region and one TMA store: rows written one
+                    // per thread straight to global memory put 32 cache lines in each warp
+                    // store, and the memory-instruction queue they fill also carries the
+                    // issuers' mbarrier waits.  Rows past N are not written by the store.
+                    const uint32_t stg = sb + L::STG + ((warp - L::EW) * 2 + xb) * 2048;
+                    const float inv = 1.f / dn;
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc)
+                        st_shared_v4(stg + swz64(lane, cc),
+                                     pack_bf16(o[8 * cc] * inv, o[8 * cc + 1] * inv),
+                                     pack_bf16(o[8 * cc + 2] * inv, o[8 * cc + 3] * inv),
+                                     pack_bf16(o[8 * cc + 4] * inv, o[8 * cc + 5] * inv),
+                                     pack_bf16(o[8 * cc + 6] * inv, o[8 * cc + 7] * inv));
+                    if (valid && den && eh == 0) den[(size_t)bh * N + t0 + t] = dn / (float)M;
+                    fence_proxy_async();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_3d(&tmap_o, stg, 32 * eh, t0 + 32 * quad, bh);
+                        bulk_commit_group();
+                        bulk_wait_group_read<1>();  // the other staging tile is free again
+                    }
+                    __syncwarp();
+                } else if (valid) {
                     const float inv = 1.f / dn;
                     uint4* dst =
                         reinterpret_cast<uint4*>(out + base + (size_t)(t0 + t) * 64 + 32 * eh);
@@ -683,7 +708,8 @@ __global__ void __launch_bounds__(Cfg<NS>::THREADS, 1)
                 }
             }
         }
-    ew_out:;
+    ew_out:
+        if (CS == 1 && lane == 0) bulk_wait_group<0>();  // stores done before the CTA exits
     }
 
     fence_before_sync();
@@ -700,8 +726,9 @@ cudaError_t launch_one(const Problem& p, const void* q, const void* k, const voi
 {
     CUtensorMap mq, mk, mv;
     const int BH = p.B * p.H;
+    CUtensorMap mo;
     if (!make_act_map(&mq, q, BH, p.N) || !make_act_map(&mk, k, BH, p.N) ||
-        !make_act_map(&mv, v, BH, p.N))
+        !make_act_map(&mv, v, BH, p.N) || !make_out_map32(&mo, out, BH, p.N))
         return cudaErrorInvalidValue;
     const int splits = tc_fwd_splits(p, sm_count());
     auto kern = tc_fwd_causal_kernel<NS, CS, KW>;
@@ -720,7 +747,7 @@ cudaError_t launch_one(const Problem& p, const void* q, const void* k, const voi
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, mq, mk, mv, p.H, p.N, p.M, splits, W1, W2, kw,
+    return cudaLaunchKernelEx(&cfg, kern, mq, mk, mv, mo, p.H, p.N, p.M, splits, W1, W2, kw,
                               (__nv_bfloat16*)out, den, status);
 }
 

@@ -229,6 +229,27 @@ inline bool make_act_map(CUtensorMap* m, const void* base, int BH, int N)
            CUDA_SUCCESS;
 }
 
+// Output tiles of 32 rows x 32 columns of a [BH][N][64] bf16 tensor, 64-byte swizzle: in
+// shared memory row r of a tile is 64 bytes at r * 64, its 16-byte chunk c stored at
+// position c ^ ((r >> 1) & 3) (tile base 512-byte aligned).
+inline bool make_out_map32(CUtensorMap* m, const void* base, int BH, int N)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[3] = {64, (cuuint64_t)N, (cuuint64_t)BH};
+    cuuint64_t strides[2] = {128, (cuuint64_t)N * 128};
+    cuuint32_t box[3] = {32, 32, 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+               box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
+}
+__host__ __device__ __forceinline__ uint32_t swz64(uint32_t row, uint32_t chunk)
+{
+    return row * 64 + ((chunk ^ ((row >> 1) & 3)) << 4);
+}
+
 // One head's frequency rows into shared memory, bf16, K-major with 128-byte swizzle: G
 // groups of P rows (s: P = 64 rows of W1; n: P = 128, U = (W1+W2)/2 then V = (W1-W2)/2),
 // row r of group g = frequency 64 g + r % 64.  8-float pieces by float4 loads, a batch of
