@@ -17,8 +17,8 @@
 // ([cos, sin] instead of M^{-1/2}[cos, sin]): the factor cancels in the output, and only
 // the stored denominator is rescaled (den = den' / M).
 //
-// Warp roles, handshakes on mbarriers (n: 896 threads, FW = 16 feature warps; s: 640
-// threads, FW = 8):
+// Warp roles, handshakes on mbarriers (896 threads with FW = 16 feature warps; the
+// stationary kernel with one CTA per sequence: 640 threads, FW = 8):
 //   warp 0      TMA: q and k chunk tiles (128B swizzle) into shared memory
 //   warp 1      one thread issues the attention MMAs (numerator, QK, state, A V); owns the
 //               tensor-memory allocation
@@ -76,13 +76,15 @@ using namespace tc;
 constexpr int kC = 128;            // tokens per chunk = MMA M
 constexpr int kWarpTMA = 0, kWarpMMA = 1, kWarpFW = 2, kEpiWarps = 8;
 
-template <bool NS>
+template <bool NS, int CS>
 struct Cfg {
     static constexpr int NH = NS ? 2 : 1;  // projections per feature tile (64 columns each)
-    // Feature warps: n 16 (four per lane quadrant, 72 registers a thread), s 8 (two per
-    // quadrant, 96 registers): the s features are cheap enough that the attention and
-    // epilogue chain sets the chunk period, and it runs faster with the larger budget.
-    static constexpr int FW = NS ? 16 : 8;
+    // Feature warps: 16 (four per lane quadrant, 72 registers a thread), except for the
+    // stationary kernel with one CTA per sequence: 8 (two per quadrant, 96 registers).  Its
+    // features are cheap enough that the attention and epilogue chain sets the chunk
+    // period, and that runs faster with the larger budget (measured: 16 warps 0.105 ms,
+    // 8 warps 0.094 ms on s_causal B8 H12 N4096; the pair kernels gain from 16).
+    static constexpr int FW = (NS || CS > 1) ? 16 : 8;
     static constexpr int EW = kWarpFW + FW;        // first epilogue warp
     static constexpr int PROJ = EW + kEpiWarps;    // projection MMA issuer
     static constexpr int TMAV = PROJ + 1;          // v tiles
@@ -131,7 +133,7 @@ __device__ __forceinline__ int segment_bound(int nch, int splits, int j)
 // NS: nonstationary features; CS: CTAs per cluster = frequency groups (M / 64); KW: key
 // weights of the norm prefactor given (a compile-time switch: the plain kernel is unchanged).
 template <bool NS, int CS, bool KW>
-__global__ void __launch_bounds__(Cfg<NS>::THREADS, 1)
+__global__ void __launch_bounds__(Cfg<NS, CS>::THREADS, 1)
     tc_fwd_causal_kernel(const __grid_constant__ CUtensorMap tmap_q,
                          const __grid_constant__ CUtensorMap tmap_k,
                          const __grid_constant__ CUtensorMap tmap_v,
@@ -140,7 +142,7 @@ __global__ void __launch_bounds__(Cfg<NS>::THREADS, 1)
                          const float* __restrict__ W2, const float* __restrict__ kw,
                          __nv_bfloat16* __restrict__ out, float* __restrict__ den, int* status)
 {
-    using L = Cfg<NS>;
+    using L = Cfg<NS, CS>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const uint32_t sb = smem_u32(sm);
@@ -546,7 +548,7 @@ __global__ void __launch_bounds__(Cfg<NS>::THREADS, 1)
             // loaded), the diagonal block (kb = quad) keeps j <= i, a block below it
             // (kb < quad) is copied.  Block b's bf16 pairs go to columns 64 eh + 16 b .. + 15,
             // which this thread read with block 0.
-            if constexpr (NS) {
+            if constexpr (L::FW == 16) {
                 // one block at a time (72-register budget)
 #pragma unroll 1
                 for (int b = 0; b < 2; ++b) {
@@ -732,12 +734,12 @@ cudaError_t launch_one(const Problem& p, const void* q, const void* k, const voi
         return cudaErrorInvalidValue;
     const int splits = tc_fwd_splits(p, sm_count());
     auto kern = tc_fwd_causal_kernel<NS, CS, KW>;
-    const int smem = (int)Cfg<NS>::BYTES + 1024;
+    const int smem = (int)Cfg<NS, CS>::BYTES + 1024;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(BH * splits * CS));
-    cfg.blockDim = dim3(Cfg<NS>::THREADS);
+    cfg.blockDim = dim3(Cfg<NS, CS>::THREADS);
     cfg.dynamicSmemBytes = (size_t)smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
